@@ -1,0 +1,290 @@
+"""fp64 CPU oracle for block-causal attention (test infrastructure only).
+
+This module is the checker, not the product: only ``tests/``, the package's
+``smoke()`` and the benchmark's CPU-baseline / reference arm may import it.
+It shares no code with the CUDA path.
+
+What it computes (Sec. 3.2, block-causal self-attention): the token sequence
+is cut into temporally ordered chunks of ``T`` tokens; a query attends to every
+key of its own chunk (bidirectionally) and of all earlier chunks (strictly
+causal across chunks).  With chunk(i) = floor(i / T):
+
+    visible(i, j)  <=>  chunk(j) <= chunk(i)
+    s_ij   = scale * <q_i, k_j>                       (visible pairs only)
+    LSE_i  = ln sum_{j visible} exp(s_ij)
+    P_ij   = exp(s_ij - LSE_i)   (0 where not visible)
+    O_i    = sum_j P_ij v_j
+
+The paper does not write the attention formula itself; the above is standard
+scaled dot-product attention restricted by the chunk mask.  The backward
+(training is bf16 mixed precision, Sec. 4.1) is the analytic gradient:
+
+    dV_j  = sum_i P_ij dO_i
+    dP_ij = <dO_i, v_j>
+    D_i   = <dO_i, O_i>
+    dS_ij = P_ij (dP_ij - D_i)
+    dQ_i  = scale * sum_j dS_ij k_j
+    dK_j  = scale * sum_i dS_ij q_i
+
+Streaming (Sec. 3.5): in-flight chunks attend to the committed history (the
+rolling KV cache, a FIFO of finished chunks) and to preceding in-flight chunks
+under the same chunk-causal rule.  Committed K/V are written once and never
+change.
+
+All arithmetic is fp64 (inputs are the bf16 tensors the GPU sees, widened).
+Three forms of the forward are kept and cross-checked: scalar loops (tiny
+shapes), a dense N x N masked matrix, and a row-block form that builds, per
+query chunk c, the [T, (c+1)T] block of visible scores (which is the mask).
+"""
+from __future__ import annotations
+
+import math
+from typing import List, Sequence, Tuple
+
+import torch
+
+F64 = torch.float64
+
+
+def chunk_of(i: int, T: int) -> int:
+    """Chunk index of token i for chunks of T tokens."""
+    return i // T
+
+
+def block_causal_mask(N: int, T: int) -> torch.Tensor:
+    """Boolean [N, N]: True where query i may attend key j (Sec. 3.2)."""
+    idx = torch.arange(N)
+    return (idx.view(1, N) // T) <= (idx.view(N, 1) // T)
+
+
+# --------------------------------------------------------------------------
+# form (i): scalar loops, one head, python floats; tiny shapes only
+# --------------------------------------------------------------------------
+
+def fwd_loops(q: Sequence[Sequence[float]], k: Sequence[Sequence[float]],
+              v: Sequence[Sequence[float]], T: int, scale: float
+              ) -> Tuple[List[List[float]], List[float]]:
+    """Forward of one head by explicit loops over i, j and the feature index."""
+    N = len(q)
+    d = len(q[0])
+    dv = len(v[0])
+    out, lse = [], []
+    for i in range(N):
+        scores = []
+        for j in range(N):
+            if chunk_of(j, T) <= chunk_of(i, T):
+                dot = 0.0
+                for x in range(d):
+                    dot += q[i][x] * k[j][x]
+                scores.append((j, scale * dot))
+        assert scores, "a query always sees its own chunk"
+        top = max(s for _, s in scores)
+        total = 0.0
+        for _, s in scores:
+            total += math.exp(s - top)
+        l_i = top + math.log(total)
+        row = [0.0] * dv
+        for j, s in scores:
+            p = math.exp(s - l_i)
+            for x in range(dv):
+                row[x] += p * v[j][x]
+        out.append(row)
+        lse.append(l_i)
+    return out, lse
+
+
+# --------------------------------------------------------------------------
+# form (ii): dense masked matrices, [..., N, d]
+# --------------------------------------------------------------------------
+
+def probs_dense(q: torch.Tensor, k: torch.Tensor, T: int, scale: float) -> torch.Tensor:
+    """P [..., N, N] with zeros at masked positions (small N only)."""
+    q = q.to(F64)
+    k = k.to(F64)
+    N = q.shape[-2]
+    s = scale * torch.matmul(q, k.transpose(-1, -2))
+    s = s.masked_fill(~block_causal_mask(N, T), float("-inf"))
+    lse = _row_lse(s)
+    return torch.exp(s - lse.unsqueeze(-1))
+
+
+def fwd_dense(q: torch.Tensor, k: torch.Tensor, v: torch.Tensor, T: int,
+              scale: float) -> Tuple[torch.Tensor, torch.Tensor]:
+    """(O, LSE) through the explicit N x N mask."""
+    q, k, v = q.to(F64), k.to(F64), v.to(F64)
+    N = q.shape[-2]
+    s = scale * torch.matmul(q, k.transpose(-1, -2))
+    s = s.masked_fill(~block_causal_mask(N, T), float("-inf"))
+    lse = _row_lse(s)
+    p = torch.exp(s - lse.unsqueeze(-1))
+    return torch.matmul(p, v), lse
+
+
+def bwd_dense(q, k, v, do, T: int, scale: float):
+    """(dQ, dK, dV) through the explicit N x N mask."""
+    q, k, v, do = (t.to(F64) for t in (q, k, v, do))
+    p = probs_dense(q, k, T, scale)
+    o = torch.matmul(p, v)
+    dv = torch.matmul(p.transpose(-1, -2), do)
+    dp = torch.matmul(do, v.transpose(-1, -2))
+    D = (do * o).sum(-1, keepdim=True)
+    ds = p * (dp - D)
+    dq = scale * torch.matmul(ds, k)
+    dk = scale * torch.matmul(ds.transpose(-1, -2), q)
+    return dq, dk, dv
+
+
+def _row_lse(s: torch.Tensor) -> torch.Tensor:
+    """ln sum_j exp(s_j) over the last axis; the row maximum is factored out
+    (ln sum exp(s) = m + ln sum exp(s - m)) so that exp never overflows."""
+    m = s.max(dim=-1, keepdim=True).values
+    return (m + torch.log(torch.exp(s - m).sum(dim=-1, keepdim=True))).squeeze(-1)
+
+
+# --------------------------------------------------------------------------
+# form (iii): row blocks per query chunk, [B, H, N, d]
+# --------------------------------------------------------------------------
+
+def fwd(q: torch.Tensor, k: torch.Tensor, v: torch.Tensor, T: int,
+        scale: float) -> Tuple[torch.Tensor, torch.Tensor]:
+    """(O [B,H,N,dv], LSE [B,H,N]) for Q, K, V [B,H,N,d]; N a multiple of T.
+
+    Query chunk c sees keys [0, (c+1) T): its score block is that slice, so the
+    mask is the slicing itself.
+    """
+    q, k, v = q.to(F64), k.to(F64), v.to(F64)
+    B, H, N, _ = q.shape
+    assert N % T == 0, "sequence length must be a whole number of chunks"
+    n = N // T
+    o = torch.empty(B, H, N, v.shape[-1], dtype=F64)
+    lse = torch.empty(B, H, N, dtype=F64)
+    for b in range(B):
+        for h in range(H):
+            for c in range(n):
+                rows = slice(c * T, (c + 1) * T)
+                keys = slice(0, (c + 1) * T)
+                s = scale * (q[b, h, rows] @ k[b, h, keys].T)
+                l_c = _row_lse(s)
+                p = torch.exp(s - l_c.unsqueeze(-1))
+                o[b, h, rows] = p @ v[b, h, keys]
+                lse[b, h, rows] = l_c
+    return o, lse
+
+
+def bwd(q: torch.Tensor, k: torch.Tensor, v: torch.Tensor, do: torch.Tensor,
+        T: int, scale: float) -> Tuple[torch.Tensor, torch.Tensor, torch.Tensor]:
+    """(dQ, dK, dV) of sum(O * dO) for Q, K, V, dO [B,H,N,d]; P is recomputed."""
+    q, k, v, do = (t.to(F64) for t in (q, k, v, do))
+    B, H, N, _ = q.shape
+    assert N % T == 0
+    n = N // T
+    dq = torch.zeros_like(q)
+    dk = torch.zeros_like(k)
+    dv = torch.zeros_like(v)
+    for b in range(B):
+        for h in range(H):
+            for c in range(n):
+                rows = slice(c * T, (c + 1) * T)
+                keys = slice(0, (c + 1) * T)
+                qc, kc, vc, doc = q[b, h, rows], k[b, h, keys], v[b, h, keys], do[b, h, rows]
+                s = scale * (qc @ kc.T)
+                p = torch.exp(s - _row_lse(s).unsqueeze(-1))
+                oc = p @ vc
+                dv[b, h, keys] += p.T @ doc
+                dp = doc @ vc.T
+                D = (doc * oc).sum(-1, keepdim=True)
+                ds = p * (dp - D)
+                dq[b, h, rows] = scale * (ds @ kc)
+                dk[b, h, keys] += scale * (ds.T @ qc)
+    return dq, dk, dv
+
+
+def fwd_rows(q: torch.Tensor, k: torch.Tensor, v: torch.Tensor, T: int,
+             scale: float, rows: Sequence[int]) -> Tuple[torch.Tensor, torch.Tensor]:
+    """(O, LSE) of selected query rows of one head (Q,K,V [N,d]), row by row."""
+    q, k, v = q.to(F64), k.to(F64), v.to(F64)
+    outs, lses = [], []
+    for i in rows:
+        end = (chunk_of(i, T) + 1) * T
+        s = scale * (k[:end] @ q[i])
+        l_i = _row_lse(s.unsqueeze(0))[0]
+        outs.append(torch.exp(s - l_i) @ v[:end])
+        lses.append(l_i)
+    return torch.stack(outs), torch.stack(lses)
+
+
+# --------------------------------------------------------------------------
+# rolling KV cache (Sec. 3.5): ring of committed chunks + in-flight chunks
+# --------------------------------------------------------------------------
+
+def ring_logical(ring: torch.Tensor, cap: int, head: int, length: int) -> torch.Tensor:
+    """Cached rows in logical (oldest first) order: logical t -> physical (head+t) mod cap.
+
+    ``ring`` is [B, H, cap, d]; the result is [B, H, length, d].
+    """
+    assert ring.shape[-2] == cap and 0 <= head < cap and 0 <= length <= cap
+    idx = torch.tensor([(head + t) % cap for t in range(length)], dtype=torch.long)
+    return ring.index_select(-2, idx)
+
+
+def cache_fwd(q: torch.Tensor, k_new: torch.Tensor, v_new: torch.Tensor,
+              k_ring: torch.Tensor, v_ring: torch.Tensor, cap: int, head: int,
+              length: int, T: int, scale: float) -> Tuple[torch.Tensor, torch.Tensor]:
+    """(O, LSE) of W in-flight chunks (Q, K_new, V_new [B,H,W*T,d]).
+
+    In-flight chunk j sees every cached token (the committed history, in
+    logical order) and in-flight chunks 0..j (Sec. 3.5: a future chunk attends
+    only to the committed history and to preceding chunks of the active window,
+    itself included as in Sec. 3.2).
+    """
+    q, k_new, v_new = q.to(F64), k_new.to(F64), v_new.to(F64)
+    kc = ring_logical(k_ring.to(F64), cap, head, length)
+    vc = ring_logical(v_ring.to(F64), cap, head, length)
+    keys = torch.cat([kc, k_new], dim=-2)
+    vals = torch.cat([vc, v_new], dim=-2)
+    B, H, M, _ = q.shape
+    assert M % T == 0
+    W = M // T
+    o = torch.empty(B, H, M, v_new.shape[-1], dtype=F64)
+    lse = torch.empty(B, H, M, dtype=F64)
+    for b in range(B):
+        for h in range(H):
+            for j in range(W):
+                rows = slice(j * T, (j + 1) * T)
+                visible = slice(0, length + (j + 1) * T)
+                s = scale * (q[b, h, rows] @ keys[b, h, visible].T)
+                l_j = _row_lse(s)
+                o[b, h, rows] = torch.exp(s - l_j.unsqueeze(-1)) @ vals[b, h, visible]
+                lse[b, h, rows] = l_j
+    return o, lse
+
+
+def cache_commit(k_ring: torch.Tensor, v_ring: torch.Tensor, cap: int, slot: int,
+                 k_src: torch.Tensor, v_src: torch.Tensor) -> Tuple[torch.Tensor, torch.Tensor]:
+    """New ring contents after writing ``rows`` tokens at physical rows (slot+r) mod cap.
+
+    Returns copies; the inputs are not modified.
+    """
+    rows = k_src.shape[-2]
+    assert 0 <= slot < cap and rows <= cap
+    k_out, v_out = k_ring.clone(), v_ring.clone()
+    for r in range(rows):
+        p = (slot + r) % cap
+        k_out[..., p, :] = k_src[..., r, :]
+        v_out[..., p, :] = v_src[..., r, :]
+    return k_out, v_out
+
+
+def ring_advance(cap: int, head: int, length: int, rows: int) -> Tuple[int, int, int]:
+    """FIFO bookkeeping for committing ``rows`` tokens (Sec. 3.5).
+
+    Returns (slot, new_head, new_length): the new rows go after the newest
+    cached token, at physical (head + length) mod cap; when the ring would
+    overflow, the oldest rows are evicted by moving ``head`` forward.
+    """
+    slot = (head + length) % cap
+    total = length + rows
+    if total <= cap:
+        return slot, head, total
+    evicted = total - cap
+    return slot, (head + evicted) % cap, cap
