@@ -1,0 +1,589 @@
+#!/usr/bin/env python
+"""Benchmark of the block-causal attention hot path on GB300.
+
+One step = block-causal attention forward + backward (every stage of the
+training path) over the workload B=2, H=12, d=64, 16 chunks x 880 tokens
+(N = 14080), bf16, synthetic N(0,1) inputs.  `value` is TFLOP/s counted over
+unmasked (query, key) pairs only: fwd 4*d*pairs + bwd 10*d*pairs.
+
+Also reported in the same JSON line: the roofline of the dominant kernel
+(backward key-tile kernel, timed with CUDA events around it), an end-to-end
+number through the C ABI with pinned host buffers, the fp64 oracle on the
+host cores (cpu_baseline), and secondary workloads (forward only, the
+d=128 peaky config, the rolling-KV-cache streaming step and the pipelined
+4-chunk window).
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+
+Under torchrun (N > 1) every rank runs its own batch of the same workload
+(independent problems: weak scaling, no collective on the data path); the
+timed region is bracketed by barriers and the max over ranks is taken.
+"""
+from __future__ import annotations
+
+import argparse
+import csv
+import io
+import json
+import math
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+import torch  # noqa: E402
+
+from workloads import CACHE_CONFIGS, TRAIN_CONFIGS, gen_cache, gen_train  # noqa: E402
+
+METRIC = "block-causal attn TFLOP/s fwd+bwd (% GB300 BF16 peak); rolling-KV chunk latency µs"
+WORKLOAD = "train_b12_d64"
+L2_FLUSH_BYTES = 256 << 20
+FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
+
+
+# ------------------------------------------------------------------ accounting
+
+def train_pairs(cfg) -> int:
+    """Unmasked (query, key) pairs: T^2 n (n+1) / 2 per head."""
+    return cfg.B * cfg.H * cfg.T * cfg.T * cfg.n_chunks * (cfg.n_chunks + 1) // 2
+
+
+def cache_pairs(cfg) -> int:
+    """Each of the W*T queries sees `length` cached keys plus its causal share
+    of the in-flight keys."""
+    inflight = cfg.T * cfg.T * cfg.W * (cfg.W + 1) // 2
+    return cfg.B * cfg.H * (cfg.W * cfg.T * cfg.length + inflight)
+
+
+def fwd_flops(pairs: int, d: int) -> float:
+    return 4.0 * d * pairs
+
+
+def bwd_flops(pairs: int, d: int) -> float:
+    return 10.0 * d * pairs
+
+
+def bwd_main_bytes(cfg) -> float:
+    """Algorithmic bytes of the backward key-tile kernel: read Q, K, V, dO
+    (bf16) and the two fp32 row vectors; write dK, dV (bf16); one fp32
+    read-modify-write of the dQ accumulator."""
+    e = cfg.B * cfg.H * cfg.N * cfg.d
+    rows = cfg.B * cfg.H * cfg.N
+    return 2.0 * 4 * e + 4.0 * 2 * rows + 2.0 * 2 * e + 8.0 * e
+
+
+def cache_bytes(cfg) -> float:
+    """Read the cached K/V once, the in-flight Q/K/V, write O and LSE, and the
+    commit (read + write of one chunk's K and V)."""
+    e_new = cfg.B * cfg.H * cfg.W * cfg.T * cfg.d
+    e_ring = cfg.B * cfg.H * cfg.length * cfg.d
+    commit = 2.0 * 2 * 2 * cfg.B * cfg.H * cfg.T * cfg.d
+    return 2.0 * 2 * e_ring + 2.0 * 3 * e_new + 2.0 * e_new + 4.0 * cfg.B * cfg.H * cfg.W * cfg.T + commit
+
+
+def load_peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(path) as f:
+            p = json.load(f)
+        return {"hbm_gbs": float(p["hbm_gbs"]), "bf16_tflops": float(p["bf16_tflops"]),
+                "bf16_tflops_sustained": float(p.get("bf16_tflops_sustained", p["bf16_tflops"])),
+                "source": "measured"}
+    except (OSError, KeyError, ValueError):
+        return {**FALLBACK_PEAKS, "source": "fallback"}
+
+
+# ------------------------------------------------------------------ distributed helpers
+
+def dist_env():
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return world, rank, local
+
+
+def init_dist(world: int, backend: str):
+    if world > 1 and not torch.distributed.is_initialized():
+        torch.distributed.init_process_group(backend=backend)
+
+
+def barrier(world: int):
+    if world > 1:
+        torch.distributed.barrier()
+
+
+def max_over_ranks(x: float, world: int, device=None) -> float:
+    if world == 1:
+        return x
+    t = torch.tensor([x], dtype=torch.float64, device=device)
+    torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+    return float(t.item())
+
+
+def aggregate_rate(units_per_rank: float, world: int, seconds_max: float) -> float:
+    """Whole-job throughput: units processed by all ranks / slowest rank's time."""
+    return units_per_rank * world / seconds_max
+
+
+# ------------------------------------------------------------------ clocks
+
+CLOCK_FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+                "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+                "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+
+class ClockSampler:
+    """nvidia-smi sampling (200 ms) while the timed region runs."""
+
+    def __init__(self, gpu_index: int):
+        self.gpu_index = gpu_index
+        self.proc = None
+
+    def __enter__(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.gpu_index), f"--query-gpu={CLOCK_FIELDS}",
+                 "--format=csv,noheader,nounits", "-lms", "200"],
+                stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except OSError:
+            self.proc = None
+        return self
+
+    def __exit__(self, *exc):
+        self.text = ""
+        if self.proc is not None:
+            time.sleep(0.25)
+            self.proc.terminate()
+            try:
+                self.text, _ = self.proc.communicate(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+                self.text = ""
+        return False
+
+    def summary(self):
+        rows = [r for r in csv.reader(io.StringIO(getattr(self, "text", ""))) if len(r) >= 9]
+        if not rows:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["unsampled"], "samples": 0}
+        sm = [float(r[1]) for r in rows if r[1].strip().replace(".", "").isdigit()]
+        mx = [float(r[2]) for r in rows if r[2].strip().replace(".", "").isdigit()]
+        names = ("hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap")
+        reasons = sorted({n for r in rows for n, v in zip(names, r[5:9]) if "Active" == v.strip()})
+        power = [float(r[3]) for r in rows if r[3].strip().replace(".", "").isdigit()]
+        return {"sm_mhz": statistics.median(sm) if sm else None,
+                "sm_max_mhz": max(mx) if mx else None, "reasons": reasons,
+                "samples": len(rows), "power_w_max": max(power) if power else None}
+
+
+# ------------------------------------------------------------------ CPU baseline (oracle)
+
+def oracle_sample(seconds: float, rank_seed: int = 0, max_heads: int = 24):
+    """fp64 oracle fwd+bwd over whole (b, h) heads of the workload until
+    `seconds` have passed (at least one head).  Returns (TFLOP/s, heads, s)."""
+    import oracle
+    cfg = TRAIN_CONFIGS[WORKLOAD]
+    x = gen_train(cfg)
+    per_head = (fwd_flops(train_pairs(cfg), cfg.d) + bwd_flops(train_pairs(cfg), cfg.d)) / (cfg.B * cfg.H)
+    t0 = time.perf_counter()
+    heads = 0
+    for idx in range(max_heads):
+        b, h = divmod(idx % (cfg.B * cfg.H), cfg.H)
+        sl = (slice(b, b + 1), slice(h, h + 1))
+        q, k, v, do = (x[n][sl] for n in ("q", "k", "v", "do"))
+        oracle.fwd(q, k, v, cfg.T, cfg.scale)
+        oracle.bwd(q, k, v, do, cfg.T, cfg.scale)
+        heads += 1
+        if time.perf_counter() - t0 >= seconds:
+            break
+    dt = time.perf_counter() - t0
+    return per_head * heads / dt / 1e12, heads, dt
+
+
+def cpu_cores() -> int:
+    try:
+        return len(os.sched_getaffinity(0))
+    except AttributeError:
+        return os.cpu_count() or 1
+
+
+# ------------------------------------------------------------------ GPU timing helpers
+
+class Events:
+    def __init__(self):
+        self.a = torch.cuda.Event(enable_timing=True)
+        self.b = torch.cuda.Event(enable_timing=True)
+
+    def start(self):
+        self.a.record()
+
+    def stop(self):
+        self.b.record()
+
+    def ms(self) -> float:
+        return self.a.elapsed_time(self.b)
+
+
+def time_repeated(fn, reps: int, warmup: int = 3, flush=None):
+    for _ in range(warmup):
+        fn()
+    torch.cuda.synchronize()
+    ts = []
+    for _ in range(reps):
+        if flush is not None:
+            flush()
+        e = Events()
+        e.start()
+        fn()
+        e.stop()
+        ts.append(e)
+    torch.cuda.synchronize()
+    return [e.ms() for e in ts]
+
+
+# ------------------------------------------------------------------ our arm
+
+def run_ours(args):
+    import paper_2608_01127_gb300 as mw
+
+    world, rank, local = dist_env()
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    init_dist(world, "nccl")
+    peaks = load_peaks()
+
+    cfg = TRAIN_CONFIGS[WORKLOAD]
+    x = gen_train(cfg) if rank == 0 else gen_train(_reseeded(cfg, rank))
+    q, k, v, do = (x[n].to(dev) for n in ("q", "k", "v", "do"))
+    o = torch.empty_like(q)
+    lse = torch.empty(cfg.B, cfg.H, cfg.N, dtype=torch.float32, device=dev)
+    dq, dk, dv = torch.empty_like(q), torch.empty_like(k), torch.empty_like(v)
+    ws = torch.empty(mw.mw_bca_bwd_workspace_size(cfg.B, cfg.H, cfg.n_chunks, cfg.T, cfg.d),
+                     dtype=torch.uint8, device=dev)
+    flush_buf = torch.empty(L2_FLUSH_BYTES, dtype=torch.uint8, device=dev)
+    lib = mw.library()
+    sc = cfg.scale
+
+    def fwd():
+        mw._check(lib.mw_bca_fwd(q.data_ptr(), k.data_ptr(), v.data_ptr(), o.data_ptr(),
+                                 lse.data_ptr(), cfg.B, cfg.H, cfg.n_chunks, cfg.T, cfg.d, sc,
+                                 torch.cuda.current_stream().cuda_stream))
+
+    def bwd_stage(stage):
+        mw._check(lib.mw_bca_bwd_stage(stage, q.data_ptr(), k.data_ptr(), v.data_ptr(),
+                                       o.data_ptr(), lse.data_ptr(), do.data_ptr(), dq.data_ptr(),
+                                       dk.data_ptr(), dv.data_ptr(), ws.data_ptr(), ws.numel(),
+                                       cfg.B, cfg.H, cfg.n_chunks, cfg.T, cfg.d, sc,
+                                       torch.cuda.current_stream().cuda_stream))
+
+    launches_per_step = 4  # forward kernel + backward pre / main / post
+    pairs = train_pairs(cfg)
+    step_flops = fwd_flops(pairs, cfg.d) + bwd_flops(pairs, cfg.d)
+
+    for _ in range(args.warmup):
+        fwd()
+        bwd_stage(0)
+    torch.cuda.synchronize()
+    barrier(world)
+    step_ev, main_ev, fwd_ev = [], [], []
+    with ClockSampler(local) as clk:
+        barrier(world)
+        torch.cuda.synchronize()
+        for _ in range(args.steps):
+            flush_buf.zero_()          # L2 flush between steps, outside the events
+            s, f, m = Events(), Events(), Events()
+            s.start()
+            f.start()
+            fwd()
+            f.stop()
+            bwd_stage(1)
+            m.start()
+            bwd_stage(2)
+            m.stop()
+            bwd_stage(3)
+            s.stop()
+            step_ev.append(s)
+            main_ev.append(m)
+            fwd_ev.append(f)
+        torch.cuda.synchronize()
+        barrier(world)
+    step_ms = [e.ms() for e in step_ev]
+    total_ms = max_over_ranks(sum(step_ms), world, dev)
+    value = aggregate_rate(step_flops * args.steps, world, total_ms / 1e3) / 1e12
+    ms_per_step = total_ms / args.steps
+    main_ms = statistics.mean(e.ms() for e in main_ev)
+    fwd_ms = statistics.mean(e.ms() for e in fwd_ev)
+    main_flops = bwd_flops(pairs, cfg.d)
+    achieved = main_flops / (main_ms / 1e3) / 1e12
+    assert mw.mw_device_status() == 0, "a kernel reported a timeout"
+
+    out = {
+        "metric": METRIC, "value": round(value, 2), "unit": "TFLOP/s", "n_gpus": world,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(ms_per_step, 4),
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
+        "data": "synthetic",
+        "config": {"workload": f"{WORKLOAD}: block-causal attention fwd+bwd, B={cfg.B} H={cfg.H} "
+                               f"d={cfg.d}, {cfg.n_chunks} chunks x {cfg.T} tokens (N={cfg.N})",
+                   "global_batch": cfg.B * world, "seq_len": cfg.N, "parallelism": f"dp{world}",
+                   "flops_per_step": step_flops, "unmasked_pairs": pairs,
+                   "l2": "256 MiB buffer written between timed steps (outside the events)"},
+        "frac_of_bf16_peak": round(value / world / peaks["bf16_tflops"], 4),
+        "roofline": {"kernel": "bca_bwd_kernel<64> (backward key-tile kernel)", "bound": "tensor",
+                     "achieved": round(achieved, 2), "peak": peaks["bf16_tflops"],
+                     "peak_source": peaks["source"] + " bf16 burst", "unit": "TFLOP/s",
+                     "frac": round(achieved / peaks["bf16_tflops"], 4),
+                     "traffic": profiled_traffic("bca_bwd_kernel<64>", WORKLOAD),
+                     "algorithmic_bytes": bwd_main_bytes(cfg),
+                     "ms_per_launch": round(main_ms, 4)},
+        "fwd": {"ms": round(fwd_ms, 4),
+                "tflops": round(fwd_flops(pairs, cfg.d) / (fwd_ms / 1e3) / 1e12, 2)},
+        "gpu_launches": launches_per_step * args.steps,
+    }
+    out["clocks"] = clk.summary()
+    out["e2e"] = run_e2e(mw, cfg, dev, args, world, step_flops)
+    if rank == 0 and world == 1 and not args.no_extras:
+        out["extra"] = run_extras(mw, dev, peaks)
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        tf, heads, dt = oracle_sample(args.cpu_seconds)
+        out["cpu_baseline"] = {"value": round(tf, 6), "unit": "TFLOP/s", "cores": torch.get_num_threads(),
+                               "host_cores": cpu_cores(), "kind": "oracle",
+                               "sample": f"fp64 oracle fwd+bwd of {heads} of {cfg.B * cfg.H} (b,h) heads "
+                                         f"of {WORKLOAD} ({dt:.1f} s)"}
+    if rank == 0:
+        print(json.dumps(out), flush=True)
+    if world > 1:
+        torch.distributed.destroy_process_group()
+
+
+def _reseeded(cfg, rank):
+    import dataclasses
+    return dataclasses.replace(cfg, seed=cfg.seed + 1000 * rank)
+
+
+def run_e2e(mw, cfg, dev, args, world, step_flops):
+    """Same step through the public API with pinned host buffers: H2D of
+    Q, K, V, dO and D2H of O, LSE, dQ, dK, dV inside the timed region."""
+    x = gen_train(cfg)
+    host_in = [x[n].pin_memory() for n in ("q", "k", "v", "do")]
+    host_out = [torch.empty_like(host_in[0]).pin_memory() for _ in range(4)]
+    host_lse = torch.empty(cfg.B, cfg.H, cfg.N, dtype=torch.float32).pin_memory()
+    dev_in = [torch.empty_like(t, device=dev) for t in host_in]
+    ws = torch.empty(mw.mw_bca_bwd_workspace_size(cfg.B, cfg.H, cfg.n_chunks, cfg.T, cfg.d),
+                     dtype=torch.uint8, device=dev)
+
+    def step():
+        for d_, h_ in zip(dev_in, host_in):
+            d_.copy_(h_, non_blocking=True)
+        q, k, v, do = dev_in
+        o, lse = mw.mw_bca_fwd(q, k, v, cfg.T, cfg.scale)
+        dq, dk, dv = mw.mw_bca_bwd(q, k, v, o, lse, do, cfg.T, cfg.scale, workspace=ws)
+        for h_, d_ in zip(host_out, (o, dq, dk, dv)):
+            h_.copy_(d_, non_blocking=True)
+        host_lse.copy_(lse, non_blocking=True)
+
+    reps = max(3, min(args.steps, 20))
+    for _ in range(2):
+        step()
+    torch.cuda.synchronize()
+    barrier(world)
+    t0 = time.perf_counter()
+    e = Events()
+    e.start()
+    for _ in range(reps):
+        step()
+    e.stop()
+    torch.cuda.synchronize()
+    ms = max_over_ranks(e.ms(), world, dev)
+    h2d = sum(t.numel() * t.element_size() for t in host_in)
+    d2h = sum(t.numel() * t.element_size() for t in host_out) + host_lse.numel() * 4
+    return {"value": round(aggregate_rate(step_flops * reps, world, ms / 1e3) / 1e12, 2),
+            "unit": "TFLOP/s", "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
+            "ms_per_step": round(ms / reps, 4),
+            "wall_ms_per_step": round((time.perf_counter() - t0) * 1e3 / reps, 4)}
+
+
+def run_extras(mw, dev, peaks):
+    flush_buf = torch.empty(L2_FLUSH_BYTES, dtype=torch.uint8, device=dev)
+    flush = flush_buf.zero_
+    extra = {}
+    # forward / backward of the d=128 peaky workload
+    cfg = TRAIN_CONFIGS["train_h16_d128_peaky"]
+    x = gen_train(cfg)
+    q, k, v, do = (x[n].to(dev) for n in ("q", "k", "v", "do"))
+    o, lse = mw.mw_bca_fwd(q, k, v, cfg.T, cfg.scale)
+    ws = torch.empty(mw.mw_bca_bwd_workspace_size(cfg.B, cfg.H, cfg.n_chunks, cfg.T, cfg.d),
+                     dtype=torch.uint8, device=dev)
+    grads = tuple(torch.empty_like(q) for _ in range(3))
+    pairs = train_pairs(cfg)
+    tf = time_repeated(lambda: mw.mw_bca_fwd(q, k, v, cfg.T, cfg.scale), 10, flush=flush)
+    tb = time_repeated(lambda: mw.mw_bca_bwd(q, k, v, o, lse, do, cfg.T, cfg.scale, workspace=ws,
+                                             out=grads), 10, flush=flush)
+    fm, bm = statistics.median(tf), statistics.median(tb)
+    extra["train_h16_d128_peaky"] = {
+        "fwd_ms": round(fm, 4), "bwd_ms": round(bm, 4),
+        "fwd_tflops": round(fwd_flops(pairs, cfg.d) / fm / 1e9, 2),
+        "fwd_bwd_tflops": round((fwd_flops(pairs, cfg.d) + bwd_flops(pairs, cfg.d)) / (fm + bm) / 1e9, 2)}
+    del q, k, v, do, o, lse, ws, grads
+    extra["rolling_cache"] = bench_rolling(mw, dev, peaks)
+    extra["pipelined"] = bench_pipelined(mw, dev, peaks, flush)
+    return extra
+
+
+def _cache_roofline(cfg, us, peaks):
+    flops = fwd_flops(cache_pairs(cfg), cfg.d)
+    nbytes = cache_bytes(cfg)
+    t_tensor = flops / (peaks["bf16_tflops"] * 1e12)
+    t_hbm = nbytes / (peaks["hbm_gbs"] * 1e9)
+    s = us / 1e6
+    return {"tflops": round(flops / s / 1e12, 2), "frac_tensor": round(t_tensor / s, 4),
+            "gbs_algorithmic": round(nbytes / s / 1e9, 1), "frac_hbm": round(t_hbm / s, 4),
+            "roofline_frac": round(max(t_tensor, t_hbm) / s, 4),
+            "bound": "tensor" if t_tensor >= t_hbm else "hbm"}
+
+
+def bench_rolling(mw, dev, peaks):
+    """64 streaming steps: cache forward of one 880-token chunk against the
+    8-chunk ring, then commit of that chunk (FIFO eviction); per-step latency."""
+    cfg = CACHE_CONFIGS["rolling_cache"]
+    x = gen_cache(cfg)
+    kr, vr = x["k_ring"].to(dev), x["v_ring"].to(dev)
+    qs, ks, vs = x["q"].to(dev), x["k_new"].to(dev), x["v_new"].to(dev)
+    ws_bytes = mw.mw_bca_cache_workspace_size(cfg.B, cfg.H, cfg.W, cfg.T, cfg.d, cfg.length)
+    ws = torch.empty(max(ws_bytes, 1), dtype=torch.uint8, device=dev)
+    o = torch.empty_like(qs[0])
+    plan = []
+    ring = mw.RingState(cfg.cap, cfg.head, cfg.length)
+    for _ in range(cfg.steps):
+        head, length = ring.head, ring.length
+        plan.append((head, length, ring.commit(cfg.T)))
+
+    def step(s):
+        h, ln, slot = plan[s]
+        mw.mw_bca_cache_fwd(qs[s], ks[s], vs[s], kr, vr, h, ln, cfg.T, cfg.scale, need_lse=False,
+                            workspace=ws, out=o)
+        mw.mw_bca_cache_commit(kr, vr, slot, ks[s], vs[s])
+
+    for s in range(3):
+        step(s)
+    torch.cuda.synchronize()
+    evs = []
+    for s in range(cfg.steps):
+        e = Events()
+        e.start()
+        step(s)
+        e.stop()
+        evs.append(e)
+    torch.cuda.synchronize()
+    us = sorted(e.ms() * 1e3 for e in evs)
+    med = statistics.median(us)
+    res = {"steps": cfg.steps, "us_per_step_median": round(med, 2),
+           "us_per_step_p90": round(us[int(0.9 * (len(us) - 1))], 2),
+           "note": "ring (57.7 MB) stays L2-resident across steps, as in streaming"}
+    res.update(_cache_roofline(cfg, med, peaks))
+    return res
+
+
+def bench_pipelined(mw, dev, peaks, flush):
+    cfg = CACHE_CONFIGS["pipelined"]
+    x = gen_cache(cfg)
+    kr, vr = x["k_ring"].to(dev), x["v_ring"].to(dev)
+    q, kn, vn = x["q"][0].to(dev), x["k_new"][0].to(dev), x["v_new"][0].to(dev)
+    ws_bytes = mw.mw_bca_cache_workspace_size(cfg.B, cfg.H, cfg.W, cfg.T, cfg.d, cfg.length)
+    ws = torch.empty(max(ws_bytes, 1), dtype=torch.uint8, device=dev)
+    o = torch.empty_like(q)
+    ts = time_repeated(lambda: mw.mw_bca_cache_fwd(q, kn, vn, kr, vr, cfg.head, cfg.length, cfg.T,
+                                                   cfg.scale, need_lse=False, workspace=ws, out=o),
+                       20, flush=flush)
+    med = statistics.median(ts) * 1e3
+    res = {"us_median": round(med, 2), "l2": "flushed between runs"}
+    res.update(_cache_roofline(cfg, med, peaks))
+    return res
+
+
+def profiled_traffic(kernel: str, workload: str):
+    """DRAM bytes per launch from the committed ncu summary, if it was taken
+    on the current kernel sources (matched by the build digest)."""
+    path = os.path.join(ROOT, "profiles", "ncu_traffic.txt")
+    try:
+        from paper_2608_01127_gb300 import _build
+        digest = _build._digest()[:16]
+        with open(path) as f:
+            for line in f:
+                parts = dict(p.split("=", 1) for p in line.split() if "=" in p)
+                if parts.get("kernel") == kernel and parts.get("workload") == workload \
+                        and parts.get("src") == digest:
+                    return float(parts["bytes_per_launch"])
+    except (OSError, ValueError, KeyError):
+        pass
+    return None
+
+
+# ------------------------------------------------------------------ reference arm (the oracle)
+
+def run_reference(args):
+    world, rank, _ = dist_env()
+    if rank != 0:
+        return
+    cfg = TRAIN_CONFIGS[WORKLOAD]
+    per_head = (fwd_flops(train_pairs(cfg), cfg.d) + bwd_flops(train_pairs(cfg), cfg.d)) / (cfg.B * cfg.H)
+    import oracle
+    x = gen_train(cfg)
+
+    def one(idx):
+        b, h = divmod(idx % (cfg.B * cfg.H), cfg.H)
+        sl = (slice(b, b + 1), slice(h, h + 1))
+        qq, kk, vv, dd = (x[n][sl] for n in ("q", "k", "v", "do"))
+        oracle.fwd(qq, kk, vv, cfg.T, cfg.scale)
+        oracle.bwd(qq, kk, vv, dd, cfg.T, cfg.scale)
+
+    for i in range(args.warmup):
+        one(i)
+    t0 = time.perf_counter()
+    for i in range(args.steps):
+        one(args.warmup + i)
+    dt = time.perf_counter() - t0
+    value = per_head * args.steps / dt / 1e12
+    out = {"impl": "reference", "metric": METRIC, "value": round(value, 6), "unit": "TFLOP/s",
+           "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
+           "ms_per_step": round(dt * 1e3 / args.steps, 2), "higher_is_better": True,
+           "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+           "config": {"workload": f"{WORKLOAD}: block-causal attention fwd+bwd; each step is one "
+                                  f"(b,h) head of B={cfg.B} H={cfg.H} d={cfg.d}, "
+                                  f"{cfg.n_chunks} chunks x {cfg.T} tokens"},
+           "cpu_baseline": {"value": round(value, 6), "unit": "TFLOP/s", "kind": "oracle",
+                            "cores": torch.get_num_threads(),
+                            "sample": f"one (b,h) head of {WORKLOAD} per step, fp64 oracle"},
+           "e2e": {"value": round(value, 6), "unit": "TFLOP/s", "h2d_bytes_per_step": 0,
+                   "d2h_bytes_per_step": 0}}
+    print(json.dumps(out), flush=True)
+
+
+def main(argv=None):
+    ap = argparse.ArgumentParser(description=__doc__.split("\n")[0])
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=50)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", choices=("ours", "reference"), default="ours")
+    ap.add_argument("--no-extras", action="store_true", help="skip the secondary workloads")
+    ap.add_argument("--cpu-seconds", type=float, default=12.0,
+                    help="budget of the oracle CPU baseline sample")
+    ap.add_argument("--no-cpu-baseline", action="store_true",
+                    help="skip the oracle CPU baseline (profiling runs)")
+    args = ap.parse_args(argv)
+    if args.warmup < 3:
+        ap.error("--warmup must be >= 3")
+    world, _, _ = dist_env()
+    if world != args.gpus and world > 1:
+        ap.error(f"--gpus {args.gpus} but WORLD_SIZE={world}")
+    if args.impl == "reference":
+        run_reference(args)
+    else:
+        run_ours(args)
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,180 @@
+/*
+ * mw_bca.h -- C ABI of the GB300 (sm_103a) block-causal attention library.
+ *
+ * The operation (paper Sec. 3.2, "Block-Causal Video DiT"): the token
+ * sequence of a video is cut into temporally ordered chunks of T_chunk tokens;
+ * a token attends bidirectionally to every token of its own chunk and causally
+ * to all tokens of earlier chunks, never to later chunks.  With
+ * chunk(i) = floor(i / T_chunk):
+ *
+ *     s_ij  = scale * <q_i, k_j>               for chunk(j) <= chunk(i)
+ *     LSE_i = ln sum_j exp(s_ij),   P_ij = exp(s_ij - LSE_i),   O_i = sum_j P_ij v_j
+ *
+ * Streaming inference (Sec. 3.5): finished chunks' keys/values are committed
+ * once to a rolling KV cache -- a FIFO of fixed capacity held here as a ring
+ * buffer -- and the chunks still being denoised (the in-flight / active
+ * window, "pipelined denoising") attend to the whole committed history and,
+ * chunk-causally, to the in-flight chunks before them and to themselves.
+ *
+ * Conventions shared by every entry point
+ *   - Tensors are DEVICE pointers to contiguous row-major arrays
+ *     [B, H, rows, d] of bf16 (raw 16-bit bfloat16 bits; nv_bfloat16 in CUDA),
+ *     16-byte aligned.  LSE arrays are fp32 [B, H, rows].  The caller owns every
+ *     buffer; the library keeps no pointer after a call returns.
+ *   - d must be 64 or 128 (the head dims of the paper's model table,
+ *     Sec. 4.1); anything else returns MW_ERR_UNSUPPORTED.
+ *   - `stream` is a cudaStream_t (NULL = legacy default stream).  Every call
+ *     validates its arguments on the host, then enqueues kernels on `stream`
+ *     and returns without synchronising.  Outputs are ready when the stream
+ *     reaches that point.
+ *   - Outputs must not overlap inputs.
+ *   - Errors: invalid arguments are rejected before anything is enqueued
+ *     (MW_ERR_INVALID_ARG / MW_ERR_UNSUPPORTED / MW_ERR_WORKSPACE) and
+ *     mw_last_error() describes why; a failed launch returns MW_ERR_CUDA.
+ *     No entry point aborts, exits, throws or traps.  Every wait inside the
+ *     kernels is bounded; a wait that runs out sets a bit in a per-device
+ *     status word that mw_device_status() reports as MW_ERR_TIMEOUT.
+ *   - The library allocates no device memory of its own except a 4-byte
+ *     status word per device (a static device variable).
+ */
+#ifndef MW_BCA_H
+#define MW_BCA_H
+
+#include <stddef.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+  MW_OK = 0,
+  MW_ERR_INVALID_ARG = 1,  /* null pointer, bad size, misalignment, bad ring state */
+  MW_ERR_UNSUPPORTED = 2,  /* valid but not implemented (d not in {64,128}) */
+  MW_ERR_CUDA = 3,         /* a CUDA runtime / driver call failed */
+  MW_ERR_TIMEOUT = 4,      /* a kernel's bounded wait expired (mw_device_status) */
+  MW_ERR_WORKSPACE = 5     /* workspace missing or smaller than *_workspace_size() */
+} mw_status;
+
+/*
+ * Block-causal attention forward (Sec. 3.2) over N = n_chunks * T_chunk tokens.
+ *   q, k, v : [B, H, N, d] bf16 (inputs, after any positional rotation)
+ *   o       : [B, H, N, d] bf16 output
+ *   lse     : [B, H, N] fp32 output, natural-log LSE_i of the scaled logits;
+ *             may be NULL when the backward pass is not needed
+ *   scale   : softmax scale (> 0), usually 1/sqrt(d)
+ * B, H, n_chunks, T_chunk >= 1.  Only the visible (query chunk, key chunk)
+ * blocks are computed; blocks above the chunk diagonal are never visited.
+ */
+mw_status mw_bca_fwd(const void* q, const void* k, const void* v, void* o, float* lse, int B,
+                     int H, int n_chunks, int T_chunk, int d, float scale, void* stream);
+
+/* Bytes of device workspace mw_bca_bwd needs (fp32 dQ accumulator plus two
+ * fp32 row vectors, each padded to a multiple of 128 rows).  0 on bad sizes. */
+size_t mw_bca_bwd_workspace_size(int B, int H, int n_chunks, int T_chunk, int d);
+
+/*
+ * Backward of mw_bca_fwd: the analytic gradient of sum(O * dO) with respect
+ * to q, k, v (training in bf16 mixed precision, Sec. 4.1), P recomputed from
+ * the saved LSE.
+ *   q, k, v, o : forward inputs and output, [B, H, N, d] bf16
+ *   lse        : forward LSE [B, H, N] fp32 (required)
+ *   dout       : upstream gradient dO [B, H, N, d] bf16
+ *   dq, dk, dv : gradients, [B, H, N, d] bf16 outputs
+ *   workspace  : device scratch of ws_bytes >= mw_bca_bwd_workspace_size(),
+ *                256-byte aligned, caller-owned; contents on entry ignored
+ * dQ is accumulated in fp32 with atomic adds, so its bits can differ from run
+ * to run in the last place; dK and dV are deterministic.
+ */
+mw_status mw_bca_bwd(const void* q, const void* k, const void* v, const void* o, const float* lse,
+                     const void* dout, void* dq, void* dk, void* dv, void* workspace,
+                     size_t ws_bytes, int B, int H, int n_chunks, int T_chunk, int d, float scale,
+                     void* stream);
+
+/*
+ * mw_bca_bwd split into its three stages, with the same arguments:
+ *   stage 1: D_i = <dO_i, O_i>, LSE_i * log2(e) and a zeroed fp32 dQ
+ *            accumulator, all in the workspace;
+ *   stage 2: the key-tile kernel: dK, dV, and dQ accumulated in the workspace;
+ *   stage 3: dQ = scale * accumulator, converted to bf16.
+ * Stages 1, 2, 3 enqueued in order on one stream with the same workspace equal
+ * mw_bca_bwd; stage 0 runs all three.  Arguments a stage does not read may be
+ * NULL (stage 1 reads o, lse, dout; stage 2 q, k, v, dout, dk, dv; stage 3 dq),
+ * the workspace is always required.  Lets a caller time or interleave stages.
+ */
+mw_status mw_bca_bwd_stage(int stage, const void* q, const void* k, const void* v, const void* o,
+                           const float* lse, const void* dout, void* dq, void* dk, void* dv,
+                           void* workspace, size_t ws_bytes, int B, int H, int n_chunks,
+                           int T_chunk, int d, float scale, void* stream);
+
+/* Bytes of device workspace mw_bca_cache_fwd needs for these sizes on the
+ * current device (split-KV partials; 0 when no split is used). */
+size_t mw_bca_cache_workspace_size(int B, int H, int n_q_chunks, int T_chunk, int d,
+                                   int cache_len);
+
+/*
+ * Forward of W = n_q_chunks in-flight chunks against the rolling KV cache
+ * (Sec. 3.5: streaming inference with a structured rolling KV cache and
+ * pipelined denoising).
+ *   q, k_new, v_new : [B, H, W*T_chunk, d] bf16, the in-flight chunks in
+ *                     temporal order
+ *   k_cache, v_cache: ring buffers [B, H, cache_cap, d] bf16 of committed
+ *                     tokens.  Logical token t (t = 0 the oldest) lives at
+ *                     physical row (cache_head + t) mod cache_cap, for
+ *                     0 <= t < cache_len; other rows are ignored.
+ *   o               : [B, H, W*T_chunk, d] bf16 output
+ *   lse             : [B, H, W*T_chunk] fp32 output or NULL
+ *   workspace       : >= mw_bca_cache_workspace_size() bytes (may be NULL
+ *                     when that size is 0), 256-byte aligned
+ * In-flight chunk j sees all cache_len cached tokens and in-flight chunks
+ * 0..j.  0 <= cache_head < cache_cap, 0 <= cache_len <= cache_cap.
+ */
+mw_status mw_bca_cache_fwd(const void* q, const void* k_new, const void* v_new,
+                           const void* k_cache, const void* v_cache, int cache_cap,
+                           int cache_head, int cache_len, void* o, float* lse, void* workspace,
+                           size_t ws_bytes, int B, int H, int n_q_chunks, int T_chunk, int d,
+                           float scale, void* stream);
+
+/*
+ * Commit of finished tokens into the ring (Sec. 3.5: once a chunk reaches the
+ * data endpoint its keys/values go to the cache and are never modified).
+ * Copies rows r = 0..rows-1 of k_src / v_src ([B, H, rows, d] bf16) to
+ * physical ring rows (slot_start + r) mod cache_cap of k_cache / v_cache
+ * ([B, H, cache_cap, d] bf16).  FIFO bookkeeping stays with the caller:
+ * append at slot (head + len) mod cap, and when the ring is full advance head
+ * by the rows written (the oldest tokens are the ones overwritten).
+ * 0 <= slot_start < cache_cap, 1 <= rows <= cache_cap.
+ */
+mw_status mw_bca_cache_commit(void* k_cache, void* v_cache, int cache_cap, int slot_start,
+                              const void* k_src, const void* v_src, int rows, int B, int H, int d,
+                              void* stream);
+
+/* Human-readable name of a status code (static string). */
+const char* mw_status_string(mw_status s);
+
+/* Message of the last failed call on this host thread ("" if none). */
+const char* mw_last_error(void);
+
+/*
+ * Reads the status word of the current device after synchronising `stream`:
+ * MW_ERR_TIMEOUT if any kernel since the last clear gave up a bounded wait,
+ * MW_ERR_CUDA if the read itself failed, else MW_OK.  clear != 0 resets it.
+ */
+mw_status mw_device_status(void* stream, int clear);
+
+/*
+ * Tuning and test knobs (process-wide; not needed for normal use):
+ *   "cache_splits"     split-KV count for mw_bca_cache_fwd, 0 = automatic
+ *                      (the workspace size follows this setting)
+ *   "wait_budget_ms"   time limit of every bounded wait inside the kernels
+ *                      (default 2000)
+ *   "debug_skip_q_load" non-zero: forward kernels never load Q, so their
+ *                      first wait expires; for testing the timeout path only
+ * Returns MW_ERR_INVALID_ARG for an unknown name or a negative value.
+ */
+mw_status mw_set_option(const char* name, long long value);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* MW_BCA_H */

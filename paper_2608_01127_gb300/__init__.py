@@ -1,0 +1,266 @@
+"""GB300 (sm_103a) block-causal attention for streaming video world models.
+
+Python binding of the C ABI in ``include/mw_bca.h`` (argument marshalling
+only; every step of the computation runs in the library's CUDA kernels).
+PyTorch provides device memory and the current stream.  There is no CPU
+path: without the built library every call raises.
+
+Entry points (same names as the C ABI, taking torch tensors):
+  mw_bca_fwd(q, k, v, T_chunk, scale=None, need_lse=True) -> (o, lse)
+  mw_bca_bwd(q, k, v, o, lse, dout, T_chunk, scale=None) -> (dq, dk, dv)
+  mw_bca_cache_fwd(q, k_new, v_new, k_cache, v_cache, cache_head, cache_len,
+                   T_chunk, scale=None, need_lse=True) -> (o, lse)
+  mw_bca_cache_commit(k_cache, v_cache, slot_start, k_src, v_src)
+  mw_device_status(clear=True), mw_set_option(name, value)
+Tensors are contiguous bf16 [B, H, rows, d] on the current CUDA device.
+"""
+from __future__ import annotations
+
+import ctypes
+import math
+import os
+from typing import Optional, Tuple
+
+import torch
+
+__all__ = [
+    "MWError", "library", "lib_path", "mw_bca_fwd", "mw_bca_bwd", "mw_bca_cache_fwd",
+    "mw_bca_cache_commit", "mw_bca_bwd_workspace_size", "mw_bca_cache_workspace_size",
+    "mw_device_status", "mw_set_option", "BlockCausalAttention", "EXPORTED_SYMBOLS",
+    "RingState",
+]
+
+_PKG = os.path.dirname(os.path.abspath(__file__))
+lib_path = os.path.join(_PKG, "_lib", "libmw_bca.so")
+
+EXPORTED_SYMBOLS = (
+    "mw_bca_fwd", "mw_bca_bwd_workspace_size", "mw_bca_bwd", "mw_bca_bwd_stage",
+    "mw_bca_cache_workspace_size",
+    "mw_bca_cache_fwd", "mw_bca_cache_commit", "mw_status_string", "mw_last_error",
+    "mw_device_status", "mw_set_option",
+)
+
+STATUS = {0: "MW_OK", 1: "MW_ERR_INVALID_ARG", 2: "MW_ERR_UNSUPPORTED", 3: "MW_ERR_CUDA",
+          4: "MW_ERR_TIMEOUT", 5: "MW_ERR_WORKSPACE"}
+
+
+class MWError(RuntimeError):
+    """A non-zero mw_status from the library, with mw_last_error()'s text."""
+
+    def __init__(self, code: int, message: str):
+        super().__init__(f"{STATUS.get(code, code)}: {message}")
+        self.code = code
+
+
+_lib: Optional[ctypes.CDLL] = None
+
+_P = ctypes.c_void_p
+_I = ctypes.c_int
+_F = ctypes.c_float
+_Z = ctypes.c_size_t
+
+
+def library() -> ctypes.CDLL:
+    """The loaded C library (raises when it has not been built)."""
+    global _lib
+    if _lib is not None:
+        return _lib
+    if not os.path.exists(lib_path):
+        raise RuntimeError(
+            f"{lib_path} is missing: build it with `python -c 'import __graft_entry__ as g; "
+            "g.build()'` (there is no CPU fallback)")
+    lib = ctypes.CDLL(lib_path)
+    sig = {
+        "mw_bca_fwd": (_I, [_P, _P, _P, _P, _P, _I, _I, _I, _I, _I, _F, _P]),
+        "mw_bca_bwd_workspace_size": (_Z, [_I, _I, _I, _I, _I]),
+        "mw_bca_bwd": (_I, [_P, _P, _P, _P, _P, _P, _P, _P, _P, _P, _Z,
+                            _I, _I, _I, _I, _I, _F, _P]),
+        "mw_bca_bwd_stage": (_I, [_I, _P, _P, _P, _P, _P, _P, _P, _P, _P, _P, _Z,
+                                  _I, _I, _I, _I, _I, _F, _P]),
+        "mw_bca_cache_workspace_size": (_Z, [_I, _I, _I, _I, _I, _I]),
+        "mw_bca_cache_fwd": (_I, [_P, _P, _P, _P, _P, _I, _I, _I, _P, _P, _P, _Z,
+                                  _I, _I, _I, _I, _I, _F, _P]),
+        "mw_bca_cache_commit": (_I, [_P, _P, _I, _I, _P, _P, _I, _I, _I, _I, _P]),
+        "mw_status_string": (ctypes.c_char_p, [_I]),
+        "mw_last_error": (ctypes.c_char_p, []),
+        "mw_device_status": (_I, [_P, _I]),
+        "mw_set_option": (_I, [ctypes.c_char_p, ctypes.c_longlong]),
+    }
+    for name, (res, args) in sig.items():
+        fn = getattr(lib, name)
+        fn.restype = res
+        fn.argtypes = args
+    _lib = lib
+    return lib
+
+
+def _check(code: int) -> None:
+    if code != 0:
+        msg = library().mw_last_error().decode(errors="replace")
+        raise MWError(code, msg)
+
+
+def _stream() -> int:
+    return torch.cuda.current_stream().cuda_stream
+
+
+def _ptr(t: Optional[torch.Tensor]) -> Optional[int]:
+    return None if t is None else t.data_ptr()
+
+
+def _bhnd(t: torch.Tensor, name: str) -> Tuple[int, int, int, int]:
+    if t.dtype != torch.bfloat16:
+        raise TypeError(f"{name} must be bfloat16, got {t.dtype}")
+    if not t.is_cuda:
+        raise ValueError(f"{name} must be a CUDA tensor (there is no CPU path)")
+    if t.dim() != 4 or not t.is_contiguous():
+        raise ValueError(f"{name} must be a contiguous [B, H, rows, d] tensor")
+    return tuple(t.shape)  # type: ignore[return-value]
+
+
+def _scale(scale: Optional[float], d: int) -> float:
+    return 1.0 / math.sqrt(d) if scale is None else float(scale)
+
+
+def mw_bca_fwd(q: torch.Tensor, k: torch.Tensor, v: torch.Tensor, T_chunk: int,
+               scale: Optional[float] = None, need_lse: bool = True
+               ) -> Tuple[torch.Tensor, Optional[torch.Tensor]]:
+    """Block-causal attention forward (Sec. 3.2); returns (O, LSE or None)."""
+    B, H, N, d = _bhnd(q, "q")
+    for t, n in ((k, "k"), (v, "v")):
+        if _bhnd(t, n) != (B, H, N, d):
+            raise ValueError(f"{n} shape {tuple(t.shape)} != q shape {(B, H, N, d)}")
+    if N % T_chunk != 0:
+        raise ValueError(f"sequence length {N} is not a multiple of T_chunk={T_chunk}")
+    o = torch.empty_like(q)
+    lse = torch.empty((B, H, N), dtype=torch.float32, device=q.device) if need_lse else None
+    _check(library().mw_bca_fwd(_ptr(q), _ptr(k), _ptr(v), _ptr(o), _ptr(lse), B, H,
+                                N // T_chunk, T_chunk, d, _scale(scale, d), _stream()))
+    return o, lse
+
+
+def mw_bca_bwd_workspace_size(B: int, H: int, n_chunks: int, T_chunk: int, d: int) -> int:
+    return int(library().mw_bca_bwd_workspace_size(B, H, n_chunks, T_chunk, d))
+
+
+def mw_bca_bwd(q, k, v, o, lse, dout, T_chunk: int, scale: Optional[float] = None,
+               workspace: Optional[torch.Tensor] = None, stage: int = 0, out=None):
+    """Gradients (dQ, dK, dV) of sum(O * dout) through mw_bca_fwd.
+
+    ``stage`` 1/2/3 runs one stage of the backward (see mw_bca_bwd_stage);
+    ``out`` = (dq, dk, dv) preallocated outputs."""
+    B, H, N, d = _bhnd(q, "q")
+    for t, n in ((k, "k"), (v, "v"), (o, "o"), (dout, "dout")):
+        if _bhnd(t, n) != (B, H, N, d):
+            raise ValueError(f"{n} shape {tuple(t.shape)} != q shape {(B, H, N, d)}")
+    if lse is None or lse.dtype != torch.float32 or tuple(lse.shape) != (B, H, N) \
+            or not lse.is_contiguous():
+        raise ValueError("lse must be a contiguous fp32 [B, H, N] tensor")
+    if N % T_chunk != 0:
+        raise ValueError(f"sequence length {N} is not a multiple of T_chunk={T_chunk}")
+    n = N // T_chunk
+    ws_bytes = mw_bca_bwd_workspace_size(B, H, n, T_chunk, d)
+    if workspace is None or workspace.numel() < ws_bytes:
+        workspace = torch.empty(ws_bytes, dtype=torch.uint8, device=q.device)
+    if out is None:
+        dq, dk, dv = torch.empty_like(q), torch.empty_like(k), torch.empty_like(v)
+    else:
+        dq, dk, dv = out
+    _check(library().mw_bca_bwd_stage(stage, _ptr(q), _ptr(k), _ptr(v), _ptr(o), _ptr(lse),
+                                      _ptr(dout), _ptr(dq), _ptr(dk), _ptr(dv), _ptr(workspace),
+                                      ws_bytes, B, H, n, T_chunk, d, _scale(scale, d), _stream()))
+    return dq, dk, dv
+
+
+def mw_bca_cache_workspace_size(B: int, H: int, n_q_chunks: int, T_chunk: int, d: int,
+                                cache_len: int) -> int:
+    return int(library().mw_bca_cache_workspace_size(B, H, n_q_chunks, T_chunk, d, cache_len))
+
+
+def mw_bca_cache_fwd(q, k_new, v_new, k_cache, v_cache, cache_head: int, cache_len: int,
+                     T_chunk: int, scale: Optional[float] = None, need_lse: bool = True,
+                     workspace: Optional[torch.Tensor] = None, out: Optional[torch.Tensor] = None):
+    """In-flight chunks against the rolling KV cache (Sec. 3.5); returns (O, LSE or None)."""
+    B, H, M, d = _bhnd(q, "q")
+    for t, n in ((k_new, "k_new"), (v_new, "v_new")):
+        if _bhnd(t, n) != (B, H, M, d):
+            raise ValueError(f"{n} shape {tuple(t.shape)} != q shape {(B, H, M, d)}")
+    Bc, Hc, cap, dc = _bhnd(k_cache, "k_cache")
+    if (Bc, Hc, dc) != (B, H, d) or tuple(v_cache.shape) != tuple(k_cache.shape):
+        raise ValueError("k_cache / v_cache must be [B, H, cap, d] matching q")
+    _bhnd(v_cache, "v_cache")
+    if M % T_chunk != 0:
+        raise ValueError(f"{M} query rows is not a multiple of T_chunk={T_chunk}")
+    W = M // T_chunk
+    ws_bytes = mw_bca_cache_workspace_size(B, H, W, T_chunk, d, cache_len)
+    if ws_bytes and (workspace is None or workspace.numel() < ws_bytes):
+        workspace = torch.empty(ws_bytes, dtype=torch.uint8, device=q.device)
+    o = torch.empty_like(q) if out is None else out
+    lse = torch.empty((B, H, M), dtype=torch.float32, device=q.device) if need_lse else None
+    _check(library().mw_bca_cache_fwd(
+        _ptr(q), _ptr(k_new), _ptr(v_new), _ptr(k_cache), _ptr(v_cache), cap, cache_head,
+        cache_len, _ptr(o), _ptr(lse), _ptr(workspace) if ws_bytes else None, ws_bytes,
+        B, H, W, T_chunk, d, _scale(scale, d), _stream()))
+    return o, lse
+
+
+def mw_bca_cache_commit(k_cache, v_cache, slot_start: int, k_src, v_src) -> None:
+    """Write k_src / v_src rows at ring rows (slot_start + r) mod cap (Sec. 3.5)."""
+    B, H, cap, d = _bhnd(k_cache, "k_cache")
+    _bhnd(v_cache, "v_cache")
+    Bs, Hs, rows, ds = _bhnd(k_src, "k_src")
+    _bhnd(v_src, "v_src")
+    if (Bs, Hs, ds) != (B, H, d) or tuple(v_src.shape) != tuple(k_src.shape):
+        raise ValueError("k_src / v_src must be [B, H, rows, d] matching the cache")
+    _check(library().mw_bca_cache_commit(_ptr(k_cache), _ptr(v_cache), cap, slot_start,
+                                         _ptr(k_src), _ptr(v_src), rows, B, H, d, _stream()))
+
+
+def mw_device_status(clear: bool = True) -> int:
+    """Synchronises the current stream and returns the device status code."""
+    return int(library().mw_device_status(_stream(), 1 if clear else 0))
+
+
+def mw_set_option(name: str, value: int) -> None:
+    _check(library().mw_set_option(name.encode(), int(value)))
+
+
+class RingState:
+    """Host-side FIFO bookkeeping of a rolling KV cache (Sec. 3.5).
+
+    ``head`` is the physical row of the logically oldest cached token and
+    ``length`` the number of cached tokens.  ``commit(rows)`` returns the
+    physical slot where the next ``rows`` tokens are written -- right after
+    the newest token -- and evicts the oldest tokens when the ring overflows.
+    """
+
+    def __init__(self, cap: int, head: int = 0, length: int = 0):
+        if not (cap >= 1 and 0 <= head < cap and 0 <= length <= cap):
+            raise ValueError(f"bad ring state cap={cap} head={head} length={length}")
+        self.cap, self.head, self.length = cap, head, length
+
+    def commit(self, rows: int) -> int:
+        if not 1 <= rows <= self.cap:
+            raise ValueError(f"rows={rows} not in [1, {self.cap}]")
+        slot = (self.head + self.length) % self.cap
+        overflow = max(0, self.length + rows - self.cap)
+        self.head = (self.head + overflow) % self.cap
+        self.length = min(self.cap, self.length + rows)
+        return slot
+
+
+class BlockCausalAttention(torch.autograd.Function):
+    """Autograd wrapper: O = block-causal attention(q, k, v) with chunks of T_chunk."""
+
+    @staticmethod
+    def forward(ctx, q, k, v, T_chunk: int, scale: Optional[float] = None):
+        o, lse = mw_bca_fwd(q, k, v, T_chunk, scale, need_lse=True)
+        ctx.save_for_backward(q, k, v, o, lse)
+        ctx.T_chunk, ctx.scale = T_chunk, scale
+        return o
+
+    @staticmethod
+    def backward(ctx, do):
+        q, k, v, o, lse = ctx.saved_tensors
+        dq, dk, dv = mw_bca_bwd(q, k, v, o, lse, do.contiguous(), ctx.T_chunk, ctx.scale)
+        return dq, dk, dv, None, None

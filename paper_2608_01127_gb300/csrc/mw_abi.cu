@@ -1,0 +1,502 @@
+// C ABI of the block-causal attention library (declared in include/mw_bca.h):
+// host-side validation, TMA descriptor creation, split-KV planning and
+// kernel launches.  Validation happens before any CUDA call, so argument
+// errors are reported without touching the device.
+#include <cudaTypedefs.h>
+
+#include <climits>
+#include <cstdarg>
+#include <cstdio>
+#include <cstring>
+#include <mutex>
+#include <string>
+
+#include "../../include/mw_bca.h"
+#include "mw_internal.h"
+#include "mw_ptx.cuh"
+
+namespace {
+
+thread_local std::string g_last_error;
+
+// Device status word (bit 0: a bounded wait expired; bit 1: misaligned
+// shared memory).  One per device: a static device variable.
+__device__ unsigned g_status_word;
+
+constexpr int kMaxDevices = 64;
+unsigned* g_status_ptr[kMaxDevices] = {};
+std::mutex g_mutex;
+
+long long g_opt_cache_splits = 0;
+long long g_opt_budget_ms = 2000;
+long long g_opt_skip_q = 0;
+
+mw_status fail(mw_status s, const char* fmt, ...) {
+  char buf[512];
+  va_list ap;
+  va_start(ap, fmt);
+  vsnprintf(buf, sizeof(buf), fmt, ap);
+  va_end(ap);
+  g_last_error = buf;
+  return s;
+}
+
+mw_status ok() {
+  g_last_error.clear();
+  return MW_OK;
+}
+
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+mw_status check_ptr(const void* p, const char* name) {
+  if (p == nullptr) return fail(MW_ERR_INVALID_ARG, "%s is NULL", name);
+  if (!aligned16(p)) return fail(MW_ERR_INVALID_ARG, "%s is not 16-byte aligned", name);
+  return MW_OK;
+}
+
+mw_status check_dims(int B, int H, int d) {
+  if (B < 1 || H < 1) return fail(MW_ERR_INVALID_ARG, "B and H must be >= 1 (B=%d H=%d)", B, H);
+  if (static_cast<long long>(B) * H > (1 << 20))
+    return fail(MW_ERR_INVALID_ARG, "B*H=%lld exceeds 2^20", static_cast<long long>(B) * H);
+  if (d != 64 && d != 128) return fail(MW_ERR_UNSUPPORTED, "head dim d=%d (supported: 64, 128)", d);
+  return MW_OK;
+}
+
+mw_status check_rows(long long rows, const char* what) {
+  if (rows < 1 || rows > (1 << 24))
+    return fail(MW_ERR_INVALID_ARG, "%s=%lld out of range [1, 2^24]", what, rows);
+  return MW_OK;
+}
+
+#define MW_TRY(expr)                 \
+  do {                               \
+    mw_status _s = (expr);           \
+    if (_s != MW_OK) return _s;      \
+  } while (0)
+
+PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
+  static PFN_cuTensorMapEncodeTiled_v12000 fn = [] {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault,
+                                         &q) != cudaSuccess ||
+        q != cudaDriverEntryPointSuccess)
+      p = nullptr;
+    return reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
+  }();
+  return fn;
+}
+
+// 3-D map over [BH, rows, d] bf16 with 64 x 128-row boxes and the 128-byte
+// swizzle the tcgen05 descriptors expect; rows past the end read as zero.
+mw_status make_map(CUtensorMap* m, const void* ptr, int rows, int BH, int d, const char* name) {
+  auto fn = encode_fn();
+  if (!fn) return fail(MW_ERR_CUDA, "cuTensorMapEncodeTiled is unavailable (no CUDA driver?)");
+  cuuint64_t dims[3] = {static_cast<cuuint64_t>(d), static_cast<cuuint64_t>(rows),
+                        static_cast<cuuint64_t>(BH)};
+  cuuint64_t strides[2] = {static_cast<cuuint64_t>(d) * 2,
+                           static_cast<cuuint64_t>(rows) * d * 2};
+  cuuint32_t box[3] = {64, static_cast<cuuint32_t>(mw::kTileRows), 1};
+  cuuint32_t estr[3] = {1, 1, 1};
+  CUresult r = fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(ptr), dims, strides, box,
+                  estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                  CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  if (r != CUDA_SUCCESS) return fail(MW_ERR_CUDA, "cuTensorMapEncodeTiled(%s) failed: %d", name, (int)r);
+  return MW_OK;
+}
+
+mw_status status_ptr(unsigned** out) {
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return fail(MW_ERR_CUDA, "cudaGetDevice: %s", cudaGetErrorString(e));
+  if (dev < 0 || dev >= kMaxDevices) return fail(MW_ERR_CUDA, "device index %d too large", dev);
+  std::lock_guard<std::mutex> lock(g_mutex);
+  if (!g_status_ptr[dev]) {
+    void* p = nullptr;
+    e = cudaGetSymbolAddress(&p, g_status_word);
+    if (e != cudaSuccess) return fail(MW_ERR_CUDA, "cudaGetSymbolAddress: %s", cudaGetErrorString(e));
+    g_status_ptr[dev] = static_cast<unsigned*>(p);
+  }
+  *out = g_status_ptr[dev];
+  return MW_OK;
+}
+
+int sm_count() {
+  int dev = 0, n = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) return 152;
+  if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n <= 0)
+    return 152;
+  return n;
+}
+
+unsigned long long budget_ns() { return static_cast<unsigned long long>(g_opt_budget_ms) * 1000000ull; }
+
+size_t align256(size_t x) { return (x + 255) & ~size_t(255); }
+
+int ceil_div(long long a, long long b) { return static_cast<int>((a + b - 1) / b); }
+
+// Split-KV count for the cache path: balances (query blocks x splits) CTAs
+// over the SMs against the per-split key-tile count plus a fixed cost.
+int plan_splits(int BH, int rows_q, int cache_len) {
+  if (g_opt_cache_splits > 0) return static_cast<int>(g_opt_cache_splits);
+  const int blocks = BH * ceil_div(rows_q, mw::kFwdBlockRows);
+  const int tiles = ceil_div(cache_len, mw::kTileRows) + 1 + ceil_div(rows_q, mw::kTileRows);
+  const int sms = sm_count();
+  int best = 1;
+  long long best_cost = LLONG_MAX;
+  for (int s = 1; s <= mw::kMaxSplits && s <= tiles; ++s) {
+    const long long waves = ceil_div(static_cast<long long>(blocks) * s, sms);
+    const long long cost = waves * (ceil_div(tiles, s) + 3);
+    if (cost < best_cost) {
+      best_cost = cost;
+      best = s;
+    }
+  }
+  return best;
+}
+
+size_t cache_ws_bytes(int splits, int BH, int rows_q, int d) {
+  if (splits <= 1) return 0;
+  const size_t o_part = static_cast<size_t>(splits) * BH * rows_q * d * sizeof(float);
+  const size_t l_part = static_cast<size_t>(splits) * BH * rows_q * sizeof(float);
+  return align256(o_part) + align256(l_part);
+}
+
+struct BwdWs {
+  size_t dq_acc, lse2, delta, total;
+};
+
+BwdWs bwd_ws_layout(int BH, int N_pad, int d) {
+  BwdWs w;
+  w.dq_acc = 0;
+  w.lse2 = align256(static_cast<size_t>(BH) * N_pad * d * sizeof(float));
+  w.delta = w.lse2 + align256(static_cast<size_t>(BH) * N_pad * sizeof(float));
+  w.total = w.delta + align256(static_cast<size_t>(BH) * N_pad * sizeof(float));
+  return w;
+}
+
+// Makes the device of `stream` current on the calling thread for the scope
+// of one entry point (binding its primary context, which driver calls such
+// as cuTensorMapEncodeTiled need on threads where nothing else did), and
+// restores the caller's device afterwards.
+class DeviceScope {
+ public:
+  explicit DeviceScope(cudaStream_t stream) {
+    if (cudaGetDevice(&prev_) != cudaSuccess) prev_ = -1;
+    int dev = prev_;
+    if (stream != nullptr && cudaStreamGetDevice(stream, &dev) != cudaSuccess) dev = prev_;
+    if (dev < 0) dev = 0;
+    err_ = cudaSetDevice(dev);
+    dev_ = dev;
+  }
+  ~DeviceScope() {
+    if (prev_ >= 0 && prev_ != dev_) cudaSetDevice(prev_);
+  }
+  mw_status status() const {
+    if (err_ != cudaSuccess) return fail(MW_ERR_CUDA, "cudaSetDevice: %s", cudaGetErrorString(err_));
+    return MW_OK;
+  }
+
+ private:
+  int prev_ = -1, dev_ = 0;
+  cudaError_t err_ = cudaSuccess;
+};
+
+mw_status launch_status(cudaError_t e, const char* what) {
+  if (e != cudaSuccess) return fail(MW_ERR_CUDA, "%s: %s", what, cudaGetErrorString(e));
+  return ok();
+}
+
+mw_status fwd_common(const void* q, const void* k, const void* v, const void* kr, const void* vr,
+                     int cap, int head, int len, void* o, float* lse, void* ws, size_t ws_bytes,
+                     int BH, int rows_q, int T, int d, float scale, int splits,
+                     cudaStream_t stream) {
+  DeviceScope scope(stream);
+  MW_TRY(scope.status());
+  unsigned* status = nullptr;
+  MW_TRY(status_ptr(&status));
+  CUtensorMap tq, tk, tv, tkr, tvr;
+  MW_TRY(make_map(&tq, q, rows_q, BH, d, "q"));
+  MW_TRY(make_map(&tk, k, rows_q, BH, d, "k"));
+  MW_TRY(make_map(&tv, v, rows_q, BH, d, "v"));
+  if (len > 0) {
+    MW_TRY(make_map(&tkr, kr, cap, BH, d, "k_cache"));
+    MW_TRY(make_map(&tvr, vr, cap, BH, d, "v_cache"));
+  } else {
+    tkr = tk;
+    tvr = tv;
+  }
+  mw::FwdParams p{};
+  p.BH = BH;
+  p.rows_q = rows_q;
+  p.T = T;
+  p.n_qblocks = ceil_div(rows_q, mw::kFwdBlockRows);
+  p.ring_cap = len > 0 ? cap : 1;
+  p.ring_head = len > 0 ? head : 0;
+  p.ring_len = len;
+  p.num_splits = splits;
+  p.scale_log2 = scale * 1.4426950408889634f;
+  p.o = static_cast<__nv_bfloat16*>(o);
+  p.lse = lse;
+  p.status = status;
+  p.budget_ns = budget_ns();
+  p.debug_skip_q = static_cast<int>(g_opt_skip_q);
+  if (p.num_splits > 1) {
+    const size_t need = cache_ws_bytes(p.num_splits, BH, rows_q, d);
+    if (ws_bytes < need)
+      return fail(MW_ERR_WORKSPACE, "workspace %zu bytes, need %zu", ws_bytes, need);
+    char* base = static_cast<char*>(ws);
+    p.o_part = reinterpret_cast<float*>(base);
+    p.lse_part = reinterpret_cast<float*>(
+        base + align256(static_cast<size_t>(p.num_splits) * BH * rows_q * d * sizeof(float)));
+  }
+  MW_TRY(launch_status(mw::launch_fwd(d, tq, tk, tv, tkr, tvr, p, stream), "forward kernel launch"));
+  if (p.num_splits > 1)
+    MW_TRY(launch_status(mw::launch_combine(d, p.o_part, p.lse_part, p.o, lse, p.num_splits, BH,
+                                            rows_q, stream),
+                         "combine kernel launch"));
+  return ok();
+}
+
+}  // namespace
+
+extern "C" {
+
+const char* mw_status_string(mw_status s) {
+  switch (s) {
+    case MW_OK: return "MW_OK";
+    case MW_ERR_INVALID_ARG: return "MW_ERR_INVALID_ARG";
+    case MW_ERR_UNSUPPORTED: return "MW_ERR_UNSUPPORTED";
+    case MW_ERR_CUDA: return "MW_ERR_CUDA";
+    case MW_ERR_TIMEOUT: return "MW_ERR_TIMEOUT";
+    case MW_ERR_WORKSPACE: return "MW_ERR_WORKSPACE";
+  }
+  return "MW_ERR_UNKNOWN";
+}
+
+const char* mw_last_error(void) { return g_last_error.c_str(); }
+
+mw_status mw_set_option(const char* name, long long value) {
+  if (name == nullptr) return fail(MW_ERR_INVALID_ARG, "option name is NULL");
+  if (value < 0) return fail(MW_ERR_INVALID_ARG, "option %s: negative value", name);
+  if (std::strcmp(name, "cache_splits") == 0) {
+    if (value > mw::kMaxSplits) return fail(MW_ERR_INVALID_ARG, "cache_splits > %d", mw::kMaxSplits);
+    g_opt_cache_splits = value;
+  } else if (std::strcmp(name, "wait_budget_ms") == 0) {
+    if (value < 1) return fail(MW_ERR_INVALID_ARG, "wait_budget_ms must be >= 1");
+    g_opt_budget_ms = value;
+  } else if (std::strcmp(name, "debug_skip_q_load") == 0) {
+    g_opt_skip_q = value;
+  } else {
+    return fail(MW_ERR_INVALID_ARG, "unknown option '%s'", name);
+  }
+  return ok();
+}
+
+mw_status mw_bca_fwd(const void* q, const void* k, const void* v, void* o, float* lse, int B,
+                     int H, int n_chunks, int T_chunk, int d, float scale, void* stream) {
+  MW_TRY(check_dims(B, H, d));
+  if (n_chunks < 1 || T_chunk < 1)
+    return fail(MW_ERR_INVALID_ARG, "n_chunks=%d and T_chunk=%d must be >= 1", n_chunks, T_chunk);
+  const long long N = static_cast<long long>(n_chunks) * T_chunk;
+  MW_TRY(check_rows(N, "n_chunks*T_chunk"));
+  if (!(scale > 0.f)) return fail(MW_ERR_INVALID_ARG, "scale must be > 0");
+  MW_TRY(check_ptr(q, "q"));
+  MW_TRY(check_ptr(k, "k"));
+  MW_TRY(check_ptr(v, "v"));
+  MW_TRY(check_ptr(o, "o"));
+  if (lse && (reinterpret_cast<uintptr_t>(lse) & 3u))
+    return fail(MW_ERR_INVALID_ARG, "lse is not 4-byte aligned");
+  return fwd_common(q, k, v, nullptr, nullptr, 1, 0, 0, o, lse, nullptr, 0, B * H,
+                    static_cast<int>(N), T_chunk, d, scale, 1, static_cast<cudaStream_t>(stream));
+}
+
+size_t mw_bca_bwd_workspace_size(int B, int H, int n_chunks, int T_chunk, int d) {
+  if (B < 1 || H < 1 || n_chunks < 1 || T_chunk < 1 || (d != 64 && d != 128)) return 0;
+  const long long N = static_cast<long long>(n_chunks) * T_chunk;
+  if (N > (1 << 24)) return 0;
+  const int N_pad = ceil_div(N, mw::kTileRows) * mw::kTileRows;
+  return bwd_ws_layout(B * H, N_pad, d).total;
+}
+
+mw_status mw_bca_bwd_stage(int stage, const void* q, const void* k, const void* v, const void* o,
+                           const float* lse, const void* dout, void* dq, void* dk, void* dv,
+                           void* workspace, size_t ws_bytes, int B, int H, int n_chunks,
+                           int T_chunk, int d, float scale, void* stream) {
+  if (stage < 0 || stage > 3) return fail(MW_ERR_INVALID_ARG, "stage=%d not in [0, 3]", stage);
+  const bool pre = stage == 0 || stage == 1;
+  const bool main = stage == 0 || stage == 2;
+  const bool post = stage == 0 || stage == 3;
+  MW_TRY(check_dims(B, H, d));
+  if (n_chunks < 1 || T_chunk < 1)
+    return fail(MW_ERR_INVALID_ARG, "n_chunks=%d and T_chunk=%d must be >= 1", n_chunks, T_chunk);
+  const long long N = static_cast<long long>(n_chunks) * T_chunk;
+  MW_TRY(check_rows(N, "n_chunks*T_chunk"));
+  if (!(scale > 0.f)) return fail(MW_ERR_INVALID_ARG, "scale must be > 0");
+  if (main) {
+    MW_TRY(check_ptr(q, "q"));
+    MW_TRY(check_ptr(k, "k"));
+    MW_TRY(check_ptr(v, "v"));
+    MW_TRY(check_ptr(dk, "dk"));
+    MW_TRY(check_ptr(dv, "dv"));
+  }
+  if (pre) {
+    MW_TRY(check_ptr(o, "o"));
+    MW_TRY(check_ptr(lse, "lse"));
+  }
+  if (pre || main) MW_TRY(check_ptr(dout, "dout"));
+  if (post) MW_TRY(check_ptr(dq, "dq"));
+  const int BH = B * H;
+  const int N_pad = ceil_div(N, mw::kTileRows) * mw::kTileRows;
+  const BwdWs w = bwd_ws_layout(BH, N_pad, d);
+  if (workspace == nullptr || ws_bytes < w.total)
+    return fail(MW_ERR_WORKSPACE, "workspace %zu bytes, need %zu", ws_bytes, w.total);
+  if (reinterpret_cast<uintptr_t>(workspace) & 255u)
+    return fail(MW_ERR_INVALID_ARG, "workspace is not 256-byte aligned");
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  DeviceScope scope(s);
+  MW_TRY(scope.status());
+  char* base = static_cast<char*>(workspace);
+  float* dq_acc = reinterpret_cast<float*>(base + w.dq_acc);
+  float* lse2 = reinterpret_cast<float*>(base + w.lse2);
+  float* delta = reinterpret_cast<float*>(base + w.delta);
+  if (pre)
+    MW_TRY(launch_status(mw::launch_bwd_pre(d, static_cast<const __nv_bfloat16*>(o),
+                                            static_cast<const __nv_bfloat16*>(dout), lse, lse2,
+                                            delta, dq_acc, BH, static_cast<int>(N), N_pad, s),
+                         "backward pre kernel launch"));
+  if (main) {
+    unsigned* status = nullptr;
+    MW_TRY(status_ptr(&status));
+    CUtensorMap tq, tk, tv, tdo;
+    MW_TRY(make_map(&tq, q, static_cast<int>(N), BH, d, "q"));
+    MW_TRY(make_map(&tk, k, static_cast<int>(N), BH, d, "k"));
+    MW_TRY(make_map(&tv, v, static_cast<int>(N), BH, d, "v"));
+    MW_TRY(make_map(&tdo, dout, static_cast<int>(N), BH, d, "dout"));
+    mw::BwdParams p{};
+    p.BH = BH;
+    p.N = static_cast<int>(N);
+    p.N_pad = N_pad;
+    p.T = T_chunk;
+    p.scale_log2 = scale * 1.4426950408889634f;
+    p.scale = scale;
+    p.lse2 = lse2;
+    p.delta = delta;
+    p.dq_acc = dq_acc;
+    p.dk = static_cast<__nv_bfloat16*>(dk);
+    p.dv = static_cast<__nv_bfloat16*>(dv);
+    p.status = status;
+    p.budget_ns = budget_ns();
+    MW_TRY(launch_status(mw::launch_bwd_main(d, tq, tk, tv, tdo, p, s), "backward kernel launch"));
+  }
+  if (post)
+    MW_TRY(launch_status(mw::launch_bwd_post(d, dq_acc, static_cast<__nv_bfloat16*>(dq), scale, BH,
+                                             static_cast<int>(N), N_pad, s),
+                         "backward post kernel launch"));
+  return ok();
+}
+
+mw_status mw_bca_bwd(const void* q, const void* k, const void* v, const void* o, const float* lse,
+                     const void* dout, void* dq, void* dk, void* dv, void* workspace,
+                     size_t ws_bytes, int B, int H, int n_chunks, int T_chunk, int d, float scale,
+                     void* stream) {
+  return mw_bca_bwd_stage(0, q, k, v, o, lse, dout, dq, dk, dv, workspace, ws_bytes, B, H,
+                          n_chunks, T_chunk, d, scale, stream);
+}
+
+size_t mw_bca_cache_workspace_size(int B, int H, int n_q_chunks, int T_chunk, int d,
+                                   int cache_len) {
+  if (B < 1 || H < 1 || n_q_chunks < 1 || T_chunk < 1 || cache_len < 0 || (d != 64 && d != 128))
+    return 0;
+  const long long rows = static_cast<long long>(n_q_chunks) * T_chunk;
+  if (rows > (1 << 24)) return 0;
+  const int splits = plan_splits(B * H, static_cast<int>(rows), cache_len);
+  return cache_ws_bytes(splits, B * H, static_cast<int>(rows), d);
+}
+
+mw_status mw_bca_cache_fwd(const void* q, const void* k_new, const void* v_new,
+                           const void* k_cache, const void* v_cache, int cache_cap,
+                           int cache_head, int cache_len, void* o, float* lse, void* workspace,
+                           size_t ws_bytes, int B, int H, int n_q_chunks, int T_chunk, int d,
+                           float scale, void* stream) {
+  MW_TRY(check_dims(B, H, d));
+  if (n_q_chunks < 1 || T_chunk < 1)
+    return fail(MW_ERR_INVALID_ARG, "n_q_chunks=%d and T_chunk=%d must be >= 1", n_q_chunks, T_chunk);
+  const long long rows = static_cast<long long>(n_q_chunks) * T_chunk;
+  MW_TRY(check_rows(rows, "n_q_chunks*T_chunk"));
+  if (cache_cap < 1 || cache_cap > (1 << 24))
+    return fail(MW_ERR_INVALID_ARG, "cache_cap=%d out of range [1, 2^24]", cache_cap);
+  if (cache_head < 0 || cache_head >= cache_cap)
+    return fail(MW_ERR_INVALID_ARG, "cache_head=%d not in [0, cache_cap=%d)", cache_head, cache_cap);
+  if (cache_len < 0 || cache_len > cache_cap)
+    return fail(MW_ERR_INVALID_ARG, "cache_len=%d not in [0, cache_cap=%d]", cache_len, cache_cap);
+  if (!(scale > 0.f)) return fail(MW_ERR_INVALID_ARG, "scale must be > 0");
+  MW_TRY(check_ptr(q, "q"));
+  MW_TRY(check_ptr(k_new, "k_new"));
+  MW_TRY(check_ptr(v_new, "v_new"));
+  MW_TRY(check_ptr(o, "o"));
+  if (cache_len > 0) {
+    MW_TRY(check_ptr(k_cache, "k_cache"));
+    MW_TRY(check_ptr(v_cache, "v_cache"));
+  }
+  if (lse && (reinterpret_cast<uintptr_t>(lse) & 3u))
+    return fail(MW_ERR_INVALID_ARG, "lse is not 4-byte aligned");
+  const int BH = B * H;
+  const int splits = plan_splits(BH, static_cast<int>(rows), cache_len);
+  const size_t need = cache_ws_bytes(splits, BH, static_cast<int>(rows), d);
+  if (need > 0) {
+    if (workspace == nullptr || ws_bytes < need)
+      return fail(MW_ERR_WORKSPACE, "workspace %zu bytes, need %zu", ws_bytes, need);
+    if (reinterpret_cast<uintptr_t>(workspace) & 255u)
+      return fail(MW_ERR_INVALID_ARG, "workspace is not 256-byte aligned");
+  }
+  return fwd_common(q, k_new, v_new, k_cache, v_cache, cache_cap, cache_head, cache_len, o, lse,
+                    need > 0 ? workspace : nullptr, ws_bytes, BH, static_cast<int>(rows), T_chunk,
+                    d, scale, splits, static_cast<cudaStream_t>(stream));
+}
+
+mw_status mw_bca_cache_commit(void* k_cache, void* v_cache, int cache_cap, int slot_start,
+                              const void* k_src, const void* v_src, int rows, int B, int H, int d,
+                              void* stream) {
+  MW_TRY(check_dims(B, H, d));
+  if (cache_cap < 1 || cache_cap > (1 << 24))
+    return fail(MW_ERR_INVALID_ARG, "cache_cap=%d out of range [1, 2^24]", cache_cap);
+  if (slot_start < 0 || slot_start >= cache_cap)
+    return fail(MW_ERR_INVALID_ARG, "slot_start=%d not in [0, cache_cap=%d)", slot_start, cache_cap);
+  if (rows < 1 || rows > cache_cap)
+    return fail(MW_ERR_INVALID_ARG, "rows=%d not in [1, cache_cap=%d]", rows, cache_cap);
+  MW_TRY(check_ptr(k_cache, "k_cache"));
+  MW_TRY(check_ptr(v_cache, "v_cache"));
+  MW_TRY(check_ptr(k_src, "k_src"));
+  MW_TRY(check_ptr(v_src, "v_src"));
+  DeviceScope scope(static_cast<cudaStream_t>(stream));
+  MW_TRY(scope.status());
+  return launch_status(
+      mw::launch_commit(d, static_cast<__nv_bfloat16*>(k_cache), static_cast<__nv_bfloat16*>(v_cache),
+                        static_cast<const __nv_bfloat16*>(k_src),
+                        static_cast<const __nv_bfloat16*>(v_src), cache_cap, slot_start, rows,
+                        B * H, static_cast<cudaStream_t>(stream)),
+      "commit kernel launch");
+}
+
+mw_status mw_device_status(void* stream, int clear) {
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  DeviceScope scope(s);
+  MW_TRY(scope.status());
+  unsigned* ptr = nullptr;
+  MW_TRY(status_ptr(&ptr));
+  cudaError_t e = cudaStreamSynchronize(s);
+  if (e != cudaSuccess) return fail(MW_ERR_CUDA, "cudaStreamSynchronize: %s", cudaGetErrorString(e));
+  unsigned word = 0;
+  e = cudaMemcpy(&word, ptr, sizeof(word), cudaMemcpyDeviceToHost);
+  if (e != cudaSuccess) return fail(MW_ERR_CUDA, "reading the status word: %s", cudaGetErrorString(e));
+  if (clear) {
+    e = cudaMemset(ptr, 0, sizeof(unsigned));
+    if (e != cudaSuccess) return fail(MW_ERR_CUDA, "clearing the status word: %s", cudaGetErrorString(e));
+  }
+  if (word & mw::kDevTimeout) return fail(MW_ERR_TIMEOUT, "a kernel wait expired (status 0x%x)", word);
+  if (word) return fail(MW_ERR_CUDA, "device status 0x%x (misaligned shared memory)", word);
+  return ok();
+}
+
+}  // extern "C"

@@ -1,0 +1,471 @@
+// Block-causal attention forward on sm_103a (Sec. 3.2 block-causal
+// self-attention; Sec. 3.5 rolling KV cache and pipelined denoising).
+//
+// One CTA owns a block of 2 x 128 query rows of one (b,h) and streams the key
+// tiles that block can see.  Only unmasked work is enumerated: the key range
+// of a query block ends at the end of the chunk of its last row, so whole
+// chunk blocks above the diagonal are never visited; a per-row limit masks
+// the few tiles that straddle a chunk edge.
+//
+// Roles (320 threads):
+//   warps 0-3 / 4-7  softmax of query tile 0 / 1 (one thread per row = TMEM lane)
+//   warp 8           TMA producer (Q once, then K/V tiles through a ring of stages)
+//   warp 9           tcgen05 issuer (S = Q K^T into TMEM, O += P V with P in TMEM)
+// TMEM (512 columns): S_t at column 128 t (P_t, bf16, overwrites its first 64
+// columns), O_t at 256 + D t.
+#include "mw_internal.h"
+#include "mw_ptx.cuh"
+
+namespace mw {
+namespace {
+
+template <int D>
+struct FwdLayout {
+  static constexpr int QT = kFwdQTiles;
+  static constexpr int REG = D / 64;                  // 64-column swizzle regions per row
+  static constexpr int REGION_BYTES = kTileRows * 128;
+  static constexpr int TILE_BYTES = REG * REGION_BYTES;
+  static constexpr int STAGES = (D == 64) ? 4 : 2;
+  static constexpr int OFF_Q = 0;
+  static constexpr int OFF_K = OFF_Q + QT * TILE_BYTES;
+  static constexpr int OFF_V = OFF_K + STAGES * TILE_BYTES;
+  static constexpr int OFF_BAR = OFF_V + STAGES * TILE_BYTES;
+  static constexpr int NBAR = 1 + 4 * STAGES + 2 * QT + 1;
+  static constexpr int OFF_MISC = OFF_BAR + NBAR * 8;
+  static constexpr int BYTES = OFF_MISC + 16;
+  static constexpr uint32_t S_COL(int t) { return 128u * t; }
+  static constexpr uint32_t O_COL(int t) { return 256u + D * t; }
+  static constexpr int THREADS = 320;
+};
+
+// Where key tile j of a query block comes from.
+struct TileSrc {
+  bool ring;   // ring buffer (segments A, B) or the queries' own keys (C)
+  int row0;    // first physical row of the tile
+  int end;     // ring: exclusive end of the valid rows; C: unused
+};
+
+struct Segs {
+  int nA, nB, nC;
+  int headA, endA, endB;
+};
+
+__device__ __forceinline__ TileSrc tile_src(const Segs& g, int j) {
+  TileSrc s;
+  if (j < g.nA) {
+    s.ring = true;
+    s.row0 = g.headA + j * kTileRows;
+    s.end = g.endA;
+  } else if (j < g.nA + g.nB) {
+    s.ring = true;
+    s.row0 = (j - g.nA) * kTileRows;
+    s.end = g.endB;
+  } else {
+    s.ring = false;
+    s.row0 = (j - g.nA - g.nB) * kTileRows;
+    s.end = 0;
+  }
+  return s;
+}
+
+template <int D>
+__global__ void __launch_bounds__(FwdLayout<D>::THREADS, 1)
+    bca_fwd_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_k,
+                   const __grid_constant__ CUtensorMap tm_v, const __grid_constant__ CUtensorMap tm_kr,
+                   const __grid_constant__ CUtensorMap tm_vr, const FwdParams p) {
+  using L = FwdLayout<D>;
+  constexpr int QT = L::QT;
+  constexpr int NS = L::STAGES;
+  extern __shared__ __align__(1024) uint8_t smem[];
+  if ((smem_u32(smem) & 1023u) != 0u) {
+    if (threadIdx.x == 0) atomicOr(p.status, kDevMisaligned);
+    return;  // uniform across the CTA, before any barrier or TMEM use
+  }
+  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + L::OFF_BAR);
+  uint64_t* q_full = bars;
+  uint64_t* k_full = bars + 1;
+  uint64_t* k_empty = k_full + NS;
+  uint64_t* v_full = k_empty + NS;
+  uint64_t* v_empty = v_full + NS;
+  uint64_t* s_full = v_empty + NS;
+  uint64_t* p_full = s_full + QT;
+  uint64_t* o_full = p_full + QT;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + L::OFF_MISC);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + L::OFF_MISC + 4);
+
+  const int warp = threadIdx.x >> 5;
+  const int lane = threadIdx.x & 31;
+
+  // ---- work item: longest query blocks first (they see the most keys)
+  int x = blockIdx.x;
+  const int split = x % p.num_splits;
+  x /= p.num_splits;
+  const int bh = x % p.BH;
+  const int qb = p.n_qblocks - 1 - x / p.BH;
+  const int r0 = qb * kFwdBlockRows;
+  const int last_row = min(r0 + kFwdBlockRows - 1, p.rows_q - 1);
+  const int c_end = (last_row / p.T + 1) * p.T;  // keys of segment C visible to the block
+
+  Segs g;
+  const int lenA = min(p.ring_len, p.ring_cap - p.ring_head);
+  const int lenB = p.ring_len - lenA;
+  g.nA = (lenA + kTileRows - 1) / kTileRows;
+  g.nB = (lenB + kTileRows - 1) / kTileRows;
+  g.nC = (c_end + kTileRows - 1) / kTileRows;
+  g.headA = p.ring_head;
+  g.endA = p.ring_head + lenA;
+  g.endB = lenB;
+  const int n_all = g.nA + g.nB + g.nC;
+  const int j0 = (int)((long long)split * n_all / p.num_splits);
+  const int j1 = (int)((long long)(split + 1) * n_all / p.num_splits);
+  const int n_local = j1 - j0;
+
+  if (threadIdx.x == 0) {
+    mbar_init(q_full, 1);
+    for (int s = 0; s < NS; ++s) {
+      mbar_init(&k_full[s], 1);
+      mbar_init(&k_empty[s], 1);
+      mbar_init(&v_full[s], 1);
+      mbar_init(&v_empty[s], 1);
+    }
+    for (int t = 0; t < QT; ++t) {
+      mbar_init(&s_full[t], 1);
+      mbar_init(&p_full[t], 4);
+    }
+    mbar_init(o_full, 1);
+    *abort_flag = 0;
+    fence_mbar_init();
+  }
+  if (warp == 9) {
+    tmem_alloc(tmem_slot, 512);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+  const WaitCtl ctl{abort_flag, p.status, p.budget_ns};
+
+  uint8_t* sQ = smem + L::OFF_Q;
+  uint8_t* sK = smem + L::OFF_K;
+  uint8_t* sV = smem + L::OFF_V;
+
+  if (warp == 8) {
+    // ------------------------------------------------------------ TMA producer
+    if (lane == 0 && n_local > 0) {
+      prefetch_tmap(&tm_q);
+      prefetch_tmap(&tm_k);
+      prefetch_tmap(&tm_v);
+      bool q_issued = false;
+      if (!p.debug_skip_q) {
+        mbar_arrive_expect_tx(q_full, QT * L::TILE_BYTES);
+        for (int t = 0; t < QT; ++t)
+          for (int r = 0; r < L::REG; ++r)
+            tma_load_3d(sQ + t * L::TILE_BYTES + r * L::REGION_BYTES, &tm_q, q_full, 64 * r,
+                        r0 + kTileRows * t, bh);
+        q_issued = true;
+      }
+      int issued_k = 0, issued_v = 0;
+      for (int i = 0; i < n_local; ++i) {
+        const int st = i % NS;
+        const uint32_t ph = (i / NS) & 1;
+        const TileSrc src = tile_src(g, j0 + i);
+        if (!mbar_wait(&k_empty[st], ph ^ 1, ctl)) break;
+        mbar_arrive_expect_tx(&k_full[st], L::TILE_BYTES);
+        for (int r = 0; r < L::REG; ++r)
+          tma_load_3d(sK + st * L::TILE_BYTES + r * L::REGION_BYTES, src.ring ? &tm_kr : &tm_k,
+                      &k_full[st], 64 * r, src.row0, bh);
+        ++issued_k;
+        if (!mbar_wait(&v_empty[st], ph ^ 1, ctl)) break;
+        mbar_arrive_expect_tx(&v_full[st], L::TILE_BYTES);
+        for (int r = 0; r < L::REG; ++r)
+          tma_load_3d(sV + st * L::TILE_BYTES + r * L::REGION_BYTES, src.ring ? &tm_vr : &tm_v,
+                      &v_full[st], 64 * r, src.row0, bh);
+        ++issued_v;
+      }
+      if (*abort_flag) {
+        // let every copy this CTA started land before shared memory goes away
+        if (q_issued) drain_wait(q_full, 0, p.budget_ns);
+        for (int i = max(0, issued_k - NS); i < issued_k; ++i)
+          drain_wait(&k_full[i % NS], (i / NS) & 1, p.budget_ns);
+        for (int i = max(0, issued_v - NS); i < issued_v; ++i)
+          drain_wait(&v_full[i % NS], (i / NS) & 1, p.budget_ns);
+      }
+    }
+  } else if (warp == 9) {
+    // ------------------------------------------------------------ MMA issuer
+    if (lane == 0 && n_local > 0) {
+      constexpr uint32_t idesc_qk = idesc_bf16_f32(128, 128, false, false);
+      constexpr uint32_t idesc_pv = idesc_bf16_f32(128, D, false, true);
+      const uint32_t q_base = smem_u32(sQ), k_base = smem_u32(sK), v_base = smem_u32(sV);
+
+      auto issue_qk = [&](int t, int st) {
+        const uint32_t qa = q_base + t * L::TILE_BYTES;
+        const uint32_t kb = k_base + st * L::TILE_BYTES;
+#pragma unroll
+        for (int kk = 0; kk < D / 16; ++kk) {
+          const uint32_t off = (kk >> 2) * L::REGION_BYTES + (kk & 3) * 32;
+          umma_ss(tmem + L::S_COL(t), sdesc_sw128(qa + off, 16, 1024), sdesc_sw128(kb + off, 16, 1024),
+                  idesc_qk, kk > 0 ? 1u : 0u);
+        }
+      };
+      auto issue_pv = [&](int t, int st, bool acc) {
+        const uint32_t vb = v_base + st * L::TILE_BYTES;
+#pragma unroll
+        for (int kk = 0; kk < kTileRows / 16; ++kk) {
+          umma_ts(tmem + L::O_COL(t), tmem + L::S_COL(t) + kk * 8,
+                  sdesc_sw128(vb + kk * 2048, L::REGION_BYTES, 1024), idesc_pv,
+                  (acc || kk > 0) ? 1u : 0u);
+        }
+      };
+
+      bool ok = mbar_wait(q_full, 0, ctl);
+      tc_fence_after();
+      for (int i = 0; ok && i < n_local; ++i) {
+        const int st = i % NS;
+        const uint32_t ph = (i / NS) & 1;
+        const int stp = (i + NS - 1) % NS;
+        const uint32_t php = ((i - 1) / NS) & 1;
+        if (!(ok = mbar_wait(&k_full[st], ph, ctl))) break;
+        tc_fence_after();
+        for (int t = 0; t < QT; ++t) {
+          if (i > 0) {
+            if (!(ok = mbar_wait(&p_full[t], (i - 1) & 1, ctl))) break;
+            if (t == 0 && !(ok = mbar_wait(&v_full[stp], php, ctl))) break;
+            tc_fence_after();
+            issue_pv(t, stp, i - 1 > 0);
+          }
+          issue_qk(t, st);
+          umma_commit(&s_full[t]);
+        }
+        if (!ok) break;
+        umma_commit(&k_empty[st]);
+        if (i > 0) umma_commit(&v_empty[stp]);
+      }
+      if (ok) {
+        const int il = n_local - 1;
+        const int stl = il % NS;
+        for (int t = 0; ok && t < QT; ++t) {
+          if (!(ok = mbar_wait(&p_full[t], il & 1, ctl))) break;
+          if (t == 0 && !(ok = mbar_wait(&v_full[stl], (il / NS) & 1, ctl))) break;
+          tc_fence_after();
+          issue_pv(t, stl, il > 0);
+        }
+        if (ok) {
+          umma_commit(&v_empty[stl]);
+          umma_commit(o_full);
+        }
+      }
+    }
+  } else {
+    // ------------------------------------------------------------ softmax
+    const int t = warp >> 2;
+    const int wq = warp & 3;
+    const int row_local = wq * 32 + lane;
+    const int row = r0 + t * kTileRows + row_local;
+    const bool row_valid = row < p.rows_q;
+    const int c_limit = (min(row, p.rows_q - 1) / p.T + 1) * p.T;
+    const uint32_t lane_base = tmem + (static_cast<uint32_t>(wq * 32) << 16);
+    const uint32_t s_addr = lane_base + L::S_COL(t);
+    const uint32_t o_addr = lane_base + L::O_COL(t);
+    const float sl2 = p.scale_log2;
+
+    float m_used = -INFINITY;
+    float l = 0.f;
+    bool ok = true;
+    for (int i = 0; i < n_local; ++i) {
+      const TileSrc src = tile_src(g, j0 + i);
+      if (!(ok = warp_wait(&s_full[t], i & 1, ctl))) break;
+      tc_fence_after();
+      float s[128];
+#pragma unroll
+      for (int c = 0; c < 4; ++c) {
+        uint32_t r[32];
+        tmem_ld32(s_addr + 32 * c, r);
+        tmem_wait_ld();
+#pragma unroll
+        for (int k = 0; k < 32; ++k) s[32 * c + k] = __uint_as_float(r[k]);
+      }
+      const int limit = (src.ring ? src.end : c_limit) - src.row0;
+      if (limit < kTileRows) {
+#pragma unroll
+        for (int c = 0; c < 128; ++c)
+          if (c >= limit) s[c] = -INFINITY;
+      }
+      float mx = s[0];
+#pragma unroll
+      for (int c = 1; c < 128; ++c) mx = fmaxf(mx, s[c]);
+      const float m_tile = mx * sl2;  // scale > 0
+      const float m_cand = fmaxf(m_used, m_tile);
+      // Rescale only when the running maximum grew by more than 2^8: P stays
+      // below 256 in between, and the final O / l is exact either way.
+      const bool need = m_cand > m_used + 8.0f;
+      if (__any_sync(0xffffffffu, need)) {
+        float alpha = 1.f;
+        if (need) {
+          alpha = ex2_approx(m_used - m_cand);
+          m_used = m_cand;
+        }
+        l *= alpha;
+        if (i > 0) {
+#pragma unroll
+          for (int c = 0; c < D / 32; ++c) {
+            uint32_t r[32];
+            tmem_ld32(o_addr + 32 * c, r);
+            tmem_wait_ld();
+#pragma unroll
+            for (int k = 0; k < 32; ++k) r[k] = __float_as_uint(__uint_as_float(r[k]) * alpha);
+            tmem_st32(o_addr + 32 * c, r);
+          }
+          tmem_wait_st();
+        }
+      }
+      const float m_eff = (m_used == -INFINITY) ? 0.f : m_used;
+      float rs = 0.f;
+#pragma unroll
+      for (int h = 0; h < 2; ++h) {
+        uint32_t packed[32];
+#pragma unroll
+        for (int k = 0; k < 32; ++k) {
+          const float p0 = ex2_approx(fmaf(s[64 * h + 2 * k], sl2, -m_eff));
+          const float p1 = ex2_approx(fmaf(s[64 * h + 2 * k + 1], sl2, -m_eff));
+          const uint32_t pk = pack_bf16x2(p0, p1);
+          // the row sum uses the bf16 weights the PV MMA consumes, so O is an
+          // exact convex combination of them
+          rs += __uint_as_float(pk << 16) + __uint_as_float(pk & 0xffff0000u);
+          packed[k] = pk;
+        }
+        tmem_st32(s_addr + 32 * h, packed);
+      }
+      l += rs;
+      tmem_wait_st();
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&p_full[t]);
+    }
+
+    // ---- epilogue
+    const bool have = __all_sync(0xffffffffu, ok) && n_local > 0 && warp_wait(o_full, 0, ctl);
+    tc_fence_after();
+    const bool nonzero = have && l > 0.f;
+    const float inv_l = nonzero ? 1.f / l : 0.f;
+    const float m_eff = (m_used == -INFINITY) ? 0.f : m_used;
+    const float lse = nonzero ? (m_eff + __log2f(l)) * 0.69314718055994530942f : -INFINITY;
+    const size_t row_off = static_cast<size_t>(bh) * p.rows_q + row;
+#pragma unroll
+    for (int c = 0; c < D / 32; ++c) {
+      uint32_t r[32];
+      if (have) {
+        tmem_ld32(o_addr + 32 * c, r);
+        tmem_wait_ld();
+      }
+      if (!row_valid) continue;
+      float v[32];
+#pragma unroll
+      for (int k = 0; k < 32; ++k) v[k] = nonzero ? __uint_as_float(r[k]) * inv_l : 0.f;
+      if (p.num_splits == 1) {
+        uint4* dst = reinterpret_cast<uint4*>(p.o + row_off * D + 32 * c);
+#pragma unroll
+        for (int k = 0; k < 4; ++k)
+          dst[k] = make_uint4(pack_bf16x2(v[8 * k], v[8 * k + 1]), pack_bf16x2(v[8 * k + 2], v[8 * k + 3]),
+                              pack_bf16x2(v[8 * k + 4], v[8 * k + 5]),
+                              pack_bf16x2(v[8 * k + 6], v[8 * k + 7]));
+      } else {
+        float4* dst = reinterpret_cast<float4*>(
+            p.o_part + (static_cast<size_t>(split) * p.BH * p.rows_q + row_off) * D + 32 * c);
+#pragma unroll
+        for (int k = 0; k < 8; ++k) dst[k] = make_float4(v[4 * k], v[4 * k + 1], v[4 * k + 2], v[4 * k + 3]);
+      }
+    }
+    if (row_valid) {
+      if (p.num_splits == 1) {
+        if (p.lse) p.lse[row_off] = lse;
+      } else {
+        p.lse_part[static_cast<size_t>(split) * p.BH * p.rows_q + row_off] = lse;
+      }
+    }
+  }
+
+  __syncwarp();
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 9) {
+    tc_fence_after();
+    tmem_dealloc(tmem, 512);
+  }
+}
+
+// Merge of split-KV partials (per row): LSE = ln sum_s exp(LSE_s),
+// O = sum_s exp(LSE_s - LSE) O_s.  One warp per row.
+template <int D>
+__global__ void __launch_bounds__(256) combine_kernel(const float* __restrict__ o_part,
+                                                      const float* __restrict__ lse_part,
+                                                      __nv_bfloat16* __restrict__ o,
+                                                      float* __restrict__ lse, int splits,
+                                                      int n_rows) {
+  const int row = blockIdx.x * 8 + (threadIdx.x >> 5);
+  const int lane = threadIdx.x & 31;
+  if (row >= n_rows) return;
+  float m = -INFINITY;
+  for (int s = 0; s < splits; ++s) m = fmaxf(m, lse_part[static_cast<size_t>(s) * n_rows + row]);
+  constexpr int PER = D / 32;
+  float acc[PER];
+#pragma unroll
+  for (int k = 0; k < PER; ++k) acc[k] = 0.f;
+  float wsum = 0.f;
+  for (int s = 0; s < splits; ++s) {
+    const float ls = lse_part[static_cast<size_t>(s) * n_rows + row];
+    if (ls == -INFINITY) continue;
+    const float w = __expf(ls - m);
+    wsum += w;
+    const float* src = o_part + (static_cast<size_t>(s) * n_rows + row) * D + lane * PER;
+#pragma unroll
+    for (int k = 0; k < PER; ++k) acc[k] += w * src[k];
+  }
+  const float inv = wsum > 0.f ? 1.f / wsum : 0.f;
+  __nv_bfloat16* dst = o + static_cast<size_t>(row) * D + lane * PER;
+#pragma unroll
+  for (int k = 0; k < PER; k += 2) {
+    *reinterpret_cast<uint32_t*>(dst + k) = pack_bf16x2(acc[k] * inv, acc[k + 1] * inv);
+  }
+  if (lse && lane == 0) lse[row] = wsum > 0.f ? m + __logf(wsum) : -INFINITY;
+}
+
+template <int D>
+cudaError_t launch_fwd_t(const CUtensorMap& tq, const CUtensorMap& tk, const CUtensorMap& tv,
+                         const CUtensorMap& tkr, const CUtensorMap& tvr, const FwdParams& p,
+                         cudaStream_t s) {
+  using L = FwdLayout<D>;
+  static bool attr_set = false;  // per process; the attribute is per function
+  if (!attr_set) {
+    cudaError_t e = cudaFuncSetAttribute(bca_fwd_kernel<D>,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize, L::BYTES);
+    if (e != cudaSuccess) return e;
+    attr_set = true;
+  }
+  const unsigned grid = static_cast<unsigned>(p.BH) * p.n_qblocks * p.num_splits;
+  bca_fwd_kernel<D><<<grid, L::THREADS, L::BYTES, s>>>(tq, tk, tv, tkr, tvr, p);
+  return cudaGetLastError();
+}
+
+}  // namespace
+
+cudaError_t launch_fwd(int d, const CUtensorMap& tq, const CUtensorMap& tk, const CUtensorMap& tv,
+                       const CUtensorMap& tkr, const CUtensorMap& tvr, const FwdParams& p,
+                       cudaStream_t s) {
+  if (d == 64) return launch_fwd_t<64>(tq, tk, tv, tkr, tvr, p, s);
+  return launch_fwd_t<128>(tq, tk, tv, tkr, tvr, p, s);
+}
+
+cudaError_t launch_combine(int d, const float* o_part, const float* lse_part, __nv_bfloat16* o,
+                           float* lse, int splits, int BH, int rows, cudaStream_t s) {
+  const int n_rows = BH * rows;
+  const unsigned grid = static_cast<unsigned>((n_rows + 7) / 8);
+  if (d == 64)
+    combine_kernel<64><<<grid, 256, 0, s>>>(o_part, lse_part, o, lse, splits, n_rows);
+  else
+    combine_kernel<128><<<grid, 256, 0, s>>>(o_part, lse_part, o, lse, splits, n_rows);
+  return cudaGetLastError();
+}
+
+}  // namespace mw

@@ -1,0 +1,76 @@
+// Internal interfaces between the C-ABI layer and the CUDA kernels.
+#pragma once
+
+#include <cuda.h>
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+namespace mw {
+
+// Rows of one query tile / key tile (the tcgen05 M and N of S = Q K^T).
+constexpr int kTileRows = 128;
+// Query tiles that share one key/value stream inside a forward CTA.
+constexpr int kFwdQTiles = 2;
+constexpr int kFwdBlockRows = kTileRows * kFwdQTiles;
+constexpr int kMaxSplits = 16;
+
+// Forward over one (b,h) query block against up to three key segments:
+//   A: ring rows [head, head + lenA)        (committed history, all visible)
+//   B: ring rows [0, lenB)                  (the part after the wrap)
+//   C: the queries' own rows [0, rows_q)    (chunk-causal: key < (chunk(i)+1) T)
+// Training uses C only (ring_len = 0).
+struct FwdParams {
+  int BH;
+  int rows_q;       // query rows (= rows of segment C) per (b,h)
+  int T;            // chunk length in tokens
+  int n_qblocks;    // ceil(rows_q / kFwdBlockRows)
+  int ring_cap;
+  int ring_head;
+  int ring_len;
+  int num_splits;   // 1: write bf16 O + LSE; >1: fp32 partials for the combine
+  float scale_log2; // softmax scale * log2(e)
+  __nv_bfloat16* o;
+  float* lse;       // nullable
+  float* o_part;    // [splits, BH, rows_q, d]
+  float* lse_part;  // [splits, BH, rows_q]
+  unsigned* status;
+  unsigned long long budget_ns;
+  int debug_skip_q;  // test hook: never load Q, so the MMA warp's wait expires
+};
+
+struct BwdParams {
+  int BH;
+  int N;            // tokens per (b,h)
+  int N_pad;        // N rounded up to kTileRows
+  int T;
+  float scale_log2;
+  float scale;
+  const float* lse2;   // [BH, N_pad]  LSE * log2(e); +inf on padding rows
+  const float* delta;  // [BH, N_pad]  rowsum(dO * O); 0 on padding rows
+  float* dq_acc;       // [BH, N_pad, d] fp32
+  __nv_bfloat16* dk;
+  __nv_bfloat16* dv;
+  unsigned* status;
+  unsigned long long budget_ns;
+};
+
+// Launchers (return cudaGetLastError() of the launch).
+cudaError_t launch_fwd(int d, const CUtensorMap& tq, const CUtensorMap& tk, const CUtensorMap& tv,
+                       const CUtensorMap& tkr, const CUtensorMap& tvr, const FwdParams& p,
+                       cudaStream_t s);
+cudaError_t launch_combine(int d, const float* o_part, const float* lse_part, __nv_bfloat16* o,
+                           float* lse, int splits, int BH, int rows, cudaStream_t s);
+cudaError_t launch_bwd_pre(int d, const __nv_bfloat16* o, const __nv_bfloat16* dout,
+                           const float* lse, float* lse2, float* delta, float* dq_acc, int BH,
+                           int N, int N_pad, cudaStream_t s);
+cudaError_t launch_bwd_main(int d, const CUtensorMap& tq, const CUtensorMap& tk,
+                            const CUtensorMap& tv, const CUtensorMap& tdo, const BwdParams& p,
+                            cudaStream_t s);
+cudaError_t launch_bwd_post(int d, const float* dq_acc, __nv_bfloat16* dq, float scale, int BH,
+                            int N, int N_pad, cudaStream_t s);
+cudaError_t launch_commit(int d, __nv_bfloat16* kc, __nv_bfloat16* vc, const __nv_bfloat16* ks,
+                          const __nv_bfloat16* vs, int cap, int slot, int rows, int BH,
+                          cudaStream_t s);
+
+}  // namespace mw

@@ -1,0 +1,152 @@
+"""C-ABI checks that need no GPU: the library builds for sm_103a, loads,
+exports every entry point the header declares, and rejects bad arguments
+with the documented status codes before touching the device."""
+import ctypes
+import os
+import re
+import subprocess
+
+import pytest
+import torch
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+HEADER = os.path.join(ROOT, "include", "mw_bca.h")
+
+OK, INVALID, UNSUPPORTED, CUDA, TIMEOUT, WORKSPACE = range(6)
+FAKE = ctypes.c_void_p(0x10000)        # aligned, never dereferenced on these paths
+MISALIGNED = ctypes.c_void_p(0x10008)
+
+
+@pytest.fixture(scope="module")
+def mw():
+    from paper_2608_01127_gb300 import _build
+    _build.build()
+    import paper_2608_01127_gb300 as pkg
+    pkg.library()
+    return pkg
+
+
+def _declared():
+    with open(HEADER) as f:
+        text = f.read()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    return sorted(set(re.findall(r"\b(mw_[a-z_]+)\s*\(", text)))
+
+
+def test_header_declares_the_python_exports(mw):
+    assert _declared() == sorted(mw.EXPORTED_SYMBOLS)
+
+
+def test_library_exports_every_declared_symbol(mw):
+    out = subprocess.run(["nm", "-D", "--defined-only", mw.lib_path], capture_output=True,
+                         text=True, check=True).stdout
+    exported = set(re.findall(r" T (mw_\w+)$", out, flags=re.M))
+    for name in _declared():
+        assert name in exported, name
+        assert hasattr(mw.library(), name)
+
+
+def test_status_strings(mw):
+    lib = mw.library()
+    for code, name in mw.STATUS.items():
+        assert lib.mw_status_string(code).decode() == name
+
+
+def test_fwd_rejects_bad_arguments(mw):
+    lib = mw.library()
+    args = dict(q=FAKE, k=FAKE, v=FAKE, o=FAKE, lse=None, B=1, H=1, n=2, T=64, d=64, s=0.125)
+
+    def call(**kw):
+        a = {**args, **kw}
+        return lib.mw_bca_fwd(a["q"], a["k"], a["v"], a["o"], a["lse"], a["B"], a["H"], a["n"],
+                              a["T"], a["d"], a["s"], None)
+
+    assert call(q=None) == INVALID
+    assert call(o=None) == INVALID
+    assert call(k=MISALIGNED) == INVALID
+    assert call(d=96) == UNSUPPORTED
+    assert call(d=0) == UNSUPPORTED
+    assert call(B=0) == INVALID
+    assert call(T=0) == INVALID
+    assert call(n=0) == INVALID
+    assert call(n=1 << 15, T=1 << 10) == INVALID   # 2^25 tokens
+    assert call(s=0.0) == INVALID
+    assert call(s=-1.0) == INVALID
+    assert "scale" in lib.mw_last_error().decode()
+
+
+def test_bwd_rejects_bad_arguments_and_workspace(mw):
+    lib = mw.library()
+    B, H, n, T, d = 1, 2, 3, 50, 64
+    need = lib.mw_bca_bwd_workspace_size(B, H, n, T, d)
+    # dQ accumulator (fp32, rows padded to 128) + two fp32 row vectors, 256-byte aligned
+    assert need == 2 * 256 * 64 * 4 + 2 * 256 * 4 + 2 * 256 * 4
+    assert lib.mw_bca_bwd_workspace_size(B, H, n, T, 96) == 0
+
+    def call(ws=FAKE, ws_bytes=need, lse=FAKE, d=d):
+        return lib.mw_bca_bwd(FAKE, FAKE, FAKE, FAKE, lse, FAKE, FAKE, FAKE, FAKE, ws, ws_bytes,
+                              B, H, n, T, d, 0.125, None)
+
+    assert call(ws=None) == WORKSPACE
+    assert call(ws_bytes=need - 1) == WORKSPACE
+    assert call(ws=ctypes.c_void_p(0x10010)) == INVALID   # not 256-byte aligned
+    assert call(lse=None) == INVALID
+    assert call(d=32) == UNSUPPORTED
+
+
+def test_cache_rejects_bad_ring_state(mw):
+    lib = mw.library()
+
+    def call(cap=1024, head=0, length=1024, kc=FAKE, B=1, H=2, W=1, T=64, d=128):
+        return lib.mw_bca_cache_fwd(FAKE, FAKE, FAKE, kc, FAKE, cap, head, length, FAKE, None,
+                                    None, 0, B, H, W, T, d, 0.1, None)
+
+    assert call(head=1024) == INVALID
+    assert call(head=-1) == INVALID
+    assert call(length=1025) == INVALID
+    assert call(length=-1) == INVALID
+    assert call(cap=0, head=0, length=0) == INVALID
+    assert call(kc=None) == INVALID
+    assert call(d=80) == UNSUPPORTED
+    assert call(T=0) == INVALID
+
+
+def test_commit_rejects_bad_slots(mw):
+    lib = mw.library()
+
+    def call(cap=100, slot=0, rows=10, src=FAKE):
+        return lib.mw_bca_cache_commit(FAKE, FAKE, cap, slot, src, FAKE, rows, 1, 1, 64, None)
+
+    assert call(slot=100) == INVALID
+    assert call(slot=-3) == INVALID
+    assert call(rows=0) == INVALID
+    assert call(rows=101) == INVALID
+    assert call(src=None) == INVALID
+    assert call(src=MISALIGNED) == INVALID
+
+
+def test_options(mw):
+    lib = mw.library()
+    assert lib.mw_set_option(b"no_such_option", 1) == INVALID
+    assert lib.mw_set_option(b"cache_splits", -1) == INVALID
+    assert lib.mw_set_option(b"cache_splits", 99) == INVALID
+    assert lib.mw_set_option(b"wait_budget_ms", 0) == INVALID
+    assert lib.mw_set_option(b"cache_splits", 0) == OK
+
+
+def test_workspace_follows_split_override(mw):
+    lib = mw.library()
+    try:
+        assert lib.mw_set_option(b"cache_splits", 3) == OK
+        size = lib.mw_bca_cache_workspace_size(1, 16, 1, 880, 128, 7040)
+        assert size == 3 * 16 * 880 * 128 * 4 + ((3 * 16 * 880 * 4 + 255) // 256) * 256
+        assert lib.mw_set_option(b"cache_splits", 1) == OK
+        assert lib.mw_bca_cache_workspace_size(1, 16, 1, 880, 128, 7040) == 0
+    finally:
+        lib.mw_set_option(b"cache_splits", 0)
+
+
+def test_python_binding_has_no_cpu_path(mw):
+    q = torch.zeros(1, 1, 64, 64, dtype=torch.bfloat16)
+    with pytest.raises(ValueError):
+        mw.mw_bca_fwd(q, q, q, 64)

@@ -1,0 +1,288 @@
+"""GPU parity: the CUDA path (through the C ABI) against the fp64 oracle on
+the same seeded bf16 inputs.
+
+Tolerances (whole-tensor): O max-abs <= 2e-2 and rel-L2 <= 5e-3;
+dQ/dK/dV rel-L2 <= 1e-2; LSE |err| <= 1e-3 * max(1, |LSE|).
+"""
+import math
+
+import pytest
+import torch
+
+import oracle
+from workloads import CACHE_CONFIGS, TRAIN_CONFIGS, gen_cache, gen_train
+
+pytestmark = pytest.mark.gpu
+
+O_MAX_ABS, O_REL, G_REL, LSE_REL = 2e-2, 5e-3, 1e-2, 1e-3
+
+
+@pytest.fixture(scope="module")
+def mw():
+    if not torch.cuda.is_available():
+        pytest.fail("a CUDA device is required for the gpu tests")
+    import paper_2608_01127_gb300 as pkg
+    pkg.library()
+    torch.cuda.set_device(0)
+    # every in-kernel wait is bounded; keep the bound short so that a broken
+    # pipeline fails fast instead of stalling each CTA for the default 2 s
+    pkg.mw_set_option("wait_budget_ms", 250)
+    assert pkg.mw_device_status(clear=True) == 0
+    return pkg
+
+
+def _rel(a, ref):
+    a = a.double().cpu()
+    return float((a - ref).norm() / ref.norm().clamp_min(1e-300))
+
+
+def check_o(o, ref, what=""):
+    a = o.double().cpu()
+    max_abs = float((a - ref).abs().max())
+    rel = _rel(o, ref)
+    assert torch.isfinite(a).all(), what
+    assert max_abs <= O_MAX_ABS and rel <= O_REL, f"{what} O max-abs {max_abs:.3e} rel-L2 {rel:.3e}"
+
+
+def check_lse(lse, ref, what=""):
+    a = lse.double().cpu()
+    err = float(((a - ref).abs() / ref.abs().clamp_min(1.0)).max())
+    assert err <= LSE_REL, f"{what} LSE rel err {err:.3e}"
+
+
+def check_grad(g, ref, what=""):
+    assert torch.isfinite(g.double()).all(), what
+    rel = _rel(g, ref)
+    assert rel <= G_REL, f"{what} rel-L2 {rel:.3e}"
+
+
+def _inputs(B, H, n, T, d, seed, gain=1.0):
+    g = torch.Generator().manual_seed(seed)
+    shape = (B, H, n * T, d)
+    q, k, v, do = (torch.randn(shape, generator=g) for _ in range(4))
+    return [(t * s).to(torch.bfloat16) for t, s in ((q, gain), (k, gain), (v, 1.0), (do, 1.0))]
+
+
+# ------------------------------------------------------------------ training path
+
+def test_tiny_config_forward(mw):
+    cfg = TRAIN_CONFIGS["tiny_fwd"]
+    x = gen_train(cfg)
+    o, lse = mw.mw_bca_fwd(*(x[n].cuda() for n in ("q", "k", "v")), cfg.T, cfg.scale)
+    o_ref, lse_ref = oracle.fwd(x["q"], x["k"], x["v"], cfg.T, cfg.scale)
+    check_o(o, o_ref, "tiny")
+    check_lse(lse, lse_ref, "tiny")
+
+
+SMALL = [
+    # B, H, n_chunks, T, d, gain
+    (1, 1, 1, 16, 64, 1.0),      # fewer rows than one tile
+    (1, 2, 3, 100, 64, 1.0),     # chunk edges inside tiles, ragged tail
+    (2, 1, 4, 64, 128, 1.0),
+    (1, 1, 300, 1, 64, 1.0),     # token-causal
+    (1, 2, 20, 16, 128, 2.0),
+    (1, 1, 2, 880, 128, 4.0),    # one latent frame per chunk, peaky logits
+    (1, 3, 5, 200, 64, 1.0),
+    (2, 2, 1, 600, 128, 1.0),    # a single chunk: full bidirectional attention
+]
+
+
+@pytest.mark.parametrize("B,H,n,T,d,gain", SMALL)
+def test_small_shapes_forward_backward(mw, B, H, n, T, d, gain):
+    q, k, v, do = _inputs(B, H, n, T, d, seed=1000 + n * T + d, gain=gain)
+    sc = 1.0 / math.sqrt(d)
+    qc, kc, vc, doc = (t.cuda() for t in (q, k, v, do))
+    o, lse = mw.mw_bca_fwd(qc, kc, vc, T, sc)
+    dq, dk, dv = mw.mw_bca_bwd(qc, kc, vc, o, lse, doc, T, sc)
+    o_ref, lse_ref = oracle.fwd(q, k, v, T, sc)
+    dq_r, dk_r, dv_r = oracle.bwd(q, k, v, do, T, sc)
+    tag = f"B{B} H{H} n{n} T{T} d{d}"
+    check_o(o, o_ref, tag)
+    check_lse(lse, lse_ref, tag)
+    check_grad(dq, dq_r, tag + " dQ")
+    check_grad(dk, dk_r, tag + " dK")
+    check_grad(dv, dv_r, tag + " dV")
+
+
+@pytest.mark.parametrize("name", ["train_b12_d64", "train_h16_d128_peaky"])
+def test_full_size_training_configs(mw, name):
+    """Full-size launch; the oracle recomputes two sampled (b, h) heads in full."""
+    cfg = TRAIN_CONFIGS[name]
+    x = gen_train(cfg)
+    qc, kc, vc, doc = (x[n].cuda() for n in ("q", "k", "v", "do"))
+    o, lse = mw.mw_bca_fwd(qc, kc, vc, cfg.T, cfg.scale)
+    dq, dk, dv = mw.mw_bca_bwd(qc, kc, vc, o, lse, doc, cfg.T, cfg.scale)
+    torch.cuda.synchronize()
+    for b, h in ((0, 0), (cfg.B - 1, cfg.H - 1)):
+        sl = (slice(b, b + 1), slice(h, h + 1))
+        q, k, v, do = (x[n][sl] for n in ("q", "k", "v", "do"))
+        o_ref, lse_ref = oracle.fwd(q, k, v, cfg.T, cfg.scale)
+        dq_r, dk_r, dv_r = oracle.bwd(q, k, v, do, cfg.T, cfg.scale)
+        tag = f"{name} b{b} h{h}"
+        check_o(o[sl], o_ref, tag)
+        check_lse(lse[sl], lse_ref, tag)
+        check_grad(dq[sl], dq_r, tag + " dQ")
+        check_grad(dk[sl], dk_r, tag + " dK")
+        check_grad(dv[sl], dv_r, tag + " dV")
+    assert mw.mw_device_status() == 0
+
+
+def test_forward_is_deterministic_and_stays_in_bounds(mw):
+    B, H, n, T, d = 1, 2, 3, 100, 64
+    q, k, v, _ = _inputs(B, H, n, T, d, seed=7)
+    N = n * T
+    qc, kc, vc = (t.cuda() for t in (q, k, v))
+    # outputs carved out of NaN-filled buffers: the guard bands must survive
+    numel = B * H * N * d
+    buf = torch.full((numel + 4096,), float("nan"), dtype=torch.bfloat16, device="cuda")
+    o = buf[2048:2048 + numel].view(B, H, N, d)
+    lbuf = torch.full((B * H * N + 512,), float("nan"), dtype=torch.float32, device="cuda")
+    lse = lbuf[256:256 + B * H * N].view(B, H, N)
+    lib = mw.library()
+    s = torch.cuda.current_stream().cuda_stream
+    assert lib.mw_bca_fwd(qc.data_ptr(), kc.data_ptr(), vc.data_ptr(), o.data_ptr(),
+                          lse.data_ptr(), B, H, n, T, d, 0.125, s) == 0
+    torch.cuda.synchronize()
+    assert torch.isnan(buf[:2048]).all() and torch.isnan(buf[2048 + numel:]).all()
+    assert torch.isnan(lbuf[:256]).all() and torch.isnan(lbuf[256 + B * H * N:]).all()
+    o2, lse2 = mw.mw_bca_fwd(qc, kc, vc, T, 0.125)
+    assert torch.equal(o, o2) and torch.equal(lse, lse2)
+
+
+def test_autograd_wrapper(mw):
+    q, k, v, do = _inputs(1, 2, 3, 64, 64, seed=11)
+    qc, kc, vc = (t.cuda().requires_grad_(True) for t in (q, k, v))
+    o = mw.BlockCausalAttention.apply(qc, kc, vc, 64, None)
+    o.backward(do.cuda())
+    dq_r, dk_r, dv_r = oracle.bwd(q, k, v, do, 64, 0.125)
+    check_grad(qc.grad, dq_r, "autograd dQ")
+    check_grad(kc.grad, dk_r, "autograd dK")
+    check_grad(vc.grad, dv_r, "autograd dV")
+
+
+# ------------------------------------------------------------------ rolling cache
+
+def _ring_case(B, H, W, T, cap, d, seed, std=1.0):
+    g = torch.Generator().manual_seed(seed)
+    q, kn, vn = (torch.randn(B, H, W * T, d, generator=g).to(torch.bfloat16) for _ in range(3))
+    kr, vr = ((std * torch.randn(B, H, cap, d, generator=g)).to(torch.bfloat16) for _ in range(2))
+    return q, kn, vn, kr, vr
+
+
+CACHE_SMALL = [
+    # B, H, W, T, cap, length, head, d, splits (0 = automatic)
+    (1, 2, 1, 64, 512, 512, 100, 128, 0),
+    (1, 2, 3, 100, 1000, 300, 900, 64, 0),     # partially filled ring that wraps
+    (2, 1, 2, 64, 640, 0, 0, 128, 0),          # empty ring: training form
+    (1, 1, 1, 880, 1760, 1760, 1759, 128, 0),  # head at cap - 1
+    (1, 2, 4, 96, 1152, 1152, 576, 64, 5),     # forced split-KV
+    (1, 2, 2, 130, 780, 780, 390, 128, 1),     # forced single pass
+    (1, 1, 1, 16, 48, 40, 30, 64, 3),          # tiny ring, more splits than needed
+]
+
+
+@pytest.mark.parametrize("B,H,W,T,cap,length,head,d,splits", CACHE_SMALL)
+def test_cache_forward_small(mw, B, H, W, T, cap, length, head, d, splits):
+    q, kn, vn, kr, vr = _ring_case(B, H, W, T, cap, d, seed=cap + head + W)
+    sc = 1.0 / math.sqrt(d)
+    mw.mw_set_option("cache_splits", splits)
+    try:
+        o, lse = mw.mw_bca_cache_fwd(q.cuda(), kn.cuda(), vn.cuda(), kr.cuda(), vr.cuda(),
+                                     head, length, T, sc)
+    finally:
+        mw.mw_set_option("cache_splits", 0)
+    o_ref, lse_ref = oracle.cache_fwd(q, kn, vn, kr, vr, cap, head, length, T, sc)
+    tag = f"W{W} T{T} cap{cap} len{length} head{head} splits{splits}"
+    check_o(o, o_ref, tag)
+    check_lse(lse, lse_ref, tag)
+
+
+def test_cache_split_count_does_not_change_the_result(mw):
+    """Split-KV partials merged by the combine kernel give the unsplit result:
+    every split count matches the oracle, and the runs agree with each other
+    to within the oracle tolerance (their bf16 P roundings differ slightly
+    because each split keeps its own running maximum)."""
+    cpu = _ring_case(1, 4, 2, 200, 2400, 128, seed=5)
+    q, kn, vn, kr, vr = (t.cuda() for t in cpu)
+    o_ref, lse_ref = oracle.cache_fwd(*cpu, 2400, 1700, 2400, 200, 0.09)
+    outs = []
+    for s in (1, 2, 7):
+        mw.mw_set_option("cache_splits", s)
+        try:
+            outs.append(mw.mw_bca_cache_fwd(q, kn, vn, kr, vr, 1700, 2400, 200, 0.09))
+        finally:
+            mw.mw_set_option("cache_splits", 0)
+        check_o(outs[-1][0], o_ref, f"splits {s}")
+        check_lse(outs[-1][1], lse_ref, f"splits {s}")
+    for o, lse in outs[1:]:
+        assert float((o.float() - outs[0][0].float()).abs().max()) <= O_MAX_ABS
+        assert float(((lse - outs[0][1]).abs() / outs[0][1].abs().clamp_min(1)).max()) <= LSE_REL
+
+
+def test_ring_rotation_matches(mw):
+    """Rotating the physical ring while moving the head by the same amount is
+    invisible (the logical key order is unchanged)."""
+    cap, T = 1024, 128
+    q, kn, vn, kr, vr = _ring_case(1, 2, 1, T, cap, 128, seed=9)
+    o_ref, lse_ref = oracle.cache_fwd(q, kn, vn, kr, vr, cap, 0, cap, T, 128 ** -0.5)
+    for r in (0, 1, 300, 1023):
+        krr, vrr = torch.roll(kr, r, 2), torch.roll(vr, r, 2)
+        o, lse = mw.mw_bca_cache_fwd(q.cuda(), kn.cuda(), vn.cuda(), krr.cuda(), vrr.cuda(), r,
+                                     cap, T)
+        check_o(o, o_ref, f"rotation {r}")
+        check_lse(lse, lse_ref, f"rotation {r}")
+
+
+def test_commit_is_bit_exact(mw):
+    B, H, d, cap, rows = 2, 3, 128, 1000, 300
+    g = torch.Generator().manual_seed(3)
+    kr, vr, ks, vs = (torch.randn(B, H, n, d, generator=g).to(torch.bfloat16)
+                      for n in (cap, cap, rows, rows))
+    for slot in (0, 650, 999):
+        kg, vg = kr.cuda(), vr.cuda()
+        mw.mw_bca_cache_commit(kg, vg, slot, ks.cuda(), vs.cuda())
+        k_ref, v_ref = oracle.cache_commit(kr, vr, cap, slot, ks, vs)
+        assert torch.equal(kg.cpu(), k_ref) and torch.equal(vg.cpu(), v_ref)
+
+
+def test_rolling_cache_config_steps(mw):
+    """The streaming workload: one 880-token chunk against an 8-chunk ring
+    whose head wraps mid-buffer; each step commits the chunk (FIFO eviction)."""
+    cfg = CACHE_CONFIGS["rolling_cache"]
+    steps = 3
+    x = gen_cache(cfg, steps=steps)
+    kr, vr = x["k_ring"].clone(), x["v_ring"].clone()
+    krg, vrg = kr.cuda(), vr.cuda()
+    head, length = cfg.head, cfg.length
+    for s in range(steps):
+        q, kn, vn = x["q"][s], x["k_new"][s], x["v_new"][s]
+        o, lse = mw.mw_bca_cache_fwd(q.cuda(), kn.cuda(), vn.cuda(), krg, vrg, head, length,
+                                     cfg.T, cfg.scale)
+        o_ref, lse_ref = oracle.cache_fwd(q, kn, vn, kr, vr, cfg.cap, head, length, cfg.T,
+                                          cfg.scale)
+        check_o(o, o_ref, f"step {s}")
+        check_lse(lse, lse_ref, f"step {s}")
+        slot, head, length = oracle.ring_advance(cfg.cap, head, length, cfg.T)
+        mw.mw_bca_cache_commit(krg, vrg, slot, kn.cuda(), vn.cuda())
+        kr, vr = oracle.cache_commit(kr, vr, cfg.cap, slot, kn, vn)
+    assert torch.equal(krg.cpu(), kr) and torch.equal(vrg.cpu(), vr)
+    assert mw.mw_device_status() == 0
+
+
+def test_pipelined_config(mw):
+    """Four in-flight chunks, block-causal among themselves, against a wrapped
+    12-chunk ring with per-chunk K/V scales."""
+    cfg = CACHE_CONFIGS["pipelined"]
+    x = gen_cache(cfg)
+    q, kn, vn = x["q"][0], x["k_new"][0], x["v_new"][0]
+    o, lse = mw.mw_bca_cache_fwd(q.cuda(), kn.cuda(), vn.cuda(), x["k_ring"].cuda(),
+                                 x["v_ring"].cuda(), cfg.head, cfg.length, cfg.T, cfg.scale)
+    o_ref, lse_ref = oracle.cache_fwd(q, kn, vn, x["k_ring"], x["v_ring"], cfg.cap, cfg.head,
+                                      cfg.length, cfg.T, cfg.scale)
+    check_o(o, o_ref, "pipelined")
+    check_lse(lse, lse_ref, "pipelined")
+
+
+def test_device_status_is_clean(mw):
+    torch.cuda.synchronize()
+    assert mw.mw_device_status() == 0

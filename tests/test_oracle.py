@@ -335,3 +335,17 @@ def test_commit_is_fifo():
     src = torch.tensor([1.0, 2.0, 3.0], dtype=F64).view(1, 1, 3, 1)
     out, _ = oracle.cache_commit(ring, ring, 5, 3, src, src)
     assert out.flatten().tolist() == [3.0, 0.0, 0.0, 1.0, 2.0]
+
+
+def test_product_ring_bookkeeping_matches_oracle():
+    """The package's host-side FIFO plan agrees with the oracle's reading of
+    the rolling cache (Sec. 3.5) over fills, wraps and evictions."""
+    from paper_2608_01127_gb300 import RingState
+    for cap, head, length, rows in ((9, 0, 0, 3), (7040, 4400, 7040, 880), (10, 7, 4, 3),
+                                    (10, 9, 10, 10), (5, 2, 1, 5)):
+        ring = RingState(cap, head, length)
+        h, n = head, length
+        for _ in range(6):
+            slot, h, n = oracle.ring_advance(cap, h, n, rows)
+            assert ring.commit(rows) == slot
+            assert (ring.head, ring.length) == (h, n)
