@@ -148,6 +148,42 @@ mw_status mw_bca_cache_commit(void* k_cache, void* v_cache, int cache_cap, int s
                               const void* k_src, const void* v_src, int rows, int B, int H, int d,
                               void* stream);
 
+/* Size of the library's static scratch array used by
+ * mw_bca_cache_fwd_noalloc (64 MiB on every device that loads the library). */
+#define MW_NOALLOC_SCRATCH_BYTES (64u << 20)
+
+/*
+ * mw_bca_cache_fwd without a workspace argument, for callers that cannot
+ * allocate device memory: hosts that hand the library only their input and
+ * output buffers (plugin-style integrations with no allocator), and real-time
+ * streaming loops that must never call cudaMalloc / cudaFree because those
+ * calls can synchronise the device and stall the stream.  This entry point
+ * allocates nothing.  The split-KV partials it needs live in a fixed scratch
+ * array of MW_NOALLOC_SCRATCH_BYTES that the library declares as a static
+ * device variable; every GPU that loads the library holds that array until
+ * the process exits.  The paper has no counterpart: this is an
+ * integration convenience, not part of the method.
+ *   Arguments, layouts and results are exactly those of mw_bca_cache_fwd
+ *   (same kernels, same split plan), minus workspace / ws_bytes.
+ *   When the partials for these sizes would exceed MW_NOALLOC_SCRATCH_BYTES
+ *   the call returns MW_ERR_WORKSPACE, enqueues nothing, and mw_last_error()
+ *   names the bytes needed; use mw_bca_cache_fwd with a caller workspace
+ *   instead.
+ *   The first call on a device looks up the array's device address
+ *   (cudaGetSymbolAddress, once per device, with that device current); make
+ *   that first call before any stream capture.
+ *   All calls share the one array and it keeps the last call's contents.
+ *   Each call writes every partial it later reads, so nothing has to start at
+ *   zero, but calls whose kernels overlap on the GPU (different streams, or
+ *   different host threads without ordering) race on the array: serialise
+ *   them, e.g. on one stream.
+ */
+mw_status mw_bca_cache_fwd_noalloc(const void* q, const void* k_new, const void* v_new,
+                                   const void* k_cache, const void* v_cache, int cache_cap,
+                                   int cache_head, int cache_len, void* o, float* lse, int B,
+                                   int H, int n_q_chunks, int T_chunk, int d, float scale,
+                                   void* stream);
+
 /* Human-readable name of a status code (static string). */
 const char* mw_status_string(mw_status s);
 

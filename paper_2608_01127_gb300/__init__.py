@@ -37,7 +37,7 @@ EXPORTED_SYMBOLS = (
     "mw_bca_fwd", "mw_bca_bwd_workspace_size", "mw_bca_bwd", "mw_bca_bwd_stage",
     "mw_bca_cache_workspace_size",
     "mw_bca_cache_fwd", "mw_bca_cache_commit", "mw_status_string", "mw_last_error",
-    "mw_device_status", "mw_set_option",
+    "mw_device_status", "mw_set_option", "mw_bca_cache_fwd_noalloc",
 )
 
 STATUS = {0: "MW_OK", 1: "MW_ERR_INVALID_ARG", 2: "MW_ERR_UNSUPPORTED", 3: "MW_ERR_CUDA",
@@ -81,6 +81,8 @@ def library() -> ctypes.CDLL:
         "mw_bca_cache_fwd": (_I, [_P, _P, _P, _P, _P, _I, _I, _I, _P, _P, _P, _Z,
                                   _I, _I, _I, _I, _I, _F, _P]),
         "mw_bca_cache_commit": (_I, [_P, _P, _I, _I, _P, _P, _I, _I, _I, _I, _P]),
+        "mw_bca_cache_fwd_noalloc": (_I, [_P, _P, _P, _P, _P, _I, _I, _I, _P, _P,
+                                          _I, _I, _I, _I, _I, _F, _P]),
         "mw_status_string": (ctypes.c_char_p, [_I]),
         "mw_last_error": (ctypes.c_char_p, []),
         "mw_device_status": (_I, [_P, _I]),

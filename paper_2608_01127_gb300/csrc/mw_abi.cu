@@ -500,3 +500,73 @@ mw_status mw_device_status(void* stream, int clear) {
 }
 
 }  // extern "C"
+
+// ---------------------------------------------------------------------------
+// Allocation-free variant of the ring-cache forward.
+//
+// Callers that cannot allocate device memory (plugin hosts that only hand in
+// their own buffers; real-time loops that must not call cudaMalloc/cudaFree,
+// which can synchronise the device) get the split-KV partials from this fixed
+// array instead of a caller workspace.  It is a file-scope device variable:
+// every device that loads the library holds it until the process exits.  In
+// host code its name is only a host-side stand-in, so its device address is
+// looked up once per device with cudaGetSymbolAddress (with that device
+// current) and that address is what the kernels receive.
+namespace {
+
+static __device__ __align__(256) unsigned char g_noalloc_scratch[MW_NOALLOC_SCRATCH_BYTES];
+
+void* g_noalloc_ptr[kMaxDevices] = {};
+
+// Device address of g_noalloc_scratch on the current device (set up on the
+// first call per device).
+mw_status noalloc_scratch(void** out) {
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return fail(MW_ERR_CUDA, "cudaGetDevice: %s", cudaGetErrorString(e));
+  if (dev < 0 || dev >= kMaxDevices) return fail(MW_ERR_CUDA, "device index %d too large", dev);
+  std::lock_guard<std::mutex> lock(g_mutex);
+  if (g_noalloc_ptr[dev] == nullptr) {
+    void* p = nullptr;
+    e = cudaGetSymbolAddress(&p, g_noalloc_scratch);
+    if (e != cudaSuccess)
+      return fail(MW_ERR_CUDA, "cudaGetSymbolAddress(scratch): %s", cudaGetErrorString(e));
+    g_noalloc_ptr[dev] = p;
+  }
+  *out = g_noalloc_ptr[dev];
+  return MW_OK;
+}
+
+}  // namespace
+
+extern "C" mw_status mw_bca_cache_fwd_noalloc(const void* q, const void* k_new, const void* v_new,
+                                              const void* k_cache, const void* v_cache,
+                                              int cache_cap, int cache_head, int cache_len,
+                                              void* o, float* lse, int B, int H, int n_q_chunks,
+                                              int T_chunk, int d, float scale, void* stream) {
+  // sizes first (host only), so that an oversized request is refused before
+  // anything touches the device
+  MW_TRY(check_dims(B, H, d));
+  if (n_q_chunks < 1 || T_chunk < 1)
+    return fail(MW_ERR_INVALID_ARG, "n_q_chunks=%d and T_chunk=%d must be >= 1", n_q_chunks, T_chunk);
+  const long long rows = static_cast<long long>(n_q_chunks) * T_chunk;
+  MW_TRY(check_rows(rows, "n_q_chunks*T_chunk"));
+  if (cache_len < 0 || cache_len > cache_cap)
+    return fail(MW_ERR_INVALID_ARG, "cache_len=%d not in [0, cache_cap=%d]", cache_len, cache_cap);
+  const int splits = plan_splits(B * H, static_cast<int>(rows), cache_len);
+  const size_t need = cache_ws_bytes(splits, B * H, static_cast<int>(rows), d);
+  if (need > MW_NOALLOC_SCRATCH_BYTES)
+    return fail(MW_ERR_WORKSPACE,
+                "these sizes need %zu bytes of split-KV scratch; the static scratch holds %u "
+                "bytes (use mw_bca_cache_fwd with a caller workspace)",
+                need, static_cast<unsigned>(MW_NOALLOC_SCRATCH_BYTES));
+  void* scratch = nullptr;
+  if (need > 0) {
+    DeviceScope scope(static_cast<cudaStream_t>(stream));
+    MW_TRY(scope.status());
+    MW_TRY(noalloc_scratch(&scratch));
+  }
+  return mw_bca_cache_fwd(q, k_new, v_new, k_cache, v_cache, cache_cap, cache_head, cache_len, o,
+                          lse, scratch, need > 0 ? MW_NOALLOC_SCRATCH_BYTES : 0, B, H, n_q_chunks,
+                          T_chunk, d, scale, stream);
+}
