@@ -11,7 +11,7 @@
 #include <mutex>
 #include <string>
 
-#include "../../include/mw_bca.h"
+#include "mw_bca.h"
 #include "mw_internal.h"
 #include "mw_ptx.cuh"
 
@@ -89,14 +89,15 @@ PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
 
 // 3-D map over [BH, rows, d] bf16 with 64 x 128-row boxes and the 128-byte
 // swizzle the tcgen05 descriptors expect; rows past the end read as zero.
-mw_status make_map(CUtensorMap* m, const void* ptr, int rows, int BH, int d, const char* name) {
+mw_status make_map(CUtensorMap* m, const void* ptr, int rows, int BH, int d, const char* name,
+                   int box_rows = mw::kTileRows) {
   auto fn = encode_fn();
   if (!fn) return fail(MW_ERR_CUDA, "cuTensorMapEncodeTiled is unavailable (no CUDA driver?)");
   cuuint64_t dims[3] = {static_cast<cuuint64_t>(d), static_cast<cuuint64_t>(rows),
                         static_cast<cuuint64_t>(BH)};
   cuuint64_t strides[2] = {static_cast<cuuint64_t>(d) * 2,
                            static_cast<cuuint64_t>(rows) * d * 2};
-  cuuint32_t box[3] = {64, static_cast<cuuint32_t>(mw::kTileRows), 1};
+  cuuint32_t box[3] = {64, static_cast<cuuint32_t>(box_rows), 1};
   cuuint32_t estr[3] = {1, 1, 1};
   CUresult r = fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(ptr), dims, strides, box,
                   estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
@@ -369,10 +370,11 @@ mw_status mw_bca_bwd_stage(int stage, const void* q, const void* k, const void* 
     unsigned* status = nullptr;
     MW_TRY(status_ptr(&status));
     CUtensorMap tq, tk, tv, tdo;
-    MW_TRY(make_map(&tq, q, static_cast<int>(N), BH, d, "q"));
+    const int qrows = mw::bwd_q_rows(d);  // query rows per backward step
+    MW_TRY(make_map(&tq, q, static_cast<int>(N), BH, d, "q", qrows));
     MW_TRY(make_map(&tk, k, static_cast<int>(N), BH, d, "k"));
     MW_TRY(make_map(&tv, v, static_cast<int>(N), BH, d, "v"));
-    MW_TRY(make_map(&tdo, dout, static_cast<int>(N), BH, d, "dout"));
+    MW_TRY(make_map(&tdo, dout, static_cast<int>(N), BH, d, "dout", qrows));
     mw::BwdParams p{};
     p.BH = BH;
     p.N = static_cast<int>(N);

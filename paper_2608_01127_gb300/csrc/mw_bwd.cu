@@ -5,19 +5,30 @@
 //   pre : D_i = <dO_i, O_i>, LSE2_i = LSE_i * log2(e) (+inf on padding rows),
 //         dQacc = 0
 //   main: one CTA per 128-row key tile of one (b,h); it owns dK, dV in TMEM
-//         and visits only the query tiles whose chunks can see it
-//         (queries i >= chunk(k0) * T).  Per query tile:
-//           S^T  = K Q^T              (tcgen05, TMEM)
-//           dP^T = V dO^T             (tcgen05, TMEM)
-//           P^T  = exp2(S^T scale log2e - LSE2)       -> TMEM (bf16)
-//           dS^T = P^T (dP^T - D)                     -> shared memory (bf16)
-//           dV  += P^T dO ;  dK += dS^T Q ;  dQ_tile = dS K  (tcgen05)
-//           dQacc += dQ_tile (fp32 vector atomics)
+//         and visits only the query rows whose chunks can see it
+//         (queries i >= chunk(k0) * T), QN query rows per step j:
+//           S^T  = K Q^T                        (tcgen05 -> TMEM)
+//           dP^T = V dO^T                       (tcgen05 -> TMEM)
+//           P^T  = exp2(S^T scale log2e - LSE2) (registers)
+//           dS^T = P^T (dP^T - D)               (registers)
+//           P^T, dS^T (bf16) -> TMEM over the dP^T columns; dS^T -> smem
+//           dV += P^T dO ;  dK += dS^T Q        (tcgen05, A from TMEM)
+//           d = 64 : dQ_j = dS K    (query rows in TMEM lanes)
+//           d = 128: dQ_j^T = K^T dS^T (head-dim columns in TMEM lanes)
+//           dQacc += dQ_j  (fp32 reductions, each warp instruction covering
+//                           contiguous memory)
 //   post: dQ = scale * dQacc -> bf16
 //
-// Roles (320 threads): warps 0-3 P/dS (one thread per key row), warps 4-7
-// dQ drain (one thread per query row), warp 8 TMA producer, warp 9 MMA.
-// TMEM: dV [0, D), dK [D, 2D), S^T [2D, 2D+128), dP^T / dQ_tile [2D+128, 2D+256).
+// Software pipeline: the P/dS warps copy S^T into registers first and
+// release it, so S^T of the next step is computed while they work; dV, dK,
+// dQ of step j and dP^T of step j+1 run while they compute P of step j+1;
+// dQ has its own TMEM columns, so draining it never blocks the next step.
+//
+// Roles (512 threads): warps 0-7 P/dS (two warpgroups, one half of the query
+// columns each, one key row per thread), warps 8-11 dQ drain, warp 12 TMA
+// producer, warp 13 MMA issuer.
+// TMEM: dV [0,D), dK [D,2D), S^T [2D,2D+QN), dP^T [2D+QN,2D+2QN),
+// dQ [384,448).
 #include "mw_internal.h"
 #include "mw_ptx.cuh"
 
@@ -26,29 +37,42 @@ namespace {
 
 template <int D>
 struct BwdLayout {
-  static constexpr int REG = D / 64;
-  static constexpr int REGION_BYTES = kTileRows * 128;
-  static constexpr int TILE_BYTES = REG * REGION_BYTES;
-  static constexpr int QSTAGES = 2;
-  static constexpr int VEC_BYTES = kTileRows * 4;
+  static constexpr int QN = bwd_q_rows(D);           // query rows per step
+  static constexpr bool DQT = (D == 128);            // dQ produced transposed
+  static constexpr int CW = QN / 2;                  // query columns per P/dS warpgroup
+  static constexpr int KPW = CW / 16;                // 16-deep MMA K steps per warpgroup half
+  static constexpr int REG = D / 64;                 // 64-column swizzle regions per row
+  static constexpr int KREGION = kTileRows * 128;    // region of a 128-row tile
+  static constexpr int QREGION = QN * 128;           // region of a QN-row tile
+  static constexpr int KTILE = REG * KREGION;
+  static constexpr int QTILE = REG * QREGION;
+  static constexpr int STAGES = (D == 64) ? 3 : 4;   // Q and dO tiles in flight
+  static constexpr int DS_BYTES = (QN / 64) * KREGION;  // dS^T: 128 key rows x QN columns
+  static constexpr int DS_BUFS = (D == 64) ? 1 : 2;
+  static constexpr int STG_BYTES = DQT ? 0 : 4 * 32 * D * 4;  // per-warp dQ staging (d = 64)
+  static constexpr int VEC_BYTES = QN * 4;
   static constexpr int OFF_K = 0;
-  static constexpr int OFF_V = OFF_K + TILE_BYTES;
-  static constexpr int OFF_Q = OFF_V + TILE_BYTES;                 // QSTAGES tiles
-  static constexpr int OFF_DO = OFF_Q + QSTAGES * TILE_BYTES;      // QSTAGES tiles
-  static constexpr int OFF_DS = OFF_DO + QSTAGES * TILE_BYTES;     // 128 x 128 bf16
-  static constexpr int DS_BYTES = 2 * REGION_BYTES;
-  static constexpr int OFF_LSE = OFF_DS + DS_BYTES;                // QSTAGES x 512 B
-  static constexpr int OFF_DELTA = OFF_LSE + QSTAGES * VEC_BYTES;  // QSTAGES x 512 B
-  static constexpr int OFF_BAR = OFF_DELTA + QSTAGES * VEC_BYTES;
-  // kv_full, q_full[2], q_empty[2], st_full, dpt_full, p_ready, dq_full, dq_free, ds_free, dkv_full
-  static constexpr int NBAR = 1 + 2 * QSTAGES + 7;
+  static constexpr int OFF_V = OFF_K + KTILE;
+  static constexpr int OFF_Q = OFF_V + KTILE;
+  static constexpr int OFF_DO = OFF_Q + STAGES * QTILE;
+  static constexpr int OFF_DS = OFF_DO + STAGES * QTILE;
+  static constexpr int OFF_STG = OFF_DS + DS_BUFS * DS_BYTES;
+  static constexpr int OFF_LSE = OFF_STG + STG_BYTES;
+  static constexpr int OFF_DELTA = OFF_LSE + STAGES * VEC_BYTES;
+  static constexpr int OFF_BAR = OFF_DELTA + STAGES * VEC_BYTES;
+  // kv_full, q_full[S], q_empty[S], do_full[S], do_empty[S], s_full, s_free,
+  // dp_full, p_ready, dq_full, dq_free, ds_free[DS_BUFS], dkv_full
+  static constexpr int NBAR = 1 + 4 * STAGES + 7 + DS_BUFS;
   static constexpr int OFF_MISC = OFF_BAR + NBAR * 8;
   static constexpr int BYTES = OFF_MISC + 16;
   static constexpr uint32_t DV_COL = 0;
   static constexpr uint32_t DK_COL = D;
   static constexpr uint32_t S_COL = 2 * D;
-  static constexpr uint32_t DP_COL = 2 * D + 128;
-  static constexpr int THREADS = 320;
+  static constexpr uint32_t DP_COL = 2 * D + QN;
+  static constexpr uint32_t DQ_COL = 384;
+  static constexpr int THREADS = 512;
+  static_assert(2 * D + 2 * QN <= 384, "TMEM columns");
+  static_assert(BYTES <= 232448, "shared memory");
 };
 
 __device__ __forceinline__ void red_add_v4(float* addr, float a, float b, float c, float d) {
@@ -57,13 +81,19 @@ __device__ __forceinline__ void red_add_v4(float* addr, float a, float b, float 
                : "memory");
 }
 
+__device__ __forceinline__ void red_add(float* addr, float a) {
+  asm volatile("red.global.add.f32 [%0], %1;" ::"l"(addr), "f"(a) : "memory");
+}
+
 template <int D>
 __global__ void __launch_bounds__(BwdLayout<D>::THREADS, 1)
     bca_bwd_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_k,
                    const __grid_constant__ CUtensorMap tm_v, const __grid_constant__ CUtensorMap tm_do,
                    const BwdParams p) {
   using L = BwdLayout<D>;
-  constexpr int NS = L::QSTAGES;
+  constexpr int NS = L::STAGES;
+  constexpr int QN = L::QN;
+  constexpr int CW = L::CW;
   extern __shared__ __align__(1024) uint8_t smem[];
   if ((smem_u32(smem) & 1023u) != 0u) {
     if (threadIdx.x == 0) atomicOr(p.status, kDevMisaligned);
@@ -73,45 +103,52 @@ __global__ void __launch_bounds__(BwdLayout<D>::THREADS, 1)
   uint64_t* kv_full = bars;
   uint64_t* q_full = bars + 1;
   uint64_t* q_empty = q_full + NS;
-  uint64_t* st_full = q_empty + NS;
-  uint64_t* dpt_full = st_full + 1;
-  uint64_t* p_ready = dpt_full + 1;
+  uint64_t* do_full = q_empty + NS;
+  uint64_t* do_empty = do_full + NS;
+  uint64_t* s_full = do_empty + NS;
+  uint64_t* s_free = s_full + 1;
+  uint64_t* dp_full = s_free + 1;
+  uint64_t* p_ready = dp_full + 1;
   uint64_t* dq_full = p_ready + 1;
   uint64_t* dq_free = dq_full + 1;
   uint64_t* ds_free = dq_free + 1;
-  uint64_t* dkv_full = ds_free + 1;
+  uint64_t* dkv_full = ds_free + L::DS_BUFS;
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + L::OFF_MISC);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + L::OFF_MISC + 4);
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
 
-  // ---- work item: key tiles near the start see the most queries; go first
-  const int bh = blockIdx.x % p.BH;
-  const int kt = blockIdx.x / p.BH;
+  // ---- work item: head-major (the CTAs running together share one head's
+  // Q, dO and dQ accumulator in L2), key tiles near the start (most work) first
+  const int n_kt = p.N_pad / kTileRows;
+  const int bh = blockIdx.x / n_kt;
+  const int kt = blockIdx.x % n_kt;
   const int k0 = kt * kTileRows;
   const int first_q = (k0 / p.T) * p.T;  // first query that sees key k0
-  const int m_begin = first_q / kTileRows;
-  const int m_end = p.N_pad / kTileRows;
-  const int n_q = m_end - m_begin;
+  const int m_begin = first_q / QN;
+  const int n_q = p.N_pad / QN - m_begin;
 
   if (threadIdx.x == 0) {
     mbar_init(kv_full, 1);
     for (int s = 0; s < NS; ++s) {
       mbar_init(&q_full[s], 1);
       mbar_init(&q_empty[s], 1);
+      mbar_init(&do_full[s], 1);
+      mbar_init(&do_empty[s], 1);
     }
-    mbar_init(st_full, 1);
-    mbar_init(dpt_full, 1);
-    mbar_init(p_ready, 4);
+    mbar_init(s_full, 1);
+    mbar_init(s_free, 8);
+    mbar_init(dp_full, 1);
+    mbar_init(p_ready, 8);
     mbar_init(dq_full, 1);
     mbar_init(dq_free, 4);
-    mbar_init(ds_free, 1);
+    for (int b = 0; b < L::DS_BUFS; ++b) mbar_init(&ds_free[b], 1);
     mbar_init(dkv_full, 1);
     *abort_flag = 0;
     fence_mbar_init();
   }
-  if (warp == 9) {
+  if (warp == 13) {
     tmem_alloc(tmem_slot, 512);
     tmem_relinquish();
   }
@@ -129,231 +166,305 @@ __global__ void __launch_bounds__(BwdLayout<D>::THREADS, 1)
   float* sLSE = reinterpret_cast<float*>(smem + L::OFF_LSE);
   float* sDelta = reinterpret_cast<float*>(smem + L::OFF_DELTA);
 
-  if (warp == 8) {
+  if (warp == 12) {
     // ------------------------------------------------------------ TMA producer
     if (lane == 0) {
       prefetch_tmap(&tm_q);
       prefetch_tmap(&tm_do);
-      mbar_arrive_expect_tx(kv_full, 2 * L::TILE_BYTES);
+      mbar_arrive_expect_tx(kv_full, 2 * L::KTILE);
       for (int r = 0; r < L::REG; ++r) {
-        tma_load_3d(sK + r * L::REGION_BYTES, &tm_k, kv_full, 64 * r, k0, bh);
-        tma_load_3d(sV + r * L::REGION_BYTES, &tm_v, kv_full, 64 * r, k0, bh);
+        tma_load_3d(sK + r * L::KREGION, &tm_k, kv_full, 64 * r, k0, bh);
+        tma_load_3d(sV + r * L::KREGION, &tm_v, kv_full, 64 * r, k0, bh);
       }
-      int issued = 0;
-      for (int i = 0; i < n_q; ++i) {
-        const int st = i % NS;
-        const uint32_t ph = (i / NS) & 1;
-        const int q0 = (m_begin + i) * kTileRows;
-        if (!mbar_wait(&q_empty[st], ph ^ 1, ctl)) break;
-        mbar_arrive_expect_tx(&q_full[st], 2 * L::TILE_BYTES + 2 * L::VEC_BYTES);
-        for (int r = 0; r < L::REG; ++r) {
-          tma_load_3d(sQ + st * L::TILE_BYTES + r * L::REGION_BYTES, &tm_q, &q_full[st], 64 * r, q0, bh);
-          tma_load_3d(sDO + st * L::TILE_BYTES + r * L::REGION_BYTES, &tm_do, &q_full[st], 64 * r, q0, bh);
-        }
+      int issued_q = 0, issued_do = 0;
+      for (int j = 0; j < n_q; ++j) {
+        const int st = j % NS;
+        const uint32_t ph = (j / NS) & 1;
+        const int q0 = (m_begin + j) * QN;
         const size_t voff = static_cast<size_t>(bh) * p.N_pad + q0;
-        bulk_load(sLSE + st * kTileRows, p.lse2 + voff, L::VEC_BYTES, &q_full[st]);
-        bulk_load(sDelta + st * kTileRows, p.delta + voff, L::VEC_BYTES, &q_full[st]);
-        ++issued;
+        if (!mbar_wait(&q_empty[st], ph ^ 1, ctl)) break;
+        mbar_arrive_expect_tx(&q_full[st], L::QTILE + L::VEC_BYTES);
+        for (int r = 0; r < L::REG; ++r)
+          tma_load_3d(sQ + st * L::QTILE + r * L::QREGION, &tm_q, &q_full[st], 64 * r, q0, bh);
+        bulk_load(sLSE + st * QN, p.lse2 + voff, L::VEC_BYTES, &q_full[st]);
+        ++issued_q;
+        if (!mbar_wait(&do_empty[st], ph ^ 1, ctl)) break;
+        mbar_arrive_expect_tx(&do_full[st], L::QTILE + L::VEC_BYTES);
+        for (int r = 0; r < L::REG; ++r)
+          tma_load_3d(sDO + st * L::QTILE + r * L::QREGION, &tm_do, &do_full[st], 64 * r, q0, bh);
+        bulk_load(sDelta + st * QN, p.delta + voff, L::VEC_BYTES, &do_full[st]);
+        ++issued_do;
       }
       if (*abort_flag) {
         drain_wait(kv_full, 0, p.budget_ns);
-        for (int i = max(0, issued - NS); i < issued; ++i)
-          drain_wait(&q_full[i % NS], (i / NS) & 1, p.budget_ns);
+        for (int j = max(0, issued_q - NS); j < issued_q; ++j)
+          drain_wait(&q_full[j % NS], (j / NS) & 1, p.budget_ns);
+        for (int j = max(0, issued_do - NS); j < issued_do; ++j)
+          drain_wait(&do_full[j % NS], (j / NS) & 1, p.budget_ns);
       }
     }
-  } else if (warp == 9) {
+  } else if (warp == 13) {
     // ------------------------------------------------------------ MMA issuer
     if (lane == 0) {
-      constexpr uint32_t idesc_ss = idesc_bf16_f32(128, 128, false, false);   // S^T, dP^T
-      constexpr uint32_t idesc_dv = idesc_bf16_f32(128, D, false, true);      // P^T dO
-      constexpr uint32_t idesc_dk = idesc_bf16_f32(128, D, false, true);      // dS^T Q
-      constexpr uint32_t idesc_dq = idesc_bf16_f32(128, D, true, true);       // dS K
+      constexpr uint32_t idesc_s = idesc_bf16_f32(128, QN, false, false);    // S^T, dP^T
+      constexpr uint32_t idesc_tn = idesc_bf16_f32(128, D, false, true);     // dV, dK
+      // d = 64: dQ = dS K (M = query rows); d = 128: dQ^T = K^T dS^T (M = head dim)
+      constexpr uint32_t idesc_dq = L::DQT ? idesc_bf16_f32(128, QN, true, true)
+                                           : idesc_bf16_f32(128, D, true, true);
       const uint32_t kb = smem_u32(sK), vb = smem_u32(sV), dsb = smem_u32(sDS);
-      bool ok = mbar_wait(kv_full, 0, ctl);
-      tc_fence_after();
-      for (int i = 0; ok && i < n_q; ++i) {
-        const int st = i % NS;
-        const uint32_t ph = (i / NS) & 1;
-        const uint32_t qb = smem_u32(sQ + st * L::TILE_BYTES);
-        const uint32_t dob = smem_u32(sDO + st * L::TILE_BYTES);
-        if (!(ok = mbar_wait(&q_full[st], ph, ctl))) break;
-        tc_fence_after();
-        // S^T = K Q^T
+      auto q_addr = [&](int st) { return smem_u32(sQ + st * L::QTILE); };
+      auto do_addr = [&](int st) { return smem_u32(sDO + st * L::QTILE); };
+      // X = A B^T, both K-major over d (S^T = K Q^T, dP^T = V dO^T)
+      auto issue_kmajor = [&](uint32_t d_col, uint32_t a, uint32_t b) {
 #pragma unroll
         for (int kk = 0; kk < D / 16; ++kk) {
-          const uint32_t off = (kk >> 2) * L::REGION_BYTES + (kk & 3) * 32;
-          umma_ss(tmem + L::S_COL, sdesc_sw128(kb + off, 16, 1024), sdesc_sw128(qb + off, 16, 1024),
-                  idesc_ss, kk > 0 ? 1u : 0u);
+          const uint32_t ka = (kk >> 2) * L::KREGION + (kk & 3) * 32;
+          const uint32_t kq = (kk >> 2) * L::QREGION + (kk & 3) * 32;
+          umma_ss(tmem + d_col, sdesc_sw128(a + ka, 16, 1024), sdesc_sw128(b + kq, 16, 1024),
+                  idesc_s, kk > 0 ? 1u : 0u);
         }
-        umma_commit(st_full);
-        // dP^T = V dO^T (its TMEM columns held dQ of the previous tile)
-        if (i > 0) {
-          if (!(ok = mbar_wait(dq_free, (i - 1) & 1, ctl))) break;
+      };
+      bool ok = mbar_wait(kv_full, 0, ctl);
+      if (ok) ok = mbar_wait(&q_full[0], 0, ctl);
+      tc_fence_after();
+      if (ok) {
+        issue_kmajor(L::S_COL, kb, q_addr(0));
+        umma_commit(s_full);
+        ok = mbar_wait(&do_full[0], 0, ctl);
+        tc_fence_after();
+      }
+      if (ok) {
+        issue_kmajor(L::DP_COL, vb, do_addr(0));
+        umma_commit(dp_full);
+      }
+      for (int j = 0; ok && j < n_q; ++j) {
+        const int st = j % NS;
+        const int st1 = (j + 1) % NS;
+        const uint32_t ph1 = ((j + 1) / NS) & 1;
+        const bool more = j + 1 < n_q;
+        if (more) {
+          // S^T of the next step as soon as the P/dS warps hold S^T_j in registers
+          if (!(ok = mbar_wait(s_free, j & 1, ctl))) break;
+          if (!(ok = mbar_wait(&q_full[st1], ph1, ctl))) break;
+          tc_fence_after();
+          issue_kmajor(L::S_COL, kb, q_addr(st1));
+          umma_commit(s_full);
+        }
+        if (!(ok = mbar_wait(p_ready, j & 1, ctl))) break;
+        tc_fence_after();
+        // dV += P^T dO_j ; P^T over the first half of each warpgroup's dP^T columns
+#pragma unroll
+        for (int kk = 0; kk < QN / 16; ++kk)
+          umma_ts(tmem + L::DV_COL, tmem + L::DP_COL + (kk / L::KPW) * CW + (kk % L::KPW) * 8,
+                  sdesc_sw128(do_addr(st) + kk * 2048, L::QREGION, 1024), idesc_tn,
+                  (j > 0 || kk > 0) ? 1u : 0u);
+        umma_commit(&do_empty[st]);
+        // dK += dS^T Q_j ; dS^T over the second half
+#pragma unroll
+        for (int kk = 0; kk < QN / 16; ++kk)
+          umma_ts(tmem + L::DK_COL, tmem + L::DP_COL + CW / 2 + (kk / L::KPW) * CW + (kk % L::KPW) * 8,
+                  sdesc_sw128(q_addr(st) + kk * 2048, L::QREGION, 1024), idesc_tn,
+                  (j > 0 || kk > 0) ? 1u : 0u);
+        umma_commit(&q_empty[st]);
+        // dQ of this step, once the drain has read the previous one
+        if (j > 0) {
+          if (!(ok = mbar_wait(dq_free, (j - 1) & 1, ctl))) break;
           tc_fence_after();
         }
-#pragma unroll
-        for (int kk = 0; kk < D / 16; ++kk) {
-          const uint32_t off = (kk >> 2) * L::REGION_BYTES + (kk & 3) * 32;
-          umma_ss(tmem + L::DP_COL, sdesc_sw128(vb + off, 16, 1024), sdesc_sw128(dob + off, 16, 1024),
-                  idesc_ss, kk > 0 ? 1u : 0u);
-        }
-        umma_commit(dpt_full);
-        if (!(ok = mbar_wait(p_ready, i & 1, ctl))) break;
-        tc_fence_after();
-        // dV += P^T dO   (P^T bf16 in TMEM over the S^T columns)
-#pragma unroll
-        for (int kk = 0; kk < kTileRows / 16; ++kk)
-          umma_ts(tmem + L::DV_COL, tmem + L::S_COL + kk * 8,
-                  sdesc_sw128(dob + kk * 2048, L::REGION_BYTES, 1024), idesc_dv,
-                  (i > 0 || kk > 0) ? 1u : 0u);
-        // dK += dS^T Q
+        const uint32_t dsj = dsb + (j % L::DS_BUFS) * L::DS_BYTES;
 #pragma unroll
         for (int kk = 0; kk < kTileRows / 16; ++kk) {
-          const uint32_t off = (kk >> 2) * L::REGION_BYTES + (kk & 3) * 32;
-          umma_ss(tmem + L::DK_COL, sdesc_sw128(dsb + off, 16, 1024),
-                  sdesc_sw128(qb + kk * 2048, L::REGION_BYTES, 1024), idesc_dk,
-                  (i > 0 || kk > 0) ? 1u : 0u);
+          if (L::DQT)   // A = K^T (MN-major over d), B = dS^T (MN-major over queries)
+            umma_ss(tmem + L::DQ_COL, sdesc_sw128(kb + kk * 2048, L::KREGION, 1024),
+                    sdesc_sw128(dsj + kk * 2048, L::KREGION, 1024), idesc_dq, kk > 0 ? 1u : 0u);
+          else          // A = dS (MN-major over queries), B = K (MN-major over d)
+            umma_ss(tmem + L::DQ_COL, sdesc_sw128(dsj + kk * 2048, L::KREGION, 1024),
+                    sdesc_sw128(kb + kk * 2048, L::KREGION, 1024), idesc_dq, kk > 0 ? 1u : 0u);
         }
-        // dQ_tile = dS K
-#pragma unroll
-        for (int kk = 0; kk < kTileRows / 16; ++kk)
-          umma_ss(tmem + L::DP_COL, sdesc_sw128(dsb + kk * 2048, L::REGION_BYTES, 1024),
-                  sdesc_sw128(kb + kk * 2048, L::REGION_BYTES, 1024), idesc_dq, kk > 0 ? 1u : 0u);
         umma_commit(dq_full);
-        umma_commit(&q_empty[st]);
-        umma_commit(ds_free);
+        umma_commit(&ds_free[j % L::DS_BUFS]);
+        if (more) {
+          if (!(ok = mbar_wait(&do_full[st1], ph1, ctl))) break;
+          tc_fence_after();
+          issue_kmajor(L::DP_COL, vb, do_addr(st1));
+          umma_commit(dp_full);
+        }
       }
       if (ok) umma_commit(dkv_full);
     }
-  } else if (warp < 4) {
+  } else if (warp < 8) {
     // ------------------------------------------------------------ P / dS (thread = key row)
-    const int j_local = warp * 32 + lane;
-    const int j = k0 + j_local;
-    const bool j_valid = j < p.N;
-    const int q_start = j_valid ? (j / p.T) * p.T : 0x7fffffff;  // first query seeing key j
-    const uint32_t lane_base = tmem + (static_cast<uint32_t>(warp * 32) << 16);
+    const int wg = warp >> 2;            // query columns [CW wg, CW wg + CW)
+    const int wq = warp & 3;             // TMEM lane quadrant
+    const int j_local = wq * 32 + lane;
+    const int krow = k0 + j_local;
+    const bool k_valid = krow < p.N;
+    const int q_start = k_valid ? (krow / p.T) * p.T : 0x7fffffff;  // first query seeing this key
+    const uint32_t lane_base = tmem + (static_cast<uint32_t>(wq * 32) << 16);
+    const uint32_t s_addr = lane_base + L::S_COL + CW * wg;
+    const uint32_t dp_addr = lane_base + L::DP_COL + CW * wg;
     const float sl2 = p.scale_log2;
-    // dS^T row j_local, swizzled like a TMA 128-byte tile (two 64-column regions)
-    uint8_t* ds_row = sDS + j_local * 128;
+    // this thread's dS^T row segment: region (CW wg) / 64, chunks from (CW wg % 64) / 8
+    const int c0 = CW * wg;
+    const int ds_off = (c0 >> 6) * L::KREGION + j_local * 128;
+    const int chunk0 = (c0 & 63) >> 3;
     const int sw = j_local & 7;
     bool ok = true;
-    for (int i = 0; i < n_q; ++i) {
-      const int st = i % NS;
-      const int q0 = (m_begin + i) * kTileRows;
-      const float* lse2 = sLSE + st * kTileRows;
-      const float* delta = sDelta + st * kTileRows;
-      if (!(ok = warp_wait(st_full, i & 1, ctl))) break;
+    for (int j = 0; j < n_q; ++j) {
+      const int st = j % NS;
+      const int q0 = (m_begin + j) * QN;
+      const float* lse2 = sLSE + st * QN + c0;
+      const float* delta = sDelta + st * QN + c0;
+      if (!(ok = warp_wait(s_full, j & 1, ctl))) break;
       tc_fence_after();
-      const int lim = q_start - q0;  // columns c < lim are masked
-      float pr[128];
+      float pr[CW];
 #pragma unroll
-      for (int c = 0; c < 4; ++c) {
+      for (int h = 0; h < CW / 32; ++h) {
         uint32_t r[32];
-        tmem_ld32(lane_base + L::S_COL + 32 * c, r);
+        tmem_ld32(s_addr + 32 * h, r);
         tmem_wait_ld();
 #pragma unroll
-        for (int k = 0; k < 32; ++k) {
-          const int col = 32 * c + k;
-          const float e = ex2_approx(fmaf(__uint_as_float(r[k]), sl2, -lse2[col]));
-          pr[col] = (col < lim) ? 0.f : e;
-        }
+        for (int k = 0; k < 32; ++k) pr[32 * h + k] = __uint_as_float(r[k]);
       }
-      // P^T -> TMEM (bf16 pairs) for the dV MMA
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(s_free);
+      const int lim = q_start - q0 - c0;  // columns c < lim are masked
 #pragma unroll
-      for (int h = 0; h < 2; ++h) {
-        uint32_t packed[32];
-#pragma unroll
-        for (int k = 0; k < 32; ++k) packed[k] = pack_bf16x2(pr[64 * h + 2 * k], pr[64 * h + 2 * k + 1]);
-        tmem_st32(lane_base + L::S_COL + 32 * h, packed);
+      for (int c = 0; c < CW; ++c) {
+        const float e = ex2_approx(fmaf(pr[c], sl2, -lse2[c]));
+        pr[c] = (c < lim) ? 0.f : e;
       }
-      if (!(ok = warp_wait(dpt_full, i & 1, ctl))) break;
+      if (!(ok = warp_wait(dp_full, j & 1, ctl))) break;
       tc_fence_after();
-      if (i > 0 && !(ok = warp_wait(ds_free, (i - 1) & 1, ctl))) break;
+      uint32_t pk[CW / 2], dk[CW / 2];
 #pragma unroll
-      for (int c = 0; c < 4; ++c) {
+      for (int h = 0; h < CW / 32; ++h) {
         uint32_t r[32];
-        tmem_ld32(lane_base + L::DP_COL + 32 * c, r);
+        tmem_ld32(dp_addr + 32 * h, r);
         tmem_wait_ld();
-        uint32_t packed[16];
 #pragma unroll
         for (int k = 0; k < 16; ++k) {
-          const int col = 32 * c + 2 * k;
-          const float d0 = pr[col] * (__uint_as_float(r[2 * k]) - delta[col]);
-          const float d1 = pr[col + 1] * (__uint_as_float(r[2 * k + 1]) - delta[col + 1]);
-          packed[k] = pack_bf16x2(d0, d1);
-        }
-        // columns [32c, 32c+32) = region c/2, 16-byte chunks 4*(c&1) .. +3
-        uint8_t* region = ds_row + (c >> 1) * L::REGION_BYTES;
-#pragma unroll
-        for (int q = 0; q < 4; ++q) {
-          const int chunk = 4 * (c & 1) + q;
-          *reinterpret_cast<uint4*>(region + ((chunk ^ sw) << 4)) =
-              make_uint4(packed[4 * q], packed[4 * q + 1], packed[4 * q + 2], packed[4 * q + 3]);
+          const int c = 32 * h + 2 * k;
+          const float d0 = pr[c] * (__uint_as_float(r[2 * k]) - delta[c]);
+          const float d1 = pr[c + 1] * (__uint_as_float(r[2 * k + 1]) - delta[c + 1]);
+          pk[16 * h + k] = pack_bf16x2(pr[c], pr[c + 1]);
+          dk[16 * h + k] = pack_bf16x2(d0, d1);
         }
       }
+      // P^T and dS^T (bf16) over the dP^T columns this warp has just read
+      if constexpr (CW == 64) {
+        tmem_st32(dp_addr, pk);
+        tmem_st32(dp_addr + 32, dk);
+      } else {
+        tmem_st16(dp_addr, pk);
+        tmem_st16(dp_addr + 16, dk);
+      }
+      // dS^T row segment -> shared memory (swizzled like a TMA 128-byte tile)
+      const int buf = j % L::DS_BUFS;
+      if (j >= L::DS_BUFS &&
+          !(ok = warp_wait(&ds_free[buf], ((j / L::DS_BUFS) - 1) & 1, ctl)))
+        break;
+      uint8_t* ds_row = sDS + buf * L::DS_BYTES + ds_off;
+#pragma unroll
+      for (int q = 0; q < CW / 8; ++q)
+        *reinterpret_cast<uint4*>(ds_row + (((chunk0 + q) ^ sw) << 4)) =
+            make_uint4(dk[4 * q], dk[4 * q + 1], dk[4 * q + 2], dk[4 * q + 3]);
       fence_proxy_async_smem();
       tmem_wait_st();
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(p_ready);
     }
-    // ---- epilogue: dK (x scale) and dV of this key tile
+    // ---- epilogue: warpgroup 0 writes dK (x scale), warpgroup 1 writes dV
     const bool have = ok && warp_wait(dkv_full, 0, ctl);
     tc_fence_after();
     if (have) {
-      const size_t row_off = (static_cast<size_t>(bh) * p.N + j) * D;
-#pragma unroll
-      for (int which = 0; which < 2; ++which) {
-        const uint32_t col0 = which == 0 ? L::DK_COL : L::DV_COL;
-        const float mul = which == 0 ? p.scale : 1.f;
-        __nv_bfloat16* out = which == 0 ? p.dk : p.dv;
-#pragma unroll
-        for (int c = 0; c < D / 32; ++c) {
-          uint32_t r[32];
-          tmem_ld32(lane_base + col0 + 32 * c, r);
-          tmem_wait_ld();
-          if (j_valid) {
-            uint4* dst = reinterpret_cast<uint4*>(out + row_off + 32 * c);
-#pragma unroll
-            for (int k = 0; k < 4; ++k)
-              dst[k] = make_uint4(pack_bf16x2(__uint_as_float(r[8 * k]) * mul, __uint_as_float(r[8 * k + 1]) * mul),
-                                  pack_bf16x2(__uint_as_float(r[8 * k + 2]) * mul, __uint_as_float(r[8 * k + 3]) * mul),
-                                  pack_bf16x2(__uint_as_float(r[8 * k + 4]) * mul, __uint_as_float(r[8 * k + 5]) * mul),
-                                  pack_bf16x2(__uint_as_float(r[8 * k + 6]) * mul, __uint_as_float(r[8 * k + 7]) * mul));
-          }
-        }
-      }
-    }
-  } else {
-    // ------------------------------------------------------------ dQ drain (thread = query row)
-    const int wq = warp & 3;
-    const int row_local = wq * 32 + lane;
-    const uint32_t lane_base = tmem + (static_cast<uint32_t>(wq * 32) << 16);
-    for (int i = 0; i < n_q; ++i) {
-      const int q0 = (m_begin + i) * kTileRows;
-      if (!warp_wait(dq_full, i & 1, ctl)) break;
-      tc_fence_after();
-      float* dst = p.dq_acc + (static_cast<size_t>(bh) * p.N_pad + q0 + row_local) * D;
+      const uint32_t col0 = wg == 0 ? L::DK_COL : L::DV_COL;
+      const float mul = wg == 0 ? p.scale : 1.f;
+      __nv_bfloat16* out = wg == 0 ? p.dk : p.dv;
+      const size_t row_off = (static_cast<size_t>(bh) * p.N + krow) * D;
 #pragma unroll
       for (int c = 0; c < D / 32; ++c) {
         uint32_t r[32];
-        tmem_ld32(lane_base + L::DP_COL + 32 * c, r);
+        tmem_ld32(lane_base + col0 + 32 * c, r);
         tmem_wait_ld();
+        if (k_valid) {
+          uint4* dst = reinterpret_cast<uint4*>(out + row_off + 32 * c);
 #pragma unroll
-        for (int k = 0; k < 8; ++k)
-          red_add_v4(dst + 32 * c + 4 * k, __uint_as_float(r[4 * k]), __uint_as_float(r[4 * k + 1]),
-                     __uint_as_float(r[4 * k + 2]), __uint_as_float(r[4 * k + 3]));
+          for (int k = 0; k < 4; ++k)
+            dst[k] = make_uint4(pack_bf16x2(__uint_as_float(r[8 * k]) * mul, __uint_as_float(r[8 * k + 1]) * mul),
+                                pack_bf16x2(__uint_as_float(r[8 * k + 2]) * mul, __uint_as_float(r[8 * k + 3]) * mul),
+                                pack_bf16x2(__uint_as_float(r[8 * k + 4]) * mul, __uint_as_float(r[8 * k + 5]) * mul),
+                                pack_bf16x2(__uint_as_float(r[8 * k + 6]) * mul, __uint_as_float(r[8 * k + 7]) * mul));
+        }
       }
-      tc_fence_before();
-      __syncwarp();
-      if (lane == 0) mbar_arrive(dq_free);
+    }
+  } else if (warp < 12) {
+    // ------------------------------------------------------------ dQ drain
+    const int wq = warp & 3;
+    const uint32_t lane_base = tmem + (static_cast<uint32_t>(wq * 32) << 16);
+    for (int j = 0; j < n_q; ++j) {
+      const int q0 = (m_begin + j) * QN;
+      if (!warp_wait(dq_full, j & 1, ctl)) break;
+      tc_fence_after();
+      if constexpr (L::DQT) {
+        // lanes = head-dim columns, TMEM columns = the QN query rows
+        uint32_t r0[32], r1[32];
+        tmem_ld32(lane_base + L::DQ_COL, r0);
+        tmem_ld32(lane_base + L::DQ_COL + 32, r1);
+        tmem_wait_ld();
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(dq_free);
+        // one warp instruction = 32 consecutive head-dim columns of one row
+        float* dst = p.dq_acc + (static_cast<size_t>(bh) * p.N_pad + q0) * D + wq * 32 + lane;
+#pragma unroll
+        for (int c = 0; c < 32; ++c) {
+          red_add(dst + static_cast<size_t>(c) * D, __uint_as_float(r0[c]));
+          red_add(dst + static_cast<size_t>(c + 32) * D, __uint_as_float(r1[c]));
+        }
+      } else {
+        // lanes = query rows; stage the warp's 32 x D block in shared memory
+        // (16-byte chunk f of row r at position (f + r) mod 16: conflict-free
+        // both ways), then reduce it row-contiguously
+        constexpr int CH = D / 4;  // 16-byte chunks per row
+        uint8_t* stg = smem + L::OFF_STG + wq * (32 * D * 4);
+#pragma unroll
+        for (int c = 0; c < D / 32; ++c) {
+          uint32_t r[32];
+          tmem_ld32(lane_base + L::DQ_COL + 32 * c, r);
+          tmem_wait_ld();
+#pragma unroll
+          for (int i = 0; i < 8; ++i) {
+            const int f = 8 * c + i;
+            *reinterpret_cast<uint4*>(stg + lane * (D * 4) + (((f + lane) % CH) << 4)) =
+                make_uint4(r[4 * i], r[4 * i + 1], r[4 * i + 2], r[4 * i + 3]);
+          }
+        }
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(dq_free);
+        constexpr int ROWS_PER = 32 / CH;  // rows covered by one warp instruction
+        float* base = p.dq_acc + (static_cast<size_t>(bh) * p.N_pad + q0 + wq * 32) * D;
+#pragma unroll
+        for (int k = 0; k < 32 / ROWS_PER; ++k) {
+          const int row = ROWS_PER * k + lane / CH;
+          const int f = lane % CH;
+          const uint4 v =
+              *reinterpret_cast<const uint4*>(stg + row * (D * 4) + (((f + row) % CH) << 4));
+          red_add_v4(base + static_cast<size_t>(row) * D + 4 * f, __uint_as_float(v.x),
+                     __uint_as_float(v.y), __uint_as_float(v.z), __uint_as_float(v.w));
+        }
+        __syncwarp();
+      }
     }
   }
 
   __syncwarp();
   tc_fence_before();
   __syncthreads();
-  if (warp == 9) {
+  if (warp == 13) {
     tc_fence_after();
     tmem_dealloc(tmem, 512);
   }
