@@ -19,16 +19,18 @@
 //                           contiguous memory)
 //   post: dQ = scale * dQacc -> bf16
 //
-// Software pipeline: the P/dS warps copy S^T into registers first and
-// release it, so S^T of the next step is computed while they work; dV, dK,
-// dQ of step j and dP^T of step j+1 run while they compute P of step j+1;
-// dQ has its own TMEM columns, so draining it never blocks the next step.
+// Software pipeline: the P/dS warps copy S^T and dP^T into registers and
+// release their TMEM columns at once, so S^T and dP^T of step j+1 are
+// computed while they work on step j; P^T/dS^T have their own columns, so
+// dV, dK, dQ of step j run while the P/dS warps start step j+1.
 //
 // Roles (512 threads): warps 0-7 P/dS (two warpgroups, one half of the query
 // columns each, one key row per thread), warps 8-11 dQ drain, warp 12 TMA
 // producer, warp 13 MMA issuer.
-// TMEM: dV [0,D), dK [D,2D), S^T [2D,2D+QN), dP^T [2D+QN,2D+2QN),
-// dQ [384,448).
+// TMEM: dV [0,D), dK [D,2D), S^T [2D,2D+QN), dP^T [2D+QN,2D+2QN), dQ from
+// column 384 (D columns, or QN when transposed), P^T and dS^T (bf16 pairs) at PDS: d = 128 uses
+// [448,512); d = 64 uses [384,512), its P^T half shared with dQ (dQ_j is
+// written after dV_j has read P^T_j, and the next P^T waits for the drain).
 #include "mw_internal.h"
 #include "mw_ptx.cuh"
 
@@ -46,9 +48,9 @@ struct BwdLayout {
   static constexpr int QREGION = QN * 128;           // region of a QN-row tile
   static constexpr int KTILE = REG * KREGION;
   static constexpr int QTILE = REG * QREGION;
-  static constexpr int STAGES = (D == 64) ? 3 : 4;   // Q and dO tiles in flight
+  static constexpr int STAGES = (D == 64) ? 3 : 2;   // Q and dO tiles in flight
   static constexpr int DS_BYTES = (QN / 64) * KREGION;  // dS^T: 128 key rows x QN columns
-  static constexpr int DS_BUFS = (D == 64) ? 1 : 2;
+  static constexpr int DS_BUFS = 1;
   static constexpr int STG_BYTES = DQT ? 0 : 4 * 32 * D * 4;  // per-warp dQ staging (d = 64)
   static constexpr int VEC_BYTES = QN * 4;
   static constexpr int OFF_K = 0;
@@ -61,17 +63,24 @@ struct BwdLayout {
   static constexpr int OFF_DELTA = OFF_LSE + STAGES * VEC_BYTES;
   static constexpr int OFF_BAR = OFF_DELTA + STAGES * VEC_BYTES;
   // kv_full, q_full[S], q_empty[S], do_full[S], do_empty[S], s_full, s_free,
-  // dp_full, p_ready, dq_full, dq_free, ds_free[DS_BUFS], dkv_full
-  static constexpr int NBAR = 1 + 4 * STAGES + 7 + DS_BUFS;
+  // dp_full, dp_free, p_ready, pds_free, dq_full, dq_free, ds_free[DS_BUFS],
+  // dkv_full
+  static constexpr int NBAR = 1 + 4 * STAGES + 9 + DS_BUFS;
   static constexpr int OFF_MISC = OFF_BAR + NBAR * 8;
   static constexpr int BYTES = OFF_MISC + 16;
+  // d = 128 has no room for separate S^T / dP^T / P^T-dS^T columns: one
+  // 128-column block X holds them in turn (each is copied to registers
+  // before the next one lands there)
+  static constexpr bool SHARED_X = (D == 128);
   static constexpr uint32_t DV_COL = 0;
   static constexpr uint32_t DK_COL = D;
   static constexpr uint32_t S_COL = 2 * D;
-  static constexpr uint32_t DP_COL = 2 * D + QN;
+  static constexpr uint32_t DP_COL = SHARED_X ? S_COL : 2 * D + QN;
+  static constexpr uint32_t PDS_COL = SHARED_X ? S_COL : 384u;
   static constexpr uint32_t DQ_COL = 384;
+  static constexpr bool PDS_SHARES_DQ = !SHARED_X;
   static constexpr int THREADS = 512;
-  static_assert(2 * D + 2 * QN <= 384, "TMEM columns");
+  static_assert(SHARED_X ? (2 * D + QN <= 384) : (2 * D + 2 * QN <= 384), "TMEM columns");
   static_assert(BYTES <= 232448, "shared memory");
 };
 
@@ -108,8 +117,10 @@ __global__ void __launch_bounds__(BwdLayout<D>::THREADS, 1)
   uint64_t* s_full = do_empty + NS;
   uint64_t* s_free = s_full + 1;
   uint64_t* dp_full = s_free + 1;
-  uint64_t* p_ready = dp_full + 1;
-  uint64_t* dq_full = p_ready + 1;
+  uint64_t* dp_free = dp_full + 1;
+  uint64_t* p_ready = dp_free + 1;
+  uint64_t* pds_free = p_ready + 1;
+  uint64_t* dq_full = pds_free + 1;
   uint64_t* dq_free = dq_full + 1;
   uint64_t* ds_free = dq_free + 1;
   uint64_t* dkv_full = ds_free + L::DS_BUFS;
@@ -140,7 +151,9 @@ __global__ void __launch_bounds__(BwdLayout<D>::THREADS, 1)
     mbar_init(s_full, 1);
     mbar_init(s_free, 8);
     mbar_init(dp_full, 1);
+    mbar_init(dp_free, 8);
     mbar_init(p_ready, 8);
+    mbar_init(pds_free, 1);
     mbar_init(dq_full, 1);
     mbar_init(dq_free, 4);
     for (int b = 0; b < L::DS_BUFS; ++b) mbar_init(&ds_free[b], 1);
@@ -211,30 +224,44 @@ __global__ void __launch_bounds__(BwdLayout<D>::THREADS, 1)
       // d = 64: dQ = dS K (M = query rows); d = 128: dQ^T = K^T dS^T (M = head dim)
       constexpr uint32_t idesc_dq = L::DQT ? idesc_bf16_f32(128, QN, true, true)
                                            : idesc_bf16_f32(128, D, true, true);
-      const uint32_t kb = smem_u32(sK), vb = smem_u32(sV), dsb = smem_u32(sDS);
-      auto q_addr = [&](int st) { return smem_u32(sQ + st * L::QTILE); };
-      auto do_addr = [&](int st) { return smem_u32(sDO + st * L::QTILE); };
+      // descriptors computed once; each MMA adds a compile-time offset
+      const uint64_t k_kmaj = sdesc_sw128(smem_u32(sK), 16, 1024);
+      const uint64_t v_kmaj = sdesc_sw128(smem_u32(sV), 16, 1024);
+      const uint64_t k_mn = sdesc_sw128(smem_u32(sK), L::KREGION, 1024);
+      const uint64_t q_kmaj0 = sdesc_sw128(smem_u32(sQ), 16, 1024);
+      const uint64_t do_kmaj0 = sdesc_sw128(smem_u32(sDO), 16, 1024);
+      const uint64_t q_mn0 = sdesc_sw128(smem_u32(sQ), L::QREGION, 1024);
+      const uint64_t do_mn0 = sdesc_sw128(smem_u32(sDO), L::QREGION, 1024);
+      const uint64_t ds_mn0 = sdesc_sw128(smem_u32(sDS), L::KREGION, 1024);
       // X = A B^T, both K-major over d (S^T = K Q^T, dP^T = V dO^T)
-      auto issue_kmajor = [&](uint32_t d_col, uint32_t a, uint32_t b) {
+      auto issue_kmajor = [&](uint32_t d_col, uint64_t a, uint64_t b) {
 #pragma unroll
         for (int kk = 0; kk < D / 16; ++kk) {
           const uint32_t ka = (kk >> 2) * L::KREGION + (kk & 3) * 32;
           const uint32_t kq = (kk >> 2) * L::QREGION + (kk & 3) * 32;
-          umma_ss(tmem + d_col, sdesc_sw128(a + ka, 16, 1024), sdesc_sw128(b + kq, 16, 1024),
-                  idesc_s, kk > 0 ? 1u : 0u);
+          umma_ss(tmem + d_col, sdesc_add(a, ka), sdesc_add(b, kq), idesc_s, kk > 0 ? 1u : 0u);
         }
+      };
+      // TMEM columns of the k-th 16-query slice of P^T and of dS^T (bf16 pairs)
+      auto pt_col = [](int kk) -> uint32_t {
+        return L::SHARED_X ? L::PDS_COL + (kk >> 2) * 64 + (kk & 3) * 8 : L::PDS_COL + kk * 8;
+      };
+      auto dst_col = [](int kk) -> uint32_t {
+        return L::SHARED_X ? L::PDS_COL + (kk >> 2) * 64 + 32 + (kk & 3) * 8
+                           : L::PDS_COL + QN / 2 + kk * 8;
       };
       bool ok = mbar_wait(kv_full, 0, ctl);
       if (ok) ok = mbar_wait(&q_full[0], 0, ctl);
       tc_fence_after();
       if (ok) {
-        issue_kmajor(L::S_COL, kb, q_addr(0));
+        issue_kmajor(L::S_COL, k_kmaj, q_kmaj0);
         umma_commit(s_full);
-        ok = mbar_wait(&do_full[0], 0, ctl);
+        if (L::SHARED_X) ok = mbar_wait(s_free, 0, ctl);  // X holds S^T_0 until read
+        if (ok) ok = mbar_wait(&do_full[0], 0, ctl);
         tc_fence_after();
       }
       if (ok) {
-        issue_kmajor(L::DP_COL, vb, do_addr(0));
+        issue_kmajor(L::DP_COL, v_kmaj, do_kmaj0);
         umma_commit(dp_full);
       }
       for (int j = 0; ok && j < n_q; ++j) {
@@ -242,53 +269,66 @@ __global__ void __launch_bounds__(BwdLayout<D>::THREADS, 1)
         const int st1 = (j + 1) % NS;
         const uint32_t ph1 = ((j + 1) / NS) & 1;
         const bool more = j + 1 < n_q;
-        if (more) {
-          // S^T of the next step as soon as the P/dS warps hold S^T_j in registers
+        if (!L::SHARED_X && more) {
+          // S^T and dP^T of the next step as soon as the P/dS warps hold
+          // step j's values in registers
           if (!(ok = mbar_wait(s_free, j & 1, ctl))) break;
           if (!(ok = mbar_wait(&q_full[st1], ph1, ctl))) break;
           tc_fence_after();
-          issue_kmajor(L::S_COL, kb, q_addr(st1));
+          issue_kmajor(L::S_COL, k_kmaj, sdesc_add(q_kmaj0, st1 * L::QTILE));
           umma_commit(s_full);
+          if (!(ok = mbar_wait(dp_free, j & 1, ctl))) break;
+          if (!(ok = mbar_wait(&do_full[st1], ph1, ctl))) break;
+          tc_fence_after();
+          issue_kmajor(L::DP_COL, v_kmaj, sdesc_add(do_kmaj0, st1 * L::QTILE));
+          umma_commit(dp_full);
         }
         if (!(ok = mbar_wait(p_ready, j & 1, ctl))) break;
         tc_fence_after();
-        // dV += P^T dO_j ; P^T over the first half of each warpgroup's dP^T columns
+        const uint64_t do_mn = sdesc_add(do_mn0, st * L::QTILE);
+        const uint64_t q_mn = sdesc_add(q_mn0, st * L::QTILE);
+        // dV += P^T dO_j
 #pragma unroll
         for (int kk = 0; kk < QN / 16; ++kk)
-          umma_ts(tmem + L::DV_COL, tmem + L::DP_COL + (kk / L::KPW) * CW + (kk % L::KPW) * 8,
-                  sdesc_sw128(do_addr(st) + kk * 2048, L::QREGION, 1024), idesc_tn,
-                  (j > 0 || kk > 0) ? 1u : 0u);
+          umma_ts(tmem + L::DV_COL, tmem + pt_col(kk), sdesc_add(do_mn, kk * 2048),
+                  idesc_tn, (j > 0 || kk > 0) ? 1u : 0u);
         umma_commit(&do_empty[st]);
-        // dK += dS^T Q_j ; dS^T over the second half
+        // dK += dS^T Q_j
 #pragma unroll
         for (int kk = 0; kk < QN / 16; ++kk)
-          umma_ts(tmem + L::DK_COL, tmem + L::DP_COL + CW / 2 + (kk / L::KPW) * CW + (kk % L::KPW) * 8,
-                  sdesc_sw128(q_addr(st) + kk * 2048, L::QREGION, 1024), idesc_tn,
-                  (j > 0 || kk > 0) ? 1u : 0u);
+          umma_ts(tmem + L::DK_COL, tmem + dst_col(kk), sdesc_add(q_mn, kk * 2048),
+                  idesc_tn, (j > 0 || kk > 0) ? 1u : 0u);
         umma_commit(&q_empty[st]);
+        if (L::SHARED_X && more) {
+          // X is free once dV/dK have read P^T/dS^T (issue order): S^T of the
+          // next step, then its dP^T once the P/dS warps have read that S^T
+          if (!(ok = mbar_wait(&q_full[st1], ph1, ctl))) break;
+          tc_fence_after();
+          issue_kmajor(L::S_COL, k_kmaj, sdesc_add(q_kmaj0, st1 * L::QTILE));
+          umma_commit(s_full);
+          if (!(ok = mbar_wait(s_free, (j + 1) & 1, ctl))) break;
+          if (!(ok = mbar_wait(&do_full[st1], ph1, ctl))) break;
+          tc_fence_after();
+          issue_kmajor(L::DP_COL, v_kmaj, sdesc_add(do_kmaj0, st1 * L::QTILE));
+          umma_commit(dp_full);
+        }
         // dQ of this step, once the drain has read the previous one
-        if (j > 0) {
+        if (!L::PDS_SHARES_DQ && j > 0) {
           if (!(ok = mbar_wait(dq_free, (j - 1) & 1, ctl))) break;
           tc_fence_after();
         }
-        const uint32_t dsj = dsb + (j % L::DS_BUFS) * L::DS_BYTES;
+        const uint64_t ds_mn = sdesc_add(ds_mn0, (j % L::DS_BUFS) * L::DS_BYTES);
 #pragma unroll
         for (int kk = 0; kk < kTileRows / 16; ++kk) {
-          if (L::DQT)   // A = K^T (MN-major over d), B = dS^T (MN-major over queries)
-            umma_ss(tmem + L::DQ_COL, sdesc_sw128(kb + kk * 2048, L::KREGION, 1024),
-                    sdesc_sw128(dsj + kk * 2048, L::KREGION, 1024), idesc_dq, kk > 0 ? 1u : 0u);
-          else          // A = dS (MN-major over queries), B = K (MN-major over d)
-            umma_ss(tmem + L::DQ_COL, sdesc_sw128(dsj + kk * 2048, L::KREGION, 1024),
-                    sdesc_sw128(kb + kk * 2048, L::KREGION, 1024), idesc_dq, kk > 0 ? 1u : 0u);
+          if constexpr (L::DQT)   // A = K^T (MN-major over d), B = dS^T (MN-major over queries)
+            umma_ss(tmem + L::DQ_COL, sdesc_add(k_mn, kk * 2048), sdesc_add(ds_mn, kk * 2048),
+                    idesc_dq, kk > 0 ? 1u : 0u);
+          else                    // A = dS (MN-major over queries), B = K (MN-major over d)
+            umma_ss(tmem + L::DQ_COL, sdesc_add(ds_mn, kk * 2048), sdesc_add(k_mn, kk * 2048),
+                    idesc_dq, kk > 0 ? 1u : 0u);
         }
         umma_commit(dq_full);
         umma_commit(&ds_free[j % L::DS_BUFS]);
-        if (more) {
-          if (!(ok = mbar_wait(&do_full[st1], ph1, ctl))) break;
-          tc_fence_after();
-          issue_kmajor(L::DP_COL, vb, do_addr(st1));
-          umma_commit(dp_full);
-        }
       }
       if (ok) umma_commit(dkv_full);
     }
@@ -303,6 +343,10 @@ __global__ void __launch_bounds__(BwdLayout<D>::THREADS, 1)
     const uint32_t lane_base = tmem + (static_cast<uint32_t>(wq * 32) << 16);
     const uint32_t s_addr = lane_base + L::S_COL + CW * wg;
     const uint32_t dp_addr = lane_base + L::DP_COL + CW * wg;
+    // P^T / dS^T destinations: within this warpgroup's own 64 X columns
+    // (d = 128), or in the separate P^T and dS^T blocks (d = 64)
+    const uint32_t pds_p = lane_base + (L::SHARED_X ? L::PDS_COL + 64 * wg : L::PDS_COL + 32 * wg);
+    const uint32_t pds_s = L::SHARED_X ? pds_p + 32 : pds_p + QN / 2;
     const float sl2 = p.scale_log2;
     // this thread's dS^T row segment: region (CW wg) / 64, chunks from (CW wg % 64) / 8
     const int c0 = CW * wg;
@@ -330,10 +374,25 @@ __global__ void __launch_bounds__(BwdLayout<D>::THREADS, 1)
       __syncwarp();
       if (lane == 0) mbar_arrive(s_free);
       const int lim = q_start - q0 - c0;  // columns c < lim are masked
+      // row vectors of this step from shared memory, 16 bytes per load
+      float2 nl[CW / 2];
 #pragma unroll
-      for (int c = 0; c < CW; ++c) {
-        const float e = ex2_approx(fmaf(pr[c], sl2, -lse2[c]));
-        pr[c] = (c < lim) ? 0.f : e;
+      for (int c = 0; c < CW / 4; ++c) {
+        const float4 v = reinterpret_cast<const float4*>(lse2)[c];
+        nl[2 * c] = make_float2(-v.x, -v.y);
+        nl[2 * c + 1] = make_float2(-v.z, -v.w);
+      }
+      const float2 sl2x2 = make_float2(sl2, sl2);
+#pragma unroll
+      for (int c = 0; c < CW / 2; ++c) {
+        const float2 x = fma2(make_float2(pr[2 * c], pr[2 * c + 1]), sl2x2, nl[c]);
+        pr[2 * c] = ex2_approx(x.x);
+        pr[2 * c + 1] = ex2_approx(x.y);
+      }
+      if (__any_sync(0xffffffffu, lim > 0)) {
+#pragma unroll
+        for (int c = 0; c < CW; ++c)
+          if (c < lim) pr[c] = 0.f;
       }
       if (!(ok = warp_wait(dp_full, j & 1, ctl))) break;
       tc_fence_after();
@@ -343,24 +402,31 @@ __global__ void __launch_bounds__(BwdLayout<D>::THREADS, 1)
         uint32_t r[32];
         tmem_ld32(dp_addr + 32 * h, r);
         tmem_wait_ld();
+        if (!L::SHARED_X && h == CW / 32 - 1) {
+          // dP^T is in registers: its columns can take the next step's dP^T
+          tc_fence_before();
+          __syncwarp();
+          if (lane == 0) mbar_arrive(dp_free);
+        }
 #pragma unroll
-        for (int k = 0; k < 16; ++k) {
-          const int c = 32 * h + 2 * k;
-          const float d0 = pr[c] * (__uint_as_float(r[2 * k]) - delta[c]);
-          const float d1 = pr[c + 1] * (__uint_as_float(r[2 * k + 1]) - delta[c + 1]);
-          pk[16 * h + k] = pack_bf16x2(pr[c], pr[c + 1]);
-          dk[16 * h + k] = pack_bf16x2(d0, d1);
+        for (int k = 0; k < 8; ++k) {
+          const float4 dv = reinterpret_cast<const float4*>(delta)[8 * h + k];
+          const int c = 32 * h + 4 * k;
+          // dS = P (dP - D), two columns per instruction
+          const float2 t0 = add2(make_float2(__uint_as_float(r[4 * k]), __uint_as_float(r[4 * k + 1])),
+                                 make_float2(-dv.x, -dv.y));
+          const float2 t1 = add2(make_float2(__uint_as_float(r[4 * k + 2]), __uint_as_float(r[4 * k + 3])),
+                                 make_float2(-dv.z, -dv.w));
+          const float2 s0 = mul2(make_float2(pr[c], pr[c + 1]), t0);
+          const float2 s1 = mul2(make_float2(pr[c + 2], pr[c + 3]), t1);
+          pk[16 * h + 2 * k] = pack_bf16x2(pr[c], pr[c + 1]);
+          pk[16 * h + 2 * k + 1] = pack_bf16x2(pr[c + 2], pr[c + 3]);
+          dk[16 * h + 2 * k] = pack_bf16x2(s0.x, s0.y);
+          dk[16 * h + 2 * k + 1] = pack_bf16x2(s1.x, s1.y);
         }
       }
-      // P^T and dS^T (bf16) over the dP^T columns this warp has just read
-      if constexpr (CW == 64) {
-        tmem_st32(dp_addr, pk);
-        tmem_st32(dp_addr + 32, dk);
-      } else {
-        tmem_st16(dp_addr, pk);
-        tmem_st16(dp_addr + 16, dk);
-      }
-      // dS^T row segment -> shared memory (swizzled like a TMA 128-byte tile)
+      // dS^T row segment -> shared memory (swizzled like a TMA 128-byte tile);
+      // independent of the TMEM columns below, so it goes first
       const int buf = j % L::DS_BUFS;
       if (j >= L::DS_BUFS &&
           !(ok = warp_wait(&ds_free[buf], ((j / L::DS_BUFS) - 1) & 1, ctl)))
@@ -370,6 +436,19 @@ __global__ void __launch_bounds__(BwdLayout<D>::THREADS, 1)
       for (int q = 0; q < CW / 8; ++q)
         *reinterpret_cast<uint4*>(ds_row + (((chunk0 + q) ^ sw) << 4)) =
             make_uint4(dk[4 * q], dk[4 * q + 1], dk[4 * q + 2], dk[4 * q + 3]);
+      // P^T and dS^T (bf16 pairs) into their own columns, once step j-1's
+      // dV/dK (and for d = 64 the drain of dQ_{j-1}, which shares them) are done
+      if (!L::SHARED_X && j > 0) {
+        if (!(ok = warp_wait(dq_free, (j - 1) & 1, ctl))) break;
+        tc_fence_after();
+      }
+      if constexpr (CW == 64) {
+        tmem_st32(pds_p, pk);
+        tmem_st32(pds_s, dk);
+      } else {
+        tmem_st16(pds_p, pk);
+        tmem_st16(pds_s, dk);
+      }
       fence_proxy_async_smem();
       tmem_wait_st();
       tc_fence_before();
@@ -409,20 +488,25 @@ __global__ void __launch_bounds__(BwdLayout<D>::THREADS, 1)
       if (!warp_wait(dq_full, j & 1, ctl)) break;
       tc_fence_after();
       if constexpr (L::DQT) {
-        // lanes = head-dim columns, TMEM columns = the QN query rows
-        uint32_t r0[32], r1[32];
-        tmem_ld32(lane_base + L::DQ_COL, r0);
-        tmem_ld32(lane_base + L::DQ_COL + 32, r1);
-        tmem_wait_ld();
-        tc_fence_before();
-        __syncwarp();
-        if (lane == 0) mbar_arrive(dq_free);
-        // one warp instruction = 32 consecutive head-dim columns of one row
+        // lanes = head-dim columns, TMEM columns = the QN query rows; one warp
+        // instruction reduces 32 consecutive head-dim columns of one row
         float* dst = p.dq_acc + (static_cast<size_t>(bh) * p.N_pad + q0) * D + wq * 32 + lane;
 #pragma unroll
-        for (int c = 0; c < 32; ++c) {
-          red_add(dst + static_cast<size_t>(c) * D, __uint_as_float(r0[c]));
-          red_add(dst + static_cast<size_t>(c + 32) * D, __uint_as_float(r1[c]));
+        for (int half = 0; half < QN / 64; ++half) {
+          uint32_t r0[32], r1[32];
+          tmem_ld32(lane_base + L::DQ_COL + 64 * half, r0);
+          tmem_ld32(lane_base + L::DQ_COL + 64 * half + 32, r1);
+          tmem_wait_ld();
+          if (half == QN / 64 - 1) {
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(dq_free);
+          }
+#pragma unroll
+          for (int c = 0; c < 32; ++c) {
+            red_add(dst + static_cast<size_t>(64 * half + c) * D, __uint_as_float(r0[c]));
+            red_add(dst + static_cast<size_t>(64 * half + c + 32) * D, __uint_as_float(r1[c]));
+          }
         }
       } else {
         // lanes = query rows; stage the warp's 32 x D block in shared memory

@@ -7,10 +7,11 @@
 // chunk blocks above the diagonal are never visited; a per-row limit masks
 // the few tiles that straddle a chunk edge.
 //
-// Roles (320 threads):
+// Roles (384 threads):
 //   warps 0-3 / 4-7  softmax of query tile 0 / 1 (one thread per row = TMEM lane)
 //   warp 8           TMA producer (Q once, then K/V tiles through a ring of stages)
 //   warp 9           tcgen05 issuer (S = Q K^T into TMEM, O += P V with P in TMEM)
+//   warps 10-11      idle (they complete warpgroup 2 for the register re-split)
 // TMEM (512 columns): S_t at column 128 t (P_t, bf16, overwrites its first 64
 // columns), O_t at 256 + D t.
 #include "mw_internal.h"
@@ -35,7 +36,15 @@ struct FwdLayout {
   static constexpr int BYTES = OFF_MISC + 16;
   static constexpr uint32_t S_COL(int t) { return 128u * t; }
   static constexpr uint32_t O_COL(int t) { return 256u + D * t; }
-  static constexpr int THREADS = 320;
+  static constexpr int THREADS = 384;
+  // registers per thread after the re-split: softmax warpgroups 0-1 get
+  // more, warpgroup 2 (TMA, MMA, two idle warps) less; 2*128*224 + 128*56
+  // equals the launch's 384 threads x 168 registers
+  static constexpr int REGS_LAUNCH = 168;
+  static constexpr int REGS_SOFTMAX = 224;
+  static constexpr int REGS_CONTROL = 56;
+  static_assert(2 * 128 * REGS_SOFTMAX + 128 * REGS_CONTROL == THREADS * REGS_LAUNCH,
+                "register re-split must hand out exactly the launch's registers");
 };
 
 // Where key tile j of a query block comes from.
@@ -150,6 +159,9 @@ __global__ void __launch_bounds__(FwdLayout<D>::THREADS, 1)
   uint8_t* sK = smem + L::OFF_K;
   uint8_t* sV = smem + L::OFF_V;
 
+  if (warp >= 8) {
+  // warpgroup 2: every warp executes this one re-split instruction
+  regs_dec<L::REGS_CONTROL>();
   if (warp == 8) {
     // ------------------------------------------------------------ TMA producer
     if (lane == 0 && n_local > 0) {
@@ -197,25 +209,27 @@ __global__ void __launch_bounds__(FwdLayout<D>::THREADS, 1)
     if (lane == 0 && n_local > 0) {
       constexpr uint32_t idesc_qk = idesc_bf16_f32(128, 128, false, false);
       constexpr uint32_t idesc_pv = idesc_bf16_f32(128, D, false, true);
-      const uint32_t q_base = smem_u32(sQ), k_base = smem_u32(sK), v_base = smem_u32(sV);
+      // descriptors computed once; each MMA adds a compile-time offset
+      const uint64_t q_desc = sdesc_sw128(smem_u32(sQ), 16, 1024);
+      const uint64_t k_desc = sdesc_sw128(smem_u32(sK), 16, 1024);
+      const uint64_t v_desc = sdesc_sw128(smem_u32(sV), L::REGION_BYTES, 1024);
 
       auto issue_qk = [&](int t, int st) {
-        const uint32_t qa = q_base + t * L::TILE_BYTES;
-        const uint32_t kb = k_base + st * L::TILE_BYTES;
+        const uint64_t qa = sdesc_add(q_desc, t * L::TILE_BYTES);
+        const uint64_t kb = sdesc_add(k_desc, st * L::TILE_BYTES);
 #pragma unroll
         for (int kk = 0; kk < D / 16; ++kk) {
           const uint32_t off = (kk >> 2) * L::REGION_BYTES + (kk & 3) * 32;
-          umma_ss(tmem + L::S_COL(t), sdesc_sw128(qa + off, 16, 1024), sdesc_sw128(kb + off, 16, 1024),
-                  idesc_qk, kk > 0 ? 1u : 0u);
+          umma_ss(tmem + L::S_COL(t), sdesc_add(qa, off), sdesc_add(kb, off), idesc_qk,
+                  kk > 0 ? 1u : 0u);
         }
       };
       auto issue_pv = [&](int t, int st, bool acc) {
-        const uint32_t vb = v_base + st * L::TILE_BYTES;
+        const uint64_t vb = sdesc_add(v_desc, st * L::TILE_BYTES);
 #pragma unroll
         for (int kk = 0; kk < kTileRows / 16; ++kk) {
-          umma_ts(tmem + L::O_COL(t), tmem + L::S_COL(t) + kk * 8,
-                  sdesc_sw128(vb + kk * 2048, L::REGION_BYTES, 1024), idesc_pv,
-                  (acc || kk > 0) ? 1u : 0u);
+          umma_ts(tmem + L::O_COL(t), tmem + L::S_COL(t) + kk * 8, sdesc_add(vb, kk * 2048),
+                  idesc_pv, (acc || kk > 0) ? 1u : 0u);
         }
       };
 
@@ -257,7 +271,9 @@ __global__ void __launch_bounds__(FwdLayout<D>::THREADS, 1)
         }
       }
     }
+  }
   } else {
+    regs_inc<L::REGS_SOFTMAX>();
     // ------------------------------------------------------------ softmax
     const int t = warp >> 2;
     const int wq = warp & 3;
@@ -321,23 +337,24 @@ __global__ void __launch_bounds__(FwdLayout<D>::THREADS, 1)
         }
       }
       const float m_eff = (m_used == -INFINITY) ? 0.f : m_used;
-      float rs = 0.f;
+      const float2 sl2x2 = make_float2(sl2, sl2);
+      const float2 negm = make_float2(-m_eff, -m_eff);
+      float2 acc = make_float2(0.f, 0.f);
 #pragma unroll
       for (int h = 0; h < 2; ++h) {
         uint32_t packed[32];
 #pragma unroll
         for (int k = 0; k < 32; ++k) {
-          const float p0 = ex2_approx(fmaf(s[64 * h + 2 * k], sl2, -m_eff));
-          const float p1 = ex2_approx(fmaf(s[64 * h + 2 * k + 1], sl2, -m_eff));
-          const uint32_t pk = pack_bf16x2(p0, p1);
+          const float2 x = fma2(make_float2(s[64 * h + 2 * k], s[64 * h + 2 * k + 1]), sl2x2, negm);
+          const uint32_t pk = pack_bf16x2(ex2_approx(x.x), ex2_approx(x.y));
           // the row sum uses the bf16 weights the PV MMA consumes, so O is an
           // exact convex combination of them
-          rs += __uint_as_float(pk << 16) + __uint_as_float(pk & 0xffff0000u);
+          acc = add2(acc, make_float2(__uint_as_float(pk << 16), __uint_as_float(pk & 0xffff0000u)));
           packed[k] = pk;
         }
         tmem_st32(s_addr + 32 * h, packed);
       }
-      l += rs;
+      l += acc.x + acc.y;
       tmem_wait_st();
       tc_fence_before();
       __syncwarp();
@@ -438,8 +455,14 @@ cudaError_t launch_fwd_t(const CUtensorMap& tq, const CUtensorMap& tk, const CUt
   using L = FwdLayout<D>;
   static bool attr_set = false;  // per process; the attribute is per function
   if (!attr_set) {
-    cudaError_t e = cudaFuncSetAttribute(bca_fwd_kernel<D>,
-                                         cudaFuncAttributeMaxDynamicSharedMemorySize, L::BYTES);
+    // The in-kernel register re-split assumes the launch register count; with
+    // any other count its setmaxnreg.inc could never be satisfied, so refuse.
+    cudaFuncAttributes fa;
+    cudaError_t e = cudaFuncGetAttributes(&fa, bca_fwd_kernel<D>);
+    if (e != cudaSuccess) return e;
+    if (fa.numRegs != L::REGS_LAUNCH) return cudaErrorInvalidKernelImage;
+    e = cudaFuncSetAttribute(bca_fwd_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             L::BYTES);
     if (e != cudaSuccess) return e;
     attr_set = true;
   }

@@ -15,10 +15,8 @@ constexpr int kFwdQTiles = 2;
 constexpr int kFwdBlockRows = kTileRows * kFwdQTiles;
 constexpr int kMaxSplits = 16;
 
-// Query rows per step of the backward key-tile kernel: 128 at d = 64, and 64
-// at d = 128 (where dQ is produced transposed, dQ^T = K^T dS^T, so that its
-// TMEM lanes are head-dim columns).
-__host__ __device__ constexpr int bwd_q_rows(int d) { return d == 64 ? 128 : 64; }
+// Query rows per step of the backward key-tile kernel.
+__host__ __device__ constexpr int bwd_q_rows(int) { return 128; }
 
 // Forward over one (b,h) query block against up to three key segments:
 //   A: ring rows [head, head + lenA)        (committed history, all visible)
