@@ -30,12 +30,19 @@ struct FwdLayout {
   static constexpr int OFF_Q = 0;
   static constexpr int OFF_K = OFF_Q + QT * TILE_BYTES;
   static constexpr int OFF_V = OFF_K + STAGES * TILE_BYTES;
-  static constexpr int OFF_BAR = OFF_V + STAGES * TILE_BYTES;
+  // d = 64: the row sum of P comes out of the PV MMA itself: V is extended
+  // by a region of bf16 ones (reached through each stage descriptor's
+  // leading-byte offset), so O gets 16 extra columns that all hold sum_j P_ij
+  static constexpr bool SUM_MMA = (D == 64);
+  static constexpr int OW = SUM_MMA ? D + 16 : D;     // O columns in TMEM
+  static constexpr int OFF_ONES = OFF_V + STAGES * TILE_BYTES;
+  static constexpr int ONES_BYTES = SUM_MMA ? REGION_BYTES : 0;
+  static constexpr int OFF_BAR = OFF_ONES + ONES_BYTES;
   static constexpr int NBAR = 1 + 4 * STAGES + 2 * QT + 1;
   static constexpr int OFF_MISC = OFF_BAR + NBAR * 8;
   static constexpr int BYTES = OFF_MISC + 16;
   static constexpr uint32_t S_COL(int t) { return 128u * t; }
-  static constexpr uint32_t O_COL(int t) { return 256u + D * t; }
+  static constexpr uint32_t O_COL(int t) { return 256u + OW * t; }
   static constexpr int THREADS = 384;
   // registers per thread after the re-split: softmax warpgroups 0-1 get
   // more, warpgroup 2 (TMA, MMA, two idle warps) less; 2*128*224 + 128*56
@@ -149,6 +156,11 @@ __global__ void __launch_bounds__(FwdLayout<D>::THREADS, 1)
     tmem_alloc(tmem_slot, 512);
     tmem_relinquish();
   }
+  if constexpr (L::SUM_MMA) {
+    uint32_t* ones = reinterpret_cast<uint32_t*>(smem + L::OFF_ONES);
+    for (int k = threadIdx.x; k < L::ONES_BYTES / 4; k += L::THREADS) ones[k] = 0x3F803F80u;  // bf16 1.0
+    fence_proxy_async_smem();  // read by the tensor core (async proxy)
+  }
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
@@ -208,11 +220,12 @@ __global__ void __launch_bounds__(FwdLayout<D>::THREADS, 1)
     // ------------------------------------------------------------ MMA issuer
     if (lane == 0 && n_local > 0) {
       constexpr uint32_t idesc_qk = idesc_bf16_f32(128, 128, false, false);
-      constexpr uint32_t idesc_pv = idesc_bf16_f32(128, D, false, true);
+      constexpr uint32_t idesc_pv = idesc_bf16_f32(128, L::OW, false, true);
       // descriptors computed once; each MMA adds a compile-time offset
       const uint64_t q_desc = sdesc_sw128(smem_u32(sQ), 16, 1024);
       const uint64_t k_desc = sdesc_sw128(smem_u32(sK), 16, 1024);
-      const uint64_t v_desc = sdesc_sw128(smem_u32(sV), L::REGION_BYTES, 1024);
+      const uint32_t v_addr = smem_u32(sV);
+      const uint32_t ones_addr = smem_u32(smem + L::OFF_ONES);
 
       auto issue_qk = [&](int t, int st) {
         const uint64_t qa = sdesc_add(q_desc, t * L::TILE_BYTES);
@@ -225,7 +238,9 @@ __global__ void __launch_bounds__(FwdLayout<D>::THREADS, 1)
         }
       };
       auto issue_pv = [&](int t, int st, bool acc) {
-        const uint64_t vb = sdesc_add(v_desc, st * L::TILE_BYTES);
+        // V stage st; for d = 64 the next 64 "columns" are the ones region
+        const uint32_t vs = v_addr + st * L::TILE_BYTES;
+        const uint64_t vb = sdesc_sw128(vs, L::SUM_MMA ? ones_addr - vs : L::REGION_BYTES, 1024);
 #pragma unroll
         for (int kk = 0; kk < kTileRows / 16; ++kk) {
           umma_ts(tmem + L::O_COL(t), tmem + L::S_COL(t) + kk * 8, sdesc_add(vb, kk * 2048),
@@ -308,9 +323,15 @@ __global__ void __launch_bounds__(FwdLayout<D>::THREADS, 1)
         for (int c = 0; c < 128; ++c)
           if (c >= limit) s[c] = -INFINITY;
       }
-      float mx = s[0];
+      float mq[4] = {s[0], s[1], s[2], s[3]};
 #pragma unroll
-      for (int c = 1; c < 128; ++c) mx = fmaxf(mx, s[c]);
+      for (int c = 4; c < 128; c += 8) {
+        mq[0] = max3(mq[0], s[c], s[c + 1]);
+        mq[1] = max3(mq[1], s[c + 2], s[c + 3]);
+        mq[2] = max3(mq[2], s[c + 4], s[c + 5]);
+        mq[3] = max3(mq[3], s[c + 6], s[c + 7]);
+      }
+      const float mx = max3(fmaxf(mq[0], mq[1]), mq[2], mq[3]);
       const float m_tile = mx * sl2;  // scale > 0
       const float m_cand = fmaxf(m_used, m_tile);
       // Rescale only when the running maximum grew by more than 2^8: P stays
@@ -333,6 +354,14 @@ __global__ void __launch_bounds__(FwdLayout<D>::THREADS, 1)
             for (int k = 0; k < 32; ++k) r[k] = __float_as_uint(__uint_as_float(r[k]) * alpha);
             tmem_st32(o_addr + 32 * c, r);
           }
+          if constexpr (L::SUM_MMA) {  // the row-sum columns scale with O
+            uint32_t r[16];
+            tmem_ld16(o_addr + D, r);
+            tmem_wait_ld();
+#pragma unroll
+            for (int k = 0; k < 16; ++k) r[k] = __float_as_uint(__uint_as_float(r[k]) * alpha);
+            tmem_st16(o_addr + D, r);
+          }
           tmem_wait_st();
         }
       }
@@ -348,8 +377,9 @@ __global__ void __launch_bounds__(FwdLayout<D>::THREADS, 1)
           const float2 x = fma2(make_float2(s[64 * h + 2 * k], s[64 * h + 2 * k + 1]), sl2x2, negm);
           const uint32_t pk = pack_bf16x2(ex2_approx(x.x), ex2_approx(x.y));
           // the row sum uses the bf16 weights the PV MMA consumes, so O is an
-          // exact convex combination of them
-          acc = add2(acc, make_float2(__uint_as_float(pk << 16), __uint_as_float(pk & 0xffff0000u)));
+          // exact convex combination of them (d = 64: summed by the MMA)
+          if constexpr (!L::SUM_MMA)
+            acc = add2(acc, make_float2(__uint_as_float(pk << 16), __uint_as_float(pk & 0xffff0000u)));
           packed[k] = pk;
         }
         tmem_st32(s_addr + 32 * h, packed);
@@ -364,6 +394,14 @@ __global__ void __launch_bounds__(FwdLayout<D>::THREADS, 1)
     // ---- epilogue
     const bool have = __all_sync(0xffffffffu, ok) && n_local > 0 && warp_wait(o_full, 0, ctl);
     tc_fence_after();
+    if constexpr (L::SUM_MMA) {
+      if (have) {
+        uint32_t r[16];
+        tmem_ld16(o_addr + D, r);
+        tmem_wait_ld();
+        l = __uint_as_float(r[0]);
+      }
+    }
     const bool nonzero = have && l > 0.f;
     const float inv_l = nonzero ? 1.f / l : 0.f;
     const float m_eff = (m_used == -INFINITY) ? 0.f : m_used;
