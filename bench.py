@@ -256,7 +256,8 @@ def run_ours(args):
     init_dist(world, "nccl")
     peaks = load_peaks()
 
-    cfg = TRAIN_CONFIGS[WORKLOAD]
+    workload = args.workload
+    cfg = TRAIN_CONFIGS[workload]
     x = gen_train(cfg) if rank == 0 else gen_train(_reseeded(cfg, rank))
     q, k, v, do = (x[n].to(dev) for n in ("q", "k", "v", "do"))
     o = torch.empty_like(q)
@@ -326,17 +327,17 @@ def run_ours(args):
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(ms_per_step, 4),
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
         "data": "synthetic",
-        "config": {"workload": f"{WORKLOAD}: block-causal attention fwd+bwd, B={cfg.B} H={cfg.H} "
+        "config": {"workload": f"{workload}: block-causal attention fwd+bwd, B={cfg.B} H={cfg.H} "
                                f"d={cfg.d}, {cfg.n_chunks} chunks x {cfg.T} tokens (N={cfg.N})",
                    "global_batch": cfg.B * world, "seq_len": cfg.N, "parallelism": f"dp{world}",
                    "flops_per_step": step_flops, "unmasked_pairs": pairs,
                    "l2": "256 MiB buffer written between timed steps (outside the events)"},
         "frac_of_bf16_peak": round(value / world / peaks["bf16_tflops"], 4),
-        "roofline": {"kernel": "bca_bwd_kernel<64> (backward key-tile kernel)", "bound": "tensor",
+        "roofline": {"kernel": f"bca_bwd_kernel<{cfg.d}> (backward key-tile kernel)", "bound": "tensor",
                      "achieved": round(achieved, 2), "peak": peaks["bf16_tflops"],
                      "peak_source": peaks["source"] + " bf16 burst", "unit": "TFLOP/s",
                      "frac": round(achieved / peaks["bf16_tflops"], 4),
-                     "traffic": profiled_traffic("bca_bwd_kernel<64>", WORKLOAD),
+                     "traffic": profiled_traffic(f"bca_bwd_kernel<{cfg.d}>", workload),
                      "algorithmic_bytes": bwd_main_bytes(cfg),
                      "ms_per_launch": round(main_ms, 4)},
         "fwd": {"ms": round(fwd_ms, 4),
@@ -569,6 +570,9 @@ def main(argv=None):
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", choices=("ours", "reference"), default="ours")
     ap.add_argument("--no-extras", action="store_true", help="skip the secondary workloads")
+    ap.add_argument("--workload", choices=sorted(n for n, c in TRAIN_CONFIGS.items() if c.backward),
+                    default=WORKLOAD,
+                    help="training workload of the timed step (default: the headline one)")
     ap.add_argument("--cpu-seconds", type=float, default=12.0,
                     help="budget of the oracle CPU baseline sample")
     ap.add_argument("--no-cpu-baseline", action="store_true",

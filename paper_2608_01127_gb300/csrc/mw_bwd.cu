@@ -21,8 +21,9 @@
 //
 // Software pipeline: the P/dS warps copy S^T and dP^T into registers and
 // release their TMEM columns at once, so S^T and dP^T of step j+1 are
-// computed while they work on step j; P^T/dS^T have their own columns, so
-// dV, dK, dQ of step j run while the P/dS warps start step j+1.
+// computed while they work on step j; P^T is handed over before dS is
+// computed, so dV_j overlaps that math; dK, dQ of step j run while the P/dS
+// warps start step j+1.
 //
 // Roles (512 threads): warps 0-7 P/dS (two warpgroups, one half of the query
 // columns each, one key row per thread), warps 8-11 dQ drain, warp 12 TMA
@@ -63,9 +64,9 @@ struct BwdLayout {
   static constexpr int OFF_DELTA = OFF_LSE + STAGES * VEC_BYTES;
   static constexpr int OFF_BAR = OFF_DELTA + STAGES * VEC_BYTES;
   // kv_full, q_full[S], q_empty[S], do_full[S], do_empty[S], s_full, s_free,
-  // dp_full, dp_free, p_ready, pds_free, dq_full, dq_free, ds_free[DS_BUFS],
-  // dkv_full
-  static constexpr int NBAR = 1 + 4 * STAGES + 9 + DS_BUFS;
+  // dp_full, dp_free, pt_ready, pt_free, p_ready, dq_full, dq_free,
+  // ds_free[DS_BUFS], dkv_full
+  static constexpr int NBAR = 1 + 4 * STAGES + 10 + DS_BUFS;
   static constexpr int OFF_MISC = OFF_BAR + NBAR * 8;
   static constexpr int BYTES = OFF_MISC + 16;
   // d = 128 has no room for separate S^T / dP^T / P^T-dS^T columns: one
@@ -76,9 +77,10 @@ struct BwdLayout {
   static constexpr uint32_t DK_COL = D;
   static constexpr uint32_t S_COL = 2 * D;
   static constexpr uint32_t DP_COL = SHARED_X ? S_COL : 2 * D + QN;
+  // P^T then dS^T (bf16 pairs); at d = 64 dQ_j reuses the dS^T half (it is
+  // written after dK_j has read dS^T_j, and the next dS^T waits for the drain)
   static constexpr uint32_t PDS_COL = SHARED_X ? S_COL : 384u;
-  static constexpr uint32_t DQ_COL = 384;
-  static constexpr bool PDS_SHARES_DQ = !SHARED_X;
+  static constexpr uint32_t DQ_COL = SHARED_X ? 384u : 448u;
   static constexpr int THREADS = 512;
   static_assert(SHARED_X ? (2 * D + QN <= 384) : (2 * D + 2 * QN <= 384), "TMEM columns");
   static_assert(BYTES <= 232448, "shared memory");
@@ -118,9 +120,10 @@ __global__ void __launch_bounds__(BwdLayout<D>::THREADS, 1)
   uint64_t* s_free = s_full + 1;
   uint64_t* dp_full = s_free + 1;
   uint64_t* dp_free = dp_full + 1;
-  uint64_t* p_ready = dp_free + 1;
-  uint64_t* pds_free = p_ready + 1;
-  uint64_t* dq_full = pds_free + 1;
+  uint64_t* pt_ready = dp_free + 1;
+  uint64_t* pt_free = pt_ready + 1;
+  uint64_t* p_ready = pt_free + 1;
+  uint64_t* dq_full = p_ready + 1;
   uint64_t* dq_free = dq_full + 1;
   uint64_t* ds_free = dq_free + 1;
   uint64_t* dkv_full = ds_free + L::DS_BUFS;
@@ -152,8 +155,9 @@ __global__ void __launch_bounds__(BwdLayout<D>::THREADS, 1)
     mbar_init(s_free, 8);
     mbar_init(dp_full, 1);
     mbar_init(dp_free, 8);
+    mbar_init(pt_ready, 8);
+    mbar_init(pt_free, 1);
     mbar_init(p_ready, 8);
-    mbar_init(pds_free, 1);
     mbar_init(dq_full, 1);
     mbar_init(dq_free, 4);
     for (int b = 0; b < L::DS_BUFS; ++b) mbar_init(&ds_free[b], 1);
@@ -269,14 +273,27 @@ __global__ void __launch_bounds__(BwdLayout<D>::THREADS, 1)
         const int st1 = (j + 1) % NS;
         const uint32_t ph1 = ((j + 1) / NS) & 1;
         const bool more = j + 1 < n_q;
+        const uint64_t do_mn = sdesc_add(do_mn0, st * L::QTILE);
+        const uint64_t q_mn = sdesc_add(q_mn0, st * L::QTILE);
         if (!L::SHARED_X && more) {
-          // S^T and dP^T of the next step as soon as the P/dS warps hold
-          // step j's values in registers
+          // S^T of the next step as soon as the P/dS warps hold S^T_j
           if (!(ok = mbar_wait(s_free, j & 1, ctl))) break;
           if (!(ok = mbar_wait(&q_full[st1], ph1, ctl))) break;
           tc_fence_after();
           issue_kmajor(L::S_COL, k_kmaj, sdesc_add(q_kmaj0, st1 * L::QTILE));
           umma_commit(s_full);
+        }
+        // dV += P^T dO_j as soon as P^T_j is in TMEM (while dS_j is computed)
+        if (!(ok = mbar_wait(pt_ready, j & 1, ctl))) break;
+        tc_fence_after();
+#pragma unroll
+        for (int kk = 0; kk < QN / 16; ++kk)
+          umma_ts(tmem + L::DV_COL, tmem + pt_col(kk), sdesc_add(do_mn, kk * 2048),
+                  idesc_tn, (j > 0 || kk > 0) ? 1u : 0u);
+        umma_commit(&do_empty[st]);
+        if (!L::SHARED_X) umma_commit(pt_free);
+        if (!L::SHARED_X && more) {
+          // dP^T of the next step once the P/dS warps hold dP^T_j
           if (!(ok = mbar_wait(dp_free, j & 1, ctl))) break;
           if (!(ok = mbar_wait(&do_full[st1], ph1, ctl))) break;
           tc_fence_after();
@@ -285,14 +302,6 @@ __global__ void __launch_bounds__(BwdLayout<D>::THREADS, 1)
         }
         if (!(ok = mbar_wait(p_ready, j & 1, ctl))) break;
         tc_fence_after();
-        const uint64_t do_mn = sdesc_add(do_mn0, st * L::QTILE);
-        const uint64_t q_mn = sdesc_add(q_mn0, st * L::QTILE);
-        // dV += P^T dO_j
-#pragma unroll
-        for (int kk = 0; kk < QN / 16; ++kk)
-          umma_ts(tmem + L::DV_COL, tmem + pt_col(kk), sdesc_add(do_mn, kk * 2048),
-                  idesc_tn, (j > 0 || kk > 0) ? 1u : 0u);
-        umma_commit(&do_empty[st]);
         // dK += dS^T Q_j
 #pragma unroll
         for (int kk = 0; kk < QN / 16; ++kk)
@@ -312,8 +321,9 @@ __global__ void __launch_bounds__(BwdLayout<D>::THREADS, 1)
           issue_kmajor(L::DP_COL, v_kmaj, sdesc_add(do_kmaj0, st1 * L::QTILE));
           umma_commit(dp_full);
         }
-        // dQ of this step, once the drain has read the previous one
-        if (!L::PDS_SHARES_DQ && j > 0) {
+        // dQ of this step; at d = 128 once the drain has read the previous one
+        // (at d = 64 the P/dS warps waited for that drain before writing dS^T_j)
+        if (L::SHARED_X && j > 0) {
           if (!(ok = mbar_wait(dq_free, (j - 1) & 1, ctl))) break;
           tc_fence_after();
         }
@@ -362,13 +372,15 @@ __global__ void __launch_bounds__(BwdLayout<D>::THREADS, 1)
       if (!(ok = warp_wait(s_full, j & 1, ctl))) break;
       tc_fence_after();
       float pr[CW];
+      {
+        uint32_t r[CW / 32][32];
 #pragma unroll
-      for (int h = 0; h < CW / 32; ++h) {
-        uint32_t r[32];
-        tmem_ld32(s_addr + 32 * h, r);
+        for (int h = 0; h < CW / 32; ++h) tmem_ld32(s_addr + 32 * h, r[h]);
         tmem_wait_ld();
 #pragma unroll
-        for (int k = 0; k < 32; ++k) pr[32 * h + k] = __uint_as_float(r[k]);
+        for (int h = 0; h < CW / 32; ++h)
+#pragma unroll
+          for (int k = 0; k < 32; ++k) pr[32 * h + k] = __uint_as_float(r[h][k]);
       }
       tc_fence_before();
       __syncwarp();
@@ -394,9 +406,30 @@ __global__ void __launch_bounds__(BwdLayout<D>::THREADS, 1)
         for (int c = 0; c < CW; ++c)
           if (c < lim) pr[c] = 0.f;
       }
+      uint32_t dk[CW / 2];
+      uint32_t pk[L::SHARED_X ? CW / 2 : 1];  // d = 128: P^T packed alongside dS^T
+      // d = 64: P^T (bf16 pairs) -> TMEM right away, so that dV_j starts
+      // while dS_j is computed.  (d = 128: X still holds dP^T_j; P^T is stored
+      // with dS^T at the end of the step, which measured faster there.)
+      auto store_pt = [&]() {
+        uint32_t pe[CW / 2];
+#pragma unroll
+        for (int c = 0; c < CW / 2; ++c) pe[c] = pack_bf16x2(pr[2 * c], pr[2 * c + 1]);
+        tmem_st32(pds_p, pe);
+        tmem_wait_st();
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(pt_ready);
+      };
+      if constexpr (!L::SHARED_X) {
+        if (j > 0) {  // dV_{j-1} has read P^T_{j-1}
+          if (!(ok = warp_wait(pt_free, (j - 1) & 1, ctl))) break;
+          tc_fence_after();
+        }
+        store_pt();
+      }
       if (!(ok = warp_wait(dp_full, j & 1, ctl))) break;
       tc_fence_after();
-      uint32_t pk[CW / 2], dk[CW / 2];
 #pragma unroll
       for (int h = 0; h < CW / 32; ++h) {
         uint32_t r[32];
@@ -419,14 +452,15 @@ __global__ void __launch_bounds__(BwdLayout<D>::THREADS, 1)
                                  make_float2(-dv.z, -dv.w));
           const float2 s0 = mul2(make_float2(pr[c], pr[c + 1]), t0);
           const float2 s1 = mul2(make_float2(pr[c + 2], pr[c + 3]), t1);
-          pk[16 * h + 2 * k] = pack_bf16x2(pr[c], pr[c + 1]);
-          pk[16 * h + 2 * k + 1] = pack_bf16x2(pr[c + 2], pr[c + 3]);
           dk[16 * h + 2 * k] = pack_bf16x2(s0.x, s0.y);
           dk[16 * h + 2 * k + 1] = pack_bf16x2(s1.x, s1.y);
+          if constexpr (L::SHARED_X) {
+            pk[16 * h + 2 * k] = pack_bf16x2(pr[c], pr[c + 1]);
+            pk[16 * h + 2 * k + 1] = pack_bf16x2(pr[c + 2], pr[c + 3]);
+          }
         }
       }
-      // dS^T row segment -> shared memory (swizzled like a TMA 128-byte tile);
-      // independent of the TMEM columns below, so it goes first
+      // dS^T row segment -> shared memory (swizzled like a TMA 128-byte tile)
       const int buf = j % L::DS_BUFS;
       if (j >= L::DS_BUFS &&
           !(ok = warp_wait(&ds_free[buf], ((j / L::DS_BUFS) - 1) & 1, ctl)))
@@ -436,24 +470,26 @@ __global__ void __launch_bounds__(BwdLayout<D>::THREADS, 1)
       for (int q = 0; q < CW / 8; ++q)
         *reinterpret_cast<uint4*>(ds_row + (((chunk0 + q) ^ sw) << 4)) =
             make_uint4(dk[4 * q], dk[4 * q + 1], dk[4 * q + 2], dk[4 * q + 3]);
-      // P^T and dS^T (bf16 pairs) into their own columns, once step j-1's
-      // dV/dK (and for d = 64 the drain of dQ_{j-1}, which shares them) are done
+      // dS^T -> TMEM (d = 64: once the drain has read dQ_{j-1}, which shares
+      // these columns)
       if (!L::SHARED_X && j > 0) {
         if (!(ok = warp_wait(dq_free, (j - 1) & 1, ctl))) break;
         tc_fence_after();
       }
-      if constexpr (CW == 64) {
+      if constexpr (L::SHARED_X) {
         tmem_st32(pds_p, pk);
         tmem_st32(pds_s, dk);
       } else {
-        tmem_st16(pds_p, pk);
-        tmem_st16(pds_s, dk);
+        tmem_st32(pds_s, dk);
       }
       fence_proxy_async_smem();
       tmem_wait_st();
       tc_fence_before();
       __syncwarp();
-      if (lane == 0) mbar_arrive(p_ready);
+      if (lane == 0) {
+        if (L::SHARED_X) mbar_arrive(pt_ready);
+        mbar_arrive(p_ready);
+      }
     }
     // ---- epilogue: warpgroup 0 writes dK (x scale), warpgroup 1 writes dV
     const bool have = ok && warp_wait(dkv_full, 0, ctl);
