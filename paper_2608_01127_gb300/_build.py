@@ -1,9 +1,10 @@
 """Builds the sm_103a shared library ``_lib/libmw_bca.so`` in-tree with nvcc.
 
 Each translation unit compiles in parallel, then one nvcc link makes the
-shared library (CUDA runtime linked statically, driver reached at run time
-through the runtime's entry-point query, so the library loads on machines
-without a GPU).  A stamp of the sources' hash skips unchanged rebuilds.
+shared library against the shared CUDA runtime (found through an rpath to
+the toolkit; inside a PyTorch process the runtime PyTorch already loaded is
+used).  The driver is reached at run time through the runtime's entry-point
+query, so the library loads on machines without a GPU.  A stamp of the sources' hash skips unchanged rebuilds.
 """
 from __future__ import annotations
 
@@ -73,7 +74,12 @@ def build(verbose: bool = False, force: bool = False, ptxas_info: bool = False) 
     with cf.ThreadPoolExecutor(max_workers=len(SOURCES)) as ex:
         objs = list(ex.map(compile_one, SOURCES))
     tmp = LIB_PATH + ".tmp"
-    cmd = [nvcc, *ARCH, "-shared", "-cudart", "static", "-o", tmp, *objs]
+    # shared CUDA runtime: inside a PyTorch process the already-loaded
+    # libcudart.so.13 is reused, so the library and PyTorch see one runtime
+    # (one current device, one view of stream capture)
+    cudart_dir = os.path.join(os.path.dirname(os.path.dirname(nvcc)), "lib64")
+    cmd = [nvcc, *ARCH, "-shared", "-cudart", "shared", "-Xlinker", "-rpath=" + cudart_dir,
+           "-o", tmp, *objs]
     r = subprocess.run(cmd, capture_output=True, text=True)
     if r.returncode != 0:
         raise RuntimeError(f"nvcc link failed:\n{r.stdout}\n{r.stderr}")

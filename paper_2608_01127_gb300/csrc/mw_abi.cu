@@ -89,8 +89,8 @@ PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
 
 // 3-D map over [BH, rows, d] bf16 with 64 x 128-row boxes and the 128-byte
 // swizzle the tcgen05 descriptors expect; rows past the end read as zero.
-mw_status make_map(CUtensorMap* m, const void* ptr, int rows, int BH, int d, const char* name,
-                   int box_rows = mw::kTileRows) {
+mw_status encode_map(CUtensorMap* m, const void* ptr, int rows, int BH, int d, const char* name,
+                     int box_rows) {
   auto fn = encode_fn();
   if (!fn) return fail(MW_ERR_CUDA, "cuTensorMapEncodeTiled is unavailable (no CUDA driver?)");
   cuuint64_t dims[3] = {static_cast<cuuint64_t>(d), static_cast<cuuint64_t>(rows),
@@ -103,6 +103,38 @@ mw_status make_map(CUtensorMap* m, const void* ptr, int rows, int BH, int d, con
                   estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
                   CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
   if (r != CUDA_SUCCESS) return fail(MW_ERR_CUDA, "cuTensorMapEncodeTiled(%s) failed: %d", name, (int)r);
+  return MW_OK;
+}
+
+// Small per-thread cache of encoded maps: streaming callers pass the same
+// buffers every step, and encoding is pure host work that depends only on
+// (address, shape, box).
+struct MapKey {
+  const void* ptr;
+  int rows, BH, d, box_rows;
+  bool operator==(const MapKey& o) const {
+    return ptr == o.ptr && rows == o.rows && BH == o.BH && d == o.d && box_rows == o.box_rows;
+  }
+};
+constexpr int kMapCache = 16;
+thread_local MapKey t_map_keys[kMapCache];
+thread_local CUtensorMap t_maps[kMapCache];
+thread_local int t_map_next = 0;
+
+mw_status make_map(CUtensorMap* m, const void* ptr, int rows, int BH, int d, const char* name,
+                   int box_rows = mw::kTileRows) {
+  const MapKey key{ptr, rows, BH, d, box_rows};
+  for (int i = 0; i < kMapCache; ++i) {
+    if (t_map_keys[i].ptr != nullptr && t_map_keys[i] == key) {
+      *m = t_maps[i];
+      return MW_OK;
+    }
+  }
+  MW_TRY(encode_map(m, ptr, rows, BH, d, name, box_rows));
+  const int slot = t_map_next;
+  t_map_next = (t_map_next + 1) % kMapCache;
+  t_map_keys[slot] = key;
+  t_maps[slot] = *m;
   return MW_OK;
 }
 
@@ -122,11 +154,15 @@ mw_status status_ptr(unsigned** out) {
   return MW_OK;
 }
 
+// SM count of the current device, queried once per device.
 int sm_count() {
+  static int cached[kMaxDevices] = {};
   int dev = 0, n = 0;
-  if (cudaGetDevice(&dev) != cudaSuccess) return 152;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return 152;
+  if (cached[dev] > 0) return cached[dev];
   if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n <= 0)
     return 152;
+  cached[dev] = n;
   return n;
 }
 
@@ -185,7 +221,12 @@ class DeviceScope {
   explicit DeviceScope(cudaStream_t stream) {
     if (cudaGetDevice(&prev_) != cudaSuccess) prev_ = -1;
     int dev = prev_;
-    if (stream != nullptr && cudaStreamGetDevice(stream, &dev) != cudaSuccess) dev = prev_;
+    // (cudaStreamGetDevice is not allowed on a stream under graph capture,
+    // and a capturing stream belongs to the current device anyway)
+    cudaStreamCaptureStatus cs = cudaStreamCaptureStatusNone;
+    if (stream != nullptr && cudaStreamIsCapturing(stream, &cs) == cudaSuccess &&
+        cs == cudaStreamCaptureStatusNone && cudaStreamGetDevice(stream, &dev) != cudaSuccess)
+      dev = prev_;
     if (dev < 0) dev = 0;
     err_ = cudaSetDevice(dev);
     dev_ = dev;

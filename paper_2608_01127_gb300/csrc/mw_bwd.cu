@@ -43,7 +43,6 @@ struct BwdLayout {
   static constexpr int QN = bwd_q_rows(D);           // query rows per step
   static constexpr bool DQT = (D == 128);            // dQ produced transposed
   static constexpr int CW = QN / 2;                  // query columns per P/dS warpgroup
-  static constexpr int KPW = CW / 16;                // 16-deep MMA K steps per warpgroup half
   static constexpr int REG = D / 64;                 // 64-column swizzle regions per row
   static constexpr int KREGION = kTileRows * 128;    // region of a 128-row tile
   static constexpr int QREGION = QN * 128;           // region of a QN-row tile

@@ -15,18 +15,19 @@ __global__ void __launch_bounds__(256) commit_kernel(__nv_bfloat16* __restrict__
                                                      const __nv_bfloat16* __restrict__ vs, int cap,
                                                      int slot, int rows, int BH) {
   constexpr int PIECES = D / 8;  // 16-byte pieces per row
-  const size_t idx = static_cast<size_t>(blockIdx.x) * blockDim.x + threadIdx.x;
-  const size_t total = static_cast<size_t>(BH) * rows * PIECES;
-  if (idx >= total) return;
-  const int piece = static_cast<int>(idx % PIECES);
-  const size_t src_row = idx / PIECES;  // over BH * rows
-  const size_t bh = src_row / rows;
-  const int r = static_cast<int>(src_row % rows);
-  const int dst = (slot + r) % cap;
-  const size_t so = src_row * D + piece * 8;
-  const size_t dso = (bh * cap + dst) * D + piece * 8;
-  *reinterpret_cast<uint4*>(kc + dso) = *reinterpret_cast<const uint4*>(ks + so);
-  *reinterpret_cast<uint4*>(vc + dso) = *reinterpret_cast<const uint4*>(vs + so);
+  // grid: x covers rows * PIECES of one head, y strides over the heads
+  const int idx = blockIdx.x * blockDim.x + threadIdx.x;
+  if (idx >= rows * PIECES) return;
+  const int piece = idx % PIECES;
+  const int r = idx / PIECES;
+  int dst = slot + r;
+  if (dst >= cap) dst -= cap;  // slot < cap and rows <= cap
+  for (int bh = blockIdx.y; bh < BH; bh += gridDim.y) {
+    const size_t so = (static_cast<size_t>(bh) * rows + r) * D + piece * 8;
+    const size_t dso = (static_cast<size_t>(bh) * cap + dst) * D + piece * 8;
+    *reinterpret_cast<uint4*>(kc + dso) = *reinterpret_cast<const uint4*>(ks + so);
+    *reinterpret_cast<uint4*>(vc + dso) = *reinterpret_cast<const uint4*>(vs + so);
+  }
 }
 
 }  // namespace
@@ -34,9 +35,10 @@ __global__ void __launch_bounds__(256) commit_kernel(__nv_bfloat16* __restrict__
 cudaError_t launch_commit(int d, __nv_bfloat16* kc, __nv_bfloat16* vc, const __nv_bfloat16* ks,
                           const __nv_bfloat16* vs, int cap, int slot, int rows, int BH,
                           cudaStream_t s) {
-  const size_t total = static_cast<size_t>(BH) * rows * (d / 8);
-  if (total == 0) return cudaSuccess;
-  const unsigned grid = static_cast<unsigned>((total + 255) / 256);
+  const int per_head = rows * (d / 8);
+  if (per_head == 0 || BH == 0) return cudaSuccess;
+  const dim3 grid(static_cast<unsigned>((per_head + 255) / 256),
+                  static_cast<unsigned>(BH < 65535 ? BH : 65535));
   if (d == 64)
     commit_kernel<64><<<grid, 256, 0, s>>>(kc, vc, ks, vs, cap, slot, rows, BH);
   else

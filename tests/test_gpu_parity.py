@@ -286,3 +286,41 @@ def test_pipelined_config(mw):
 def test_device_status_is_clean(mw):
     torch.cuda.synchronize()
     assert mw.mw_device_status() == 0
+
+
+def test_cuda_graph_replay_matches_eager(mw):
+    """A training step and a streaming step captured once as CUDA graphs and
+    replayed give the eager results (the entry points only enqueue work on
+    the caller's stream)."""
+    B, H, n, T, d = 1, 2, 3, 128, 64
+    q, k, v, do = (t.cuda() for t in _inputs(B, H, n, T, d, seed=21))
+    o_e, lse_e = mw.mw_bca_fwd(q, k, v, T)
+    dq_e, dk_e, dv_e = mw.mw_bca_bwd(q, k, v, o_e, lse_e, do, T)
+    ws = torch.empty(mw.mw_bca_bwd_workspace_size(B, H, n, T, d), dtype=torch.uint8, device="cuda")
+    cq, ckn, cvn, ckr, cvr = (t.cuda() for t in _ring_case(1, 2, 2, 64, 512, 128, seed=22))
+    cws = torch.empty(max(1, mw.mw_bca_cache_workspace_size(1, 2, 2, 64, 128, 512)),
+                      dtype=torch.uint8, device="cuda")
+    co_e, clse_e = mw.mw_bca_cache_fwd(cq, ckn, cvn, ckr, cvr, 100, 512, 64, workspace=cws)
+    kr_g, vr_g = ckr.clone(), cvr.clone()
+    kr_e, vr_e = ckr.clone(), cvr.clone()
+    mw.mw_bca_cache_commit(kr_e, vr_e, 100, ckn, cvn)
+    out = {}
+    graph = torch.cuda.CUDAGraph()
+    side = torch.cuda.Stream()
+    side.wait_stream(torch.cuda.current_stream())
+    with torch.cuda.stream(side):
+        with torch.cuda.graph(graph, stream=side):
+            out["o"], out["lse"] = mw.mw_bca_fwd(q, k, v, T)
+            out["grads"] = mw.mw_bca_bwd(q, k, v, out["o"], out["lse"], do, T, workspace=ws)
+            out["co"], out["clse"] = mw.mw_bca_cache_fwd(cq, ckn, cvn, kr_g, vr_g, 100, 512, 64,
+                                                         workspace=cws)
+            mw.mw_bca_cache_commit(kr_g, vr_g, 100, ckn, cvn)
+    torch.cuda.current_stream().wait_stream(side)
+    graph.replay()
+    torch.cuda.synchronize()
+    assert torch.equal(out["o"], o_e) and torch.equal(out["lse"], lse_e)
+    for g_, e_ in zip(out["grads"], (dq_e, dk_e, dv_e)):
+        assert float((g_.float() - e_.float()).abs().max()) <= 1e-2
+    assert torch.equal(out["co"], co_e) and torch.equal(out["clse"], clse_e)
+    assert torch.equal(kr_g, kr_e) and torch.equal(vr_g, vr_e)
+    assert mw.mw_device_status() == 0
