@@ -87,21 +87,25 @@ PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
   return fn;
 }
 
-// 3-D map over [BH, rows, d] bf16 with 64 x 128-row boxes and the 128-byte
-// swizzle the tcgen05 descriptors expect; rows past the end read as zero.
+// 3-D map over [BH, rows, d] with the 128-byte swizzle the tcgen05
+// descriptors and the drain's boxes use; rows past the end read as zero.
+// bf16 operands: 64-column x box_rows boxes.  f32 (the dQ accumulator):
+// 32-column x box_rows boxes.
 mw_status encode_map(CUtensorMap* m, const void* ptr, int rows, int BH, int d, const char* name,
-                     int box_rows) {
+                     int box_rows, bool f32 = false) {
   auto fn = encode_fn();
   if (!fn) return fail(MW_ERR_CUDA, "cuTensorMapEncodeTiled is unavailable (no CUDA driver?)");
+  const cuuint64_t es = f32 ? 4 : 2;
   cuuint64_t dims[3] = {static_cast<cuuint64_t>(d), static_cast<cuuint64_t>(rows),
                         static_cast<cuuint64_t>(BH)};
-  cuuint64_t strides[2] = {static_cast<cuuint64_t>(d) * 2,
-                           static_cast<cuuint64_t>(rows) * d * 2};
-  cuuint32_t box[3] = {64, static_cast<cuuint32_t>(box_rows), 1};
+  cuuint64_t strides[2] = {static_cast<cuuint64_t>(d) * es,
+                           static_cast<cuuint64_t>(rows) * d * es};
+  cuuint32_t box[3] = {f32 ? 32u : 64u, static_cast<cuuint32_t>(box_rows), 1};
   cuuint32_t estr[3] = {1, 1, 1};
-  CUresult r = fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(ptr), dims, strides, box,
-                  estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
-                  CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  CUresult r = fn(m, f32 ? CU_TENSOR_MAP_DATA_TYPE_FLOAT32 : CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3,
+                  const_cast<void*>(ptr), dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
+                  CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                  CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
   if (r != CUDA_SUCCESS) return fail(MW_ERR_CUDA, "cuTensorMapEncodeTiled(%s) failed: %d", name, (int)r);
   return MW_OK;
 }
@@ -112,8 +116,10 @@ mw_status encode_map(CUtensorMap* m, const void* ptr, int rows, int BH, int d, c
 struct MapKey {
   const void* ptr;
   int rows, BH, d, box_rows;
+  bool f32;
   bool operator==(const MapKey& o) const {
-    return ptr == o.ptr && rows == o.rows && BH == o.BH && d == o.d && box_rows == o.box_rows;
+    return ptr == o.ptr && rows == o.rows && BH == o.BH && d == o.d && box_rows == o.box_rows &&
+           f32 == o.f32;
   }
 };
 constexpr int kMapCache = 16;
@@ -122,15 +128,15 @@ thread_local CUtensorMap t_maps[kMapCache];
 thread_local int t_map_next = 0;
 
 mw_status make_map(CUtensorMap* m, const void* ptr, int rows, int BH, int d, const char* name,
-                   int box_rows = mw::kTileRows) {
-  const MapKey key{ptr, rows, BH, d, box_rows};
+                   int box_rows = mw::kTileRows, bool f32 = false) {
+  const MapKey key{ptr, rows, BH, d, box_rows, f32};
   for (int i = 0; i < kMapCache; ++i) {
     if (t_map_keys[i].ptr != nullptr && t_map_keys[i] == key) {
       *m = t_maps[i];
       return MW_OK;
     }
   }
-  MW_TRY(encode_map(m, ptr, rows, BH, d, name, box_rows));
+  MW_TRY(encode_map(m, ptr, rows, BH, d, name, box_rows, f32));
   const int slot = t_map_next;
   t_map_next = (t_map_next + 1) % kMapCache;
   t_map_keys[slot] = key;
@@ -410,12 +416,13 @@ mw_status mw_bca_bwd_stage(int stage, const void* q, const void* k, const void* 
   if (main) {
     unsigned* status = nullptr;
     MW_TRY(status_ptr(&status));
-    CUtensorMap tq, tk, tv, tdo;
+    CUtensorMap tq, tk, tv, tdo, tdq;
     const int qrows = mw::bwd_q_rows(d);  // query rows per backward step
     MW_TRY(make_map(&tq, q, static_cast<int>(N), BH, d, "q", qrows));
     MW_TRY(make_map(&tk, k, static_cast<int>(N), BH, d, "k"));
     MW_TRY(make_map(&tv, v, static_cast<int>(N), BH, d, "v"));
     MW_TRY(make_map(&tdo, dout, static_cast<int>(N), BH, d, "dout", qrows));
+    MW_TRY(make_map(&tdq, dq_acc, N_pad, BH, d, "dq_acc", 32, true));
     mw::BwdParams p{};
     p.BH = BH;
     p.N = static_cast<int>(N);
@@ -430,7 +437,7 @@ mw_status mw_bca_bwd_stage(int stage, const void* q, const void* k, const void* 
     p.dv = static_cast<__nv_bfloat16*>(dv);
     p.status = status;
     p.budget_ns = budget_ns();
-    MW_TRY(launch_status(mw::launch_bwd_main(d, tq, tk, tv, tdo, p, s), "backward kernel launch"));
+    MW_TRY(launch_status(mw::launch_bwd_main(d, tq, tk, tv, tdo, tdq, p, s), "backward kernel launch"));
   }
   if (post)
     MW_TRY(launch_status(mw::launch_bwd_post(d, dq_acc, static_cast<__nv_bfloat16*>(dq), scale, BH,

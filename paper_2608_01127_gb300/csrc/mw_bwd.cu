@@ -51,7 +51,9 @@ struct BwdLayout {
   static constexpr int STAGES = (D == 64) ? 3 : 2;   // Q and dO tiles in flight
   static constexpr int DS_BYTES = (QN / 64) * KREGION;  // dS^T: 128 key rows x QN columns
   static constexpr int DS_BUFS = 1;
-  static constexpr int STG_BYTES = DQT ? 0 : 4 * 32 * D * 4;  // per-warp dQ staging (d = 64)
+  // d = 64: per drain warp, its 32 x D dQ block as 32-column f32 boxes with the
+  // 128-byte swizzle (the TMA reduce-add source); 1024-byte aligned
+  static constexpr int STG_BYTES = DQT ? 0 : 4 * 32 * D * 4;
   static constexpr int VEC_BYTES = QN * 4;
   static constexpr int OFF_K = 0;
   static constexpr int OFF_V = OFF_K + KTILE;
@@ -76,20 +78,14 @@ struct BwdLayout {
   static constexpr uint32_t DK_COL = D;
   static constexpr uint32_t S_COL = 2 * D;
   static constexpr uint32_t DP_COL = SHARED_X ? S_COL : 2 * D + QN;
-  // P^T then dS^T (bf16 pairs); at d = 64 dQ_j reuses the dS^T half (it is
-  // written after dK_j has read dS^T_j, and the next dS^T waits for the drain)
+  // P^T (bf16 pairs; at d = 128 followed by dS^T).  At d = 64 dK reads dS^T
+  // from shared memory (the copy dQ reads too), so dQ has columns of its own.
   static constexpr uint32_t PDS_COL = SHARED_X ? S_COL : 384u;
   static constexpr uint32_t DQ_COL = SHARED_X ? 384u : 448u;
   static constexpr int THREADS = 512;
   static_assert(SHARED_X ? (2 * D + QN <= 384) : (2 * D + 2 * QN <= 384), "TMEM columns");
   static_assert(BYTES <= 232448, "shared memory");
 };
-
-__device__ __forceinline__ void red_add_v4(float* addr, float a, float b, float c, float d) {
-  asm volatile("red.global.add.v4.f32 [%0], {%1, %2, %3, %4};" ::"l"(addr), "f"(a), "f"(b),
-               "f"(c), "f"(d)
-               : "memory");
-}
 
 __device__ __forceinline__ void red_add(float* addr, float a) {
   asm volatile("red.global.add.f32 [%0], %1;" ::"l"(addr), "f"(a) : "memory");
@@ -99,7 +95,7 @@ template <int D>
 __global__ void __launch_bounds__(BwdLayout<D>::THREADS, 1)
     bca_bwd_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_k,
                    const __grid_constant__ CUtensorMap tm_v, const __grid_constant__ CUtensorMap tm_do,
-                   const BwdParams p) {
+                   const __grid_constant__ CUtensorMap tm_dq, const BwdParams p) {
   using L = BwdLayout<D>;
   constexpr int NS = L::STAGES;
   constexpr int QN = L::QN;
@@ -141,6 +137,10 @@ __global__ void __launch_bounds__(BwdLayout<D>::THREADS, 1)
   const int first_q = (k0 / p.T) * p.T;  // first query that sees key k0
   const int m_begin = first_q / QN;
   const int n_q = p.N_pad / QN - m_begin;
+  // each key tile starts its sweep over the query tiles at its own offset, so
+  // that the key tiles of one head running side by side reduce into different
+  // dQ tiles instead of contending for the same L2 lines
+  const int q_rot = kt % n_q;
 
   if (threadIdx.x == 0) {
     mbar_init(kv_full, 1);
@@ -196,7 +196,7 @@ __global__ void __launch_bounds__(BwdLayout<D>::THREADS, 1)
       for (int j = 0; j < n_q; ++j) {
         const int st = j % NS;
         const uint32_t ph = (j / NS) & 1;
-        const int q0 = (m_begin + j) * QN;
+        const int q0 = (m_begin + (j + q_rot) % n_q) * QN;
         const size_t voff = static_cast<size_t>(bh) * p.N_pad + q0;
         if (!mbar_wait(&q_empty[st], ph ^ 1, ctl)) break;
         mbar_arrive_expect_tx(&q_full[st], L::QTILE + L::VEC_BYTES);
@@ -220,8 +220,8 @@ __global__ void __launch_bounds__(BwdLayout<D>::THREADS, 1)
       }
     }
   } else if (warp == 13) {
-    // ------------------------------------------------------------ MMA issuer
-    if (lane == 0) {
+    // ------------------------------------------------------------ MMA issuer (whole warp)
+    {
       constexpr uint32_t idesc_s = idesc_bf16_f32(128, QN, false, false);    // S^T, dP^T
       constexpr uint32_t idesc_tn = idesc_bf16_f32(128, D, false, true);     // dV, dK
       // d = 64: dQ = dS K (M = query rows); d = 128: dQ^T = K^T dS^T (M = head dim)
@@ -236,6 +236,7 @@ __global__ void __launch_bounds__(BwdLayout<D>::THREADS, 1)
       const uint64_t q_mn0 = sdesc_sw128(smem_u32(sQ), L::QREGION, 1024);
       const uint64_t do_mn0 = sdesc_sw128(smem_u32(sDO), L::QREGION, 1024);
       const uint64_t ds_mn0 = sdesc_sw128(smem_u32(sDS), L::KREGION, 1024);
+      const uint64_t ds_kmaj0 = sdesc_sw128(smem_u32(sDS), 16, 1024);
       // X = A B^T, both K-major over d (S^T = K Q^T, dP^T = V dO^T)
       auto issue_kmajor = [&](uint32_t d_col, uint64_t a, uint64_t b) {
 #pragma unroll
@@ -253,14 +254,14 @@ __global__ void __launch_bounds__(BwdLayout<D>::THREADS, 1)
         return L::SHARED_X ? L::PDS_COL + (kk >> 2) * 64 + 32 + (kk & 3) * 8
                            : L::PDS_COL + QN / 2 + kk * 8;
       };
-      bool ok = mbar_wait(kv_full, 0, ctl);
-      if (ok) ok = mbar_wait(&q_full[0], 0, ctl);
+      bool ok = warp_wait(kv_full, 0, ctl);
+      if (ok) ok = warp_wait(&q_full[0], 0, ctl);
       tc_fence_after();
       if (ok) {
         issue_kmajor(L::S_COL, k_kmaj, q_kmaj0);
         umma_commit(s_full);
-        if (L::SHARED_X) ok = mbar_wait(s_free, 0, ctl);  // X holds S^T_0 until read
-        if (ok) ok = mbar_wait(&do_full[0], 0, ctl);
+        if (L::SHARED_X) ok = warp_wait(s_free, 0, ctl);  // X holds S^T_0 until read
+        if (ok) ok = warp_wait(&do_full[0], 0, ctl);
         tc_fence_after();
       }
       if (ok) {
@@ -276,14 +277,14 @@ __global__ void __launch_bounds__(BwdLayout<D>::THREADS, 1)
         const uint64_t q_mn = sdesc_add(q_mn0, st * L::QTILE);
         if (!L::SHARED_X && more) {
           // S^T of the next step as soon as the P/dS warps hold S^T_j
-          if (!(ok = mbar_wait(s_free, j & 1, ctl))) break;
-          if (!(ok = mbar_wait(&q_full[st1], ph1, ctl))) break;
+          if (!(ok = warp_wait(s_free, j & 1, ctl))) break;
+          if (!(ok = warp_wait(&q_full[st1], ph1, ctl))) break;
           tc_fence_after();
           issue_kmajor(L::S_COL, k_kmaj, sdesc_add(q_kmaj0, st1 * L::QTILE));
           umma_commit(s_full);
         }
         // dV += P^T dO_j as soon as P^T_j is in TMEM (while dS_j is computed)
-        if (!(ok = mbar_wait(pt_ready, j & 1, ctl))) break;
+        if (!(ok = warp_wait(pt_ready, j & 1, ctl))) break;
         tc_fence_after();
 #pragma unroll
         for (int kk = 0; kk < QN / 16; ++kk)
@@ -293,37 +294,42 @@ __global__ void __launch_bounds__(BwdLayout<D>::THREADS, 1)
         if (!L::SHARED_X) umma_commit(pt_free);
         if (!L::SHARED_X && more) {
           // dP^T of the next step once the P/dS warps hold dP^T_j
-          if (!(ok = mbar_wait(dp_free, j & 1, ctl))) break;
-          if (!(ok = mbar_wait(&do_full[st1], ph1, ctl))) break;
+          if (!(ok = warp_wait(dp_free, j & 1, ctl))) break;
+          if (!(ok = warp_wait(&do_full[st1], ph1, ctl))) break;
           tc_fence_after();
           issue_kmajor(L::DP_COL, v_kmaj, sdesc_add(do_kmaj0, st1 * L::QTILE));
           umma_commit(dp_full);
         }
-        if (!(ok = mbar_wait(p_ready, j & 1, ctl))) break;
+        if (!(ok = warp_wait(p_ready, j & 1, ctl))) break;
         tc_fence_after();
-        // dK += dS^T Q_j
+        // dK += dS^T Q_j (d = 64: dS^T read from shared memory, K-major)
+        const uint64_t ds_kmaj = sdesc_add(ds_kmaj0, (j % L::DS_BUFS) * L::DS_BYTES);
 #pragma unroll
-        for (int kk = 0; kk < QN / 16; ++kk)
-          umma_ts(tmem + L::DK_COL, tmem + dst_col(kk), sdesc_add(q_mn, kk * 2048),
-                  idesc_tn, (j > 0 || kk > 0) ? 1u : 0u);
+        for (int kk = 0; kk < QN / 16; ++kk) {
+          if constexpr (L::SHARED_X)
+            umma_ts(tmem + L::DK_COL, tmem + dst_col(kk), sdesc_add(q_mn, kk * 2048),
+                    idesc_tn, (j > 0 || kk > 0) ? 1u : 0u);
+          else
+            umma_ss(tmem + L::DK_COL, sdesc_add(ds_kmaj, (kk >> 2) * L::KREGION + (kk & 3) * 32),
+                    sdesc_add(q_mn, kk * 2048), idesc_tn, (j > 0 || kk > 0) ? 1u : 0u);
+        }
         umma_commit(&q_empty[st]);
         if (L::SHARED_X && more) {
           // X is free once dV/dK have read P^T/dS^T (issue order): S^T of the
           // next step, then its dP^T once the P/dS warps have read that S^T
-          if (!(ok = mbar_wait(&q_full[st1], ph1, ctl))) break;
+          if (!(ok = warp_wait(&q_full[st1], ph1, ctl))) break;
           tc_fence_after();
           issue_kmajor(L::S_COL, k_kmaj, sdesc_add(q_kmaj0, st1 * L::QTILE));
           umma_commit(s_full);
-          if (!(ok = mbar_wait(s_free, (j + 1) & 1, ctl))) break;
-          if (!(ok = mbar_wait(&do_full[st1], ph1, ctl))) break;
+          if (!(ok = warp_wait(s_free, (j + 1) & 1, ctl))) break;
+          if (!(ok = warp_wait(&do_full[st1], ph1, ctl))) break;
           tc_fence_after();
           issue_kmajor(L::DP_COL, v_kmaj, sdesc_add(do_kmaj0, st1 * L::QTILE));
           umma_commit(dp_full);
         }
-        // dQ of this step; at d = 128 once the drain has read the previous one
-        // (at d = 64 the P/dS warps waited for that drain before writing dS^T_j)
-        if (L::SHARED_X && j > 0) {
-          if (!(ok = mbar_wait(dq_free, (j - 1) & 1, ctl))) break;
+        // dQ of this step, once the drain has read the previous one
+        if (j > 0) {
+          if (!(ok = warp_wait(dq_free, (j - 1) & 1, ctl))) break;
           tc_fence_after();
         }
         const uint64_t ds_mn = sdesc_add(ds_mn0, (j % L::DS_BUFS) * L::DS_BYTES);
@@ -365,7 +371,7 @@ __global__ void __launch_bounds__(BwdLayout<D>::THREADS, 1)
     bool ok = true;
     for (int j = 0; j < n_q; ++j) {
       const int st = j % NS;
-      const int q0 = (m_begin + j) * QN;
+      const int q0 = (m_begin + (j + q_rot) % n_q) * QN;
       const float* lse2 = sLSE + st * QN + c0;
       const float* delta = sDelta + st * QN + c0;
       if (!(ok = warp_wait(s_full, j & 1, ctl))) break;
@@ -469,20 +475,13 @@ __global__ void __launch_bounds__(BwdLayout<D>::THREADS, 1)
       for (int q = 0; q < CW / 8; ++q)
         *reinterpret_cast<uint4*>(ds_row + (((chunk0 + q) ^ sw) << 4)) =
             make_uint4(dk[4 * q], dk[4 * q + 1], dk[4 * q + 2], dk[4 * q + 3]);
-      // dS^T -> TMEM (d = 64: once the drain has read dQ_{j-1}, which shares
-      // these columns)
-      if (!L::SHARED_X && j > 0) {
-        if (!(ok = warp_wait(dq_free, (j - 1) & 1, ctl))) break;
-        tc_fence_after();
-      }
+      // d = 128: P^T and dS^T -> TMEM (the dK and dV A operands)
       if constexpr (L::SHARED_X) {
         tmem_st32(pds_p, pk);
         tmem_st32(pds_s, dk);
-      } else {
-        tmem_st32(pds_s, dk);
       }
       fence_proxy_async_smem();
-      tmem_wait_st();
+      if constexpr (L::SHARED_X) tmem_wait_st();
       tc_fence_before();
       __syncwarp();
       if (lane == 0) {
@@ -519,7 +518,7 @@ __global__ void __launch_bounds__(BwdLayout<D>::THREADS, 1)
     const int wq = warp & 3;
     const uint32_t lane_base = tmem + (static_cast<uint32_t>(wq * 32) << 16);
     for (int j = 0; j < n_q; ++j) {
-      const int q0 = (m_begin + j) * QN;
+      const int q0 = (m_begin + (j + q_rot) % n_q) * QN;
       if (!warp_wait(dq_full, j & 1, ctl)) break;
       tc_fence_after();
       if constexpr (L::DQT) {
@@ -544,39 +543,42 @@ __global__ void __launch_bounds__(BwdLayout<D>::THREADS, 1)
           }
         }
       } else {
-        // lanes = query rows; stage the warp's 32 x D block in shared memory
-        // (16-byte chunk f of row r at position (f + r) mod 16: conflict-free
-        // both ways), then reduce it row-contiguously
-        constexpr int CH = D / 4;  // 16-byte chunks per row
+        // lanes = query rows: the warp's 32 x D block goes to shared memory as
+        // 32-column boxes with the 128-byte swizzle (16-byte chunk c of row r
+        // at c ^ (r mod 8): conflict-free), and one lane hands each box to the
+        // TMA unit as a reduce-add into dQacc
         uint8_t* stg = smem + L::OFF_STG + wq * (32 * D * 4);
+        if (lane == 0) bulk_wait_read_all();  // the previous step's boxes were read
+        __syncwarp();
 #pragma unroll
         for (int c = 0; c < D / 32; ++c) {
           uint32_t r[32];
           tmem_ld32(lane_base + L::DQ_COL + 32 * c, r);
           tmem_wait_ld();
-#pragma unroll
-          for (int i = 0; i < 8; ++i) {
-            const int f = 8 * c + i;
-            *reinterpret_cast<uint4*>(stg + lane * (D * 4) + (((f + lane) % CH) << 4)) =
-                make_uint4(r[4 * i], r[4 * i + 1], r[4 * i + 2], r[4 * i + 3]);
+          if (c == D / 32 - 1) {
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(dq_free);
           }
-        }
-        tc_fence_before();
-        __syncwarp();
-        if (lane == 0) mbar_arrive(dq_free);
-        constexpr int ROWS_PER = 32 / CH;  // rows covered by one warp instruction
-        float* base = p.dq_acc + (static_cast<size_t>(bh) * p.N_pad + q0 + wq * 32) * D;
 #pragma unroll
-        for (int k = 0; k < 32 / ROWS_PER; ++k) {
-          const int row = ROWS_PER * k + lane / CH;
-          const int f = lane % CH;
-          const uint4 v =
-              *reinterpret_cast<const uint4*>(stg + row * (D * 4) + (((f + row) % CH) << 4));
-          red_add_v4(base + static_cast<size_t>(row) * D + 4 * f, __uint_as_float(v.x),
-                     __uint_as_float(v.y), __uint_as_float(v.z), __uint_as_float(v.w));
+          for (int i = 0; i < 8; ++i)
+            *reinterpret_cast<uint4*>(stg + c * 4096 + lane * 128 + ((i ^ (lane & 7)) << 4)) =
+                make_uint4(r[4 * i], r[4 * i + 1], r[4 * i + 2], r[4 * i + 3]);
         }
+        fence_proxy_async_smem();
         __syncwarp();
+        if (lane == 0) {
+#pragma unroll
+          for (int c = 0; c < D / 32; ++c)
+            tma_reduce_add_3d(&tm_dq, stg + c * 4096, 32 * c, q0 + wq * 32, bh);
+          bulk_commit_group();
+        }
       }
+    }
+    // every reduce-add has completed before the CTA's shared memory goes away
+    if constexpr (!L::DQT) {
+      if (lane == 0) bulk_wait_all();
+      __syncwarp();
     }
   }
 
@@ -642,7 +644,8 @@ __global__ void __launch_bounds__(256) bwd_post_kernel(const float* __restrict__
 
 template <int D>
 cudaError_t launch_bwd_main_t(const CUtensorMap& tq, const CUtensorMap& tk, const CUtensorMap& tv,
-                              const CUtensorMap& tdo, const BwdParams& p, cudaStream_t s) {
+                              const CUtensorMap& tdo, const CUtensorMap& tdq, const BwdParams& p,
+                              cudaStream_t s) {
   using L = BwdLayout<D>;
   static bool attr_set = false;
   if (!attr_set) {
@@ -652,7 +655,7 @@ cudaError_t launch_bwd_main_t(const CUtensorMap& tq, const CUtensorMap& tk, cons
     attr_set = true;
   }
   const unsigned grid = static_cast<unsigned>(p.BH) * (p.N_pad / kTileRows);
-  bca_bwd_kernel<D><<<grid, L::THREADS, L::BYTES, s>>>(tq, tk, tv, tdo, p);
+  bca_bwd_kernel<D><<<grid, L::THREADS, L::BYTES, s>>>(tq, tk, tv, tdo, tdq, p);
   return cudaGetLastError();
 }
 
@@ -670,10 +673,10 @@ cudaError_t launch_bwd_pre(int d, const __nv_bfloat16* o, const __nv_bfloat16* d
 }
 
 cudaError_t launch_bwd_main(int d, const CUtensorMap& tq, const CUtensorMap& tk,
-                            const CUtensorMap& tv, const CUtensorMap& tdo, const BwdParams& p,
-                            cudaStream_t s) {
-  if (d == 64) return launch_bwd_main_t<64>(tq, tk, tv, tdo, p, s);
-  return launch_bwd_main_t<128>(tq, tk, tv, tdo, p, s);
+                            const CUtensorMap& tv, const CUtensorMap& tdo, const CUtensorMap& tdq,
+                            const BwdParams& p, cudaStream_t s) {
+  if (d == 64) return launch_bwd_main_t<64>(tq, tk, tv, tdo, tdq, p, s);
+  return launch_bwd_main_t<128>(tq, tk, tv, tdo, tdq, p, s);
 }
 
 cudaError_t launch_bwd_post(int d, const float* dq_acc, __nv_bfloat16* dq, float scale, int BH,

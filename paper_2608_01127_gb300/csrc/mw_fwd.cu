@@ -217,8 +217,8 @@ __global__ void __launch_bounds__(FwdLayout<D>::THREADS, 1)
       }
     }
   } else if (warp == 9) {
-    // ------------------------------------------------------------ MMA issuer
-    if (lane == 0 && n_local > 0) {
+    // ------------------------------------------------------------ MMA issuer (whole warp)
+    if (n_local > 0) {
       constexpr uint32_t idesc_qk = idesc_bf16_f32(128, 128, false, false);
       constexpr uint32_t idesc_pv = idesc_bf16_f32(128, L::OW, false, true);
       // descriptors computed once; each MMA adds a compile-time offset
@@ -248,19 +248,19 @@ __global__ void __launch_bounds__(FwdLayout<D>::THREADS, 1)
         }
       };
 
-      bool ok = mbar_wait(q_full, 0, ctl);
+      bool ok = warp_wait(q_full, 0, ctl);
       tc_fence_after();
       for (int i = 0; ok && i < n_local; ++i) {
         const int st = i % NS;
         const uint32_t ph = (i / NS) & 1;
         const int stp = (i + NS - 1) % NS;
         const uint32_t php = ((i - 1) / NS) & 1;
-        if (!(ok = mbar_wait(&k_full[st], ph, ctl))) break;
+        if (!(ok = warp_wait(&k_full[st], ph, ctl))) break;
         tc_fence_after();
         for (int t = 0; t < QT; ++t) {
           if (i > 0) {
-            if (!(ok = mbar_wait(&p_full[t], (i - 1) & 1, ctl))) break;
-            if (t == 0 && !(ok = mbar_wait(&v_full[stp], php, ctl))) break;
+            if (!(ok = warp_wait(&p_full[t], (i - 1) & 1, ctl))) break;
+            if (t == 0 && !(ok = warp_wait(&v_full[stp], php, ctl))) break;
             tc_fence_after();
             issue_pv(t, stp, i - 1 > 0);
           }
@@ -275,8 +275,8 @@ __global__ void __launch_bounds__(FwdLayout<D>::THREADS, 1)
         const int il = n_local - 1;
         const int stl = il % NS;
         for (int t = 0; ok && t < QT; ++t) {
-          if (!(ok = mbar_wait(&p_full[t], il & 1, ctl))) break;
-          if (t == 0 && !(ok = mbar_wait(&v_full[stl], (il / NS) & 1, ctl))) break;
+          if (!(ok = warp_wait(&p_full[t], il & 1, ctl))) break;
+          if (t == 0 && !(ok = warp_wait(&v_full[stl], (il / NS) & 1, ctl))) break;
           tc_fence_after();
           issue_pv(t, stl, il > 0);
         }

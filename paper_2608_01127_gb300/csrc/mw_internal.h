@@ -67,9 +67,11 @@ cudaError_t launch_combine(int d, const float* o_part, const float* lse_part, __
 cudaError_t launch_bwd_pre(int d, const __nv_bfloat16* o, const __nv_bfloat16* dout,
                            const float* lse, float* lse2, float* delta, float* dq_acc, int BH,
                            int N, int N_pad, cudaStream_t s);
+// tdq: f32 map over dQacc [BH, N_pad, d] with 32 x 32 boxes (128-byte
+// swizzle), the target of the d = 64 kernel's TMA reduce-adds
 cudaError_t launch_bwd_main(int d, const CUtensorMap& tq, const CUtensorMap& tk,
-                            const CUtensorMap& tv, const CUtensorMap& tdo, const BwdParams& p,
-                            cudaStream_t s);
+                            const CUtensorMap& tv, const CUtensorMap& tdo, const CUtensorMap& tdq,
+                            const BwdParams& p, cudaStream_t s);
 cudaError_t launch_bwd_post(int d, const float* dq_acc, __nv_bfloat16* dq, float scale, int BH,
                             int N, int N_pad, cudaStream_t s);
 cudaError_t launch_commit(int d, __nv_bfloat16* kc, __nv_bfloat16* vc, const __nv_bfloat16* ks,
