@@ -50,10 +50,11 @@ struct BwdLayout {
   static constexpr int QTILE = REG * QREGION;
   static constexpr int STAGES = (D == 64) ? 3 : 2;   // Q and dO tiles in flight
   static constexpr int DS_BYTES = (QN / 64) * KREGION;  // dS^T: 128 key rows x QN columns
-  static constexpr int DS_BUFS = 1;
-  // d = 64: per drain warp, its 32 x D dQ block as 32-column f32 boxes with the
-  // 128-byte swizzle (the TMA reduce-add source); 1024-byte aligned
-  static constexpr int STG_BYTES = DQT ? 0 : 4 * 32 * D * 4;
+  // d = 64: two dS^T buffers, so dS^T_{j+1} is written while dK_j / dQ_j read dS^T_j
+  static constexpr int DS_BUFS = (D == 64) ? 2 : 1;
+  // d = 64: per drain warp, one 32 x 32 f32 box with the 128-byte swizzle (the
+  // TMA reduce-add source); 1024-byte aligned
+  static constexpr int STG_BYTES = DQT ? 0 : 4 * 32 * 32 * 4;
   static constexpr int VEC_BYTES = QN * 4;
   static constexpr int OFF_K = 0;
   static constexpr int OFF_V = OFF_K + KTILE;
@@ -74,6 +75,7 @@ struct BwdLayout {
   // 128-column block X holds them in turn (each is copied to registers
   // before the next one lands there)
   static constexpr bool SHARED_X = (D == 128);
+  static constexpr bool TWO_ISSUERS = !SHARED_X;  // MMA issue split over warps 13 and 14
   static constexpr uint32_t DV_COL = 0;
   static constexpr uint32_t DK_COL = D;
   static constexpr uint32_t S_COL = 2 * D;
@@ -160,7 +162,7 @@ __global__ void __launch_bounds__(BwdLayout<D>::THREADS, 1)
     mbar_init(dq_full, 1);
     mbar_init(dq_free, 4);
     for (int b = 0; b < L::DS_BUFS; ++b) mbar_init(&ds_free[b], 1);
-    mbar_init(dkv_full, 1);
+    mbar_init(dkv_full, L::TWO_ISSUERS ? 2 : 1);
     *abort_flag = 0;
     fence_mbar_init();
   }
@@ -219,9 +221,15 @@ __global__ void __launch_bounds__(BwdLayout<D>::THREADS, 1)
           drain_wait(&do_full[j % NS], (j / NS) & 1, p.budget_ns);
       }
     }
-  } else if (warp == 13) {
-    // ------------------------------------------------------------ MMA issuer (whole warp)
+  } else if (warp == 13 || (L::TWO_ISSUERS && warp == 14)) {
+    // ------------------------------------------------------------ MMA issuers (whole warps)
+    // d = 64: warp 13 issues S^T, dV and dP^T, warp 14 dK and dQ, so that one
+    // warp's waits never leave the tensor core's short queue empty.  They
+    // share no TMEM columns; the P/dS barriers order their operands.
+    // d = 128 (S^T, dP^T, P^T and dS^T share columns): warp 13 issues all.
     {
+      const bool role_a = !L::TWO_ISSUERS || warp == 13;  // S^T, dV, dP^T
+      const bool role_b = !L::TWO_ISSUERS || warp == 14;  // dK, dQ
       constexpr uint32_t idesc_s = idesc_bf16_f32(128, QN, false, false);    // S^T, dP^T
       constexpr uint32_t idesc_tn = idesc_bf16_f32(128, D, false, true);     // dV, dK
       // d = 64: dQ = dS K (M = query rows); d = 128: dQ^T = K^T dS^T (M = head dim)
@@ -255,16 +263,16 @@ __global__ void __launch_bounds__(BwdLayout<D>::THREADS, 1)
                            : L::PDS_COL + QN / 2 + kk * 8;
       };
       bool ok = warp_wait(kv_full, 0, ctl);
-      if (ok) ok = warp_wait(&q_full[0], 0, ctl);
+      if (ok && role_a) ok = warp_wait(&q_full[0], 0, ctl);
       tc_fence_after();
-      if (ok) {
+      if (ok && role_a) {
         issue_kmajor(L::S_COL, k_kmaj, q_kmaj0);
         umma_commit(s_full);
         if (L::SHARED_X) ok = warp_wait(s_free, 0, ctl);  // X holds S^T_0 until read
         if (ok) ok = warp_wait(&do_full[0], 0, ctl);
         tc_fence_after();
       }
-      if (ok) {
+      if (ok && role_a) {
         issue_kmajor(L::DP_COL, v_kmaj, do_kmaj0);
         umma_commit(dp_full);
       }
@@ -275,45 +283,49 @@ __global__ void __launch_bounds__(BwdLayout<D>::THREADS, 1)
         const bool more = j + 1 < n_q;
         const uint64_t do_mn = sdesc_add(do_mn0, st * L::QTILE);
         const uint64_t q_mn = sdesc_add(q_mn0, st * L::QTILE);
-        if (!L::SHARED_X && more) {
-          // S^T of the next step as soon as the P/dS warps hold S^T_j
-          if (!(ok = warp_wait(s_free, j & 1, ctl))) break;
-          if (!(ok = warp_wait(&q_full[st1], ph1, ctl))) break;
+        if (role_a) {
+          if (!L::SHARED_X && more) {
+            // S^T of the next step as soon as the P/dS warps hold S^T_j
+            if (!(ok = warp_wait(s_free, j & 1, ctl))) break;
+            if (!(ok = warp_wait(&q_full[st1], ph1, ctl))) break;
+            tc_fence_after();
+            issue_kmajor(L::S_COL, k_kmaj, sdesc_add(q_kmaj0, st1 * L::QTILE));
+            umma_commit(s_full);
+          }
+          // dV += P^T dO_j as soon as P^T_j is in TMEM (while dS_j is computed)
+          if (!(ok = warp_wait(pt_ready, j & 1, ctl))) break;
           tc_fence_after();
-          issue_kmajor(L::S_COL, k_kmaj, sdesc_add(q_kmaj0, st1 * L::QTILE));
-          umma_commit(s_full);
-        }
-        // dV += P^T dO_j as soon as P^T_j is in TMEM (while dS_j is computed)
-        if (!(ok = warp_wait(pt_ready, j & 1, ctl))) break;
-        tc_fence_after();
 #pragma unroll
-        for (int kk = 0; kk < QN / 16; ++kk)
-          umma_ts(tmem + L::DV_COL, tmem + pt_col(kk), sdesc_add(do_mn, kk * 2048),
-                  idesc_tn, (j > 0 || kk > 0) ? 1u : 0u);
-        umma_commit(&do_empty[st]);
-        if (!L::SHARED_X) umma_commit(pt_free);
-        if (!L::SHARED_X && more) {
-          // dP^T of the next step once the P/dS warps hold dP^T_j
-          if (!(ok = warp_wait(dp_free, j & 1, ctl))) break;
-          if (!(ok = warp_wait(&do_full[st1], ph1, ctl))) break;
-          tc_fence_after();
-          issue_kmajor(L::DP_COL, v_kmaj, sdesc_add(do_kmaj0, st1 * L::QTILE));
-          umma_commit(dp_full);
-        }
-        if (!(ok = warp_wait(p_ready, j & 1, ctl))) break;
-        tc_fence_after();
-        // dK += dS^T Q_j (d = 64: dS^T read from shared memory, K-major)
-        const uint64_t ds_kmaj = sdesc_add(ds_kmaj0, (j % L::DS_BUFS) * L::DS_BYTES);
-#pragma unroll
-        for (int kk = 0; kk < QN / 16; ++kk) {
-          if constexpr (L::SHARED_X)
-            umma_ts(tmem + L::DK_COL, tmem + dst_col(kk), sdesc_add(q_mn, kk * 2048),
+          for (int kk = 0; kk < QN / 16; ++kk)
+            umma_ts(tmem + L::DV_COL, tmem + pt_col(kk), sdesc_add(do_mn, kk * 2048),
                     idesc_tn, (j > 0 || kk > 0) ? 1u : 0u);
-          else
-            umma_ss(tmem + L::DK_COL, sdesc_add(ds_kmaj, (kk >> 2) * L::KREGION + (kk & 3) * 32),
-                    sdesc_add(q_mn, kk * 2048), idesc_tn, (j > 0 || kk > 0) ? 1u : 0u);
+          umma_commit(&do_empty[st]);
+          if (!L::SHARED_X) umma_commit(pt_free);
+          if (!L::SHARED_X && more) {
+            // dP^T of the next step once the P/dS warps hold dP^T_j
+            if (!(ok = warp_wait(dp_free, j & 1, ctl))) break;
+            if (!(ok = warp_wait(&do_full[st1], ph1, ctl))) break;
+            tc_fence_after();
+            issue_kmajor(L::DP_COL, v_kmaj, sdesc_add(do_kmaj0, st1 * L::QTILE));
+            umma_commit(dp_full);
+          }
         }
-        umma_commit(&q_empty[st]);
+        if (role_b) {
+          if (!(ok = warp_wait(p_ready, j & 1, ctl))) break;
+          tc_fence_after();
+          // dK += dS^T Q_j (d = 64: dS^T read from shared memory, K-major)
+          const uint64_t ds_kmaj = sdesc_add(ds_kmaj0, (j % L::DS_BUFS) * L::DS_BYTES);
+#pragma unroll
+          for (int kk = 0; kk < QN / 16; ++kk) {
+            if constexpr (L::SHARED_X)
+              umma_ts(tmem + L::DK_COL, tmem + dst_col(kk), sdesc_add(q_mn, kk * 2048),
+                      idesc_tn, (j > 0 || kk > 0) ? 1u : 0u);
+            else
+              umma_ss(tmem + L::DK_COL, sdesc_add(ds_kmaj, (kk >> 2) * L::KREGION + (kk & 3) * 32),
+                      sdesc_add(q_mn, kk * 2048), idesc_tn, (j > 0 || kk > 0) ? 1u : 0u);
+          }
+          umma_commit(&q_empty[st]);
+        }
         if (L::SHARED_X && more) {
           // X is free once dV/dK have read P^T/dS^T (issue order): S^T of the
           // next step, then its dP^T once the P/dS warps have read that S^T
@@ -327,25 +339,27 @@ __global__ void __launch_bounds__(BwdLayout<D>::THREADS, 1)
           issue_kmajor(L::DP_COL, v_kmaj, sdesc_add(do_kmaj0, st1 * L::QTILE));
           umma_commit(dp_full);
         }
-        // dQ of this step, once the drain has read the previous one
-        if (j > 0) {
-          if (!(ok = warp_wait(dq_free, (j - 1) & 1, ctl))) break;
-          tc_fence_after();
-        }
-        const uint64_t ds_mn = sdesc_add(ds_mn0, (j % L::DS_BUFS) * L::DS_BYTES);
+        if (role_b) {
+          // dQ of this step, once the drain has read the previous one
+          if (j > 0) {
+            if (!(ok = warp_wait(dq_free, (j - 1) & 1, ctl))) break;
+            tc_fence_after();
+          }
+          const uint64_t ds_mn = sdesc_add(ds_mn0, (j % L::DS_BUFS) * L::DS_BYTES);
 #pragma unroll
-        for (int kk = 0; kk < kTileRows / 16; ++kk) {
-          if constexpr (L::DQT)   // A = K^T (MN-major over d), B = dS^T (MN-major over queries)
-            umma_ss(tmem + L::DQ_COL, sdesc_add(k_mn, kk * 2048), sdesc_add(ds_mn, kk * 2048),
-                    idesc_dq, kk > 0 ? 1u : 0u);
-          else                    // A = dS (MN-major over queries), B = K (MN-major over d)
-            umma_ss(tmem + L::DQ_COL, sdesc_add(ds_mn, kk * 2048), sdesc_add(k_mn, kk * 2048),
-                    idesc_dq, kk > 0 ? 1u : 0u);
+          for (int kk = 0; kk < kTileRows / 16; ++kk) {
+            if constexpr (L::DQT)   // A = K^T (MN-major over d), B = dS^T (MN-major over queries)
+              umma_ss(tmem + L::DQ_COL, sdesc_add(k_mn, kk * 2048), sdesc_add(ds_mn, kk * 2048),
+                      idesc_dq, kk > 0 ? 1u : 0u);
+            else                    // A = dS (MN-major over queries), B = K (MN-major over d)
+              umma_ss(tmem + L::DQ_COL, sdesc_add(ds_mn, kk * 2048), sdesc_add(k_mn, kk * 2048),
+                      idesc_dq, kk > 0 ? 1u : 0u);
+          }
+          umma_commit(dq_full);
+          umma_commit(&ds_free[j % L::DS_BUFS]);
         }
-        umma_commit(dq_full);
-        umma_commit(&ds_free[j % L::DS_BUFS]);
       }
-      if (ok) umma_commit(dkv_full);
+      if (ok) umma_commit(dkv_full);  // one arrival per issuing warp
     }
   } else if (warp < 8) {
     // ------------------------------------------------------------ P / dS (thread = key row)
@@ -547,31 +561,29 @@ __global__ void __launch_bounds__(BwdLayout<D>::THREADS, 1)
         // 32-column boxes with the 128-byte swizzle (16-byte chunk c of row r
         // at c ^ (r mod 8): conflict-free), and one lane hands each box to the
         // TMA unit as a reduce-add into dQacc
-        uint8_t* stg = smem + L::OFF_STG + wq * (32 * D * 4);
-        if (lane == 0) bulk_wait_read_all();  // the previous step's boxes were read
+        static_assert(D == 64, "the drain below covers two 32-column boxes");
+        uint8_t* stg = smem + L::OFF_STG + wq * 4096;
+        uint32_t r[2][32];
+        tmem_ld32(lane_base + L::DQ_COL, r[0]);
+        tmem_ld32(lane_base + L::DQ_COL + 32, r[1]);
+        tmem_wait_ld();
+        tc_fence_before();
         __syncwarp();
+        if (lane == 0) mbar_arrive(dq_free);  // dQ_j is in registers
 #pragma unroll
-        for (int c = 0; c < D / 32; ++c) {
-          uint32_t r[32];
-          tmem_ld32(lane_base + L::DQ_COL + 32 * c, r);
-          tmem_wait_ld();
-          if (c == D / 32 - 1) {
-            tc_fence_before();
-            __syncwarp();
-            if (lane == 0) mbar_arrive(dq_free);
-          }
+        for (int c = 0; c < 2; ++c) {
+          if (lane == 0) bulk_wait_read_all();  // the box buffer was read by the TMA unit
+          __syncwarp();
 #pragma unroll
           for (int i = 0; i < 8; ++i)
-            *reinterpret_cast<uint4*>(stg + c * 4096 + lane * 128 + ((i ^ (lane & 7)) << 4)) =
-                make_uint4(r[4 * i], r[4 * i + 1], r[4 * i + 2], r[4 * i + 3]);
-        }
-        fence_proxy_async_smem();
-        __syncwarp();
-        if (lane == 0) {
-#pragma unroll
-          for (int c = 0; c < D / 32; ++c)
-            tma_reduce_add_3d(&tm_dq, stg + c * 4096, 32 * c, q0 + wq * 32, bh);
-          bulk_commit_group();
+            *reinterpret_cast<uint4*>(stg + lane * 128 + ((i ^ (lane & 7)) << 4)) =
+                make_uint4(r[c][4 * i], r[c][4 * i + 1], r[c][4 * i + 2], r[c][4 * i + 3]);
+          fence_proxy_async_smem();
+          __syncwarp();
+          if (lane == 0) {
+            tma_reduce_add_3d(&tm_dq, stg, 32 * c, q0 + wq * 32, bh);
+            bulk_commit_group();
+          }
         }
       }
     }
