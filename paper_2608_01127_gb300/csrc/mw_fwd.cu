@@ -38,7 +38,7 @@ struct FwdLayout {
   static constexpr int OFF_ONES = OFF_V + STAGES * TILE_BYTES;
   static constexpr int ONES_BYTES = SUM_MMA ? REGION_BYTES : 0;
   static constexpr int OFF_BAR = OFF_ONES + ONES_BYTES;
-  static constexpr int NBAR = 1 + 4 * STAGES + 2 * QT + 1;
+  static constexpr int NBAR = 1 + 4 * STAGES + 3 * QT + 1;
   static constexpr int OFF_MISC = OFF_BAR + NBAR * 8;
   static constexpr int BYTES = OFF_MISC + 16;
   static constexpr uint32_t S_COL(int t) { return 128u * t; }
@@ -105,7 +105,8 @@ __global__ void __launch_bounds__(FwdLayout<D>::THREADS, 1)
   uint64_t* v_empty = v_full + NS;
   uint64_t* s_full = v_empty + NS;
   uint64_t* p_full = s_full + QT;
-  uint64_t* o_full = p_full + QT;
+  uint64_t* p_half = p_full + QT;  // first 64 keys of P in TMEM
+  uint64_t* o_full = p_half + QT;
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + L::OFF_MISC);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + L::OFF_MISC + 4);
 
@@ -147,6 +148,7 @@ __global__ void __launch_bounds__(FwdLayout<D>::THREADS, 1)
     for (int t = 0; t < QT; ++t) {
       mbar_init(&s_full[t], 1);
       mbar_init(&p_full[t], 4);
+      mbar_init(&p_half[t], 4);
     }
     mbar_init(o_full, 1);
     *abort_flag = 0;
@@ -237,12 +239,14 @@ __global__ void __launch_bounds__(FwdLayout<D>::THREADS, 1)
                   kk > 0 ? 1u : 0u);
         }
       };
-      auto issue_pv = [&](int t, int st, bool acc) {
+      // O_t (+)= P_t V for keys [64 half, 64 half + 64) of the tile
+      auto issue_pv = [&](int t, int st, bool acc, int half) {
         // V stage st; for d = 64 the next 64 "columns" are the ones region
         const uint32_t vs = v_addr + st * L::TILE_BYTES;
         const uint64_t vb = sdesc_sw128(vs, L::SUM_MMA ? ones_addr - vs : L::REGION_BYTES, 1024);
 #pragma unroll
-        for (int kk = 0; kk < kTileRows / 16; ++kk) {
+        for (int k4 = 0; k4 < 4; ++k4) {
+          const int kk = 4 * half + k4;
           umma_ts(tmem + L::O_COL(t), tmem + L::S_COL(t) + kk * 8, sdesc_add(vb, kk * 2048),
                   idesc_pv, (acc || kk > 0) ? 1u : 0u);
         }
@@ -259,10 +263,14 @@ __global__ void __launch_bounds__(FwdLayout<D>::THREADS, 1)
         tc_fence_after();
         for (int t = 0; t < QT; ++t) {
           if (i > 0) {
-            if (!(ok = warp_wait(&p_full[t], (i - 1) & 1, ctl))) break;
+            // PV of the first 64 keys while the softmax warps store the rest of P
+            if (!(ok = warp_wait(&p_half[t], (i - 1) & 1, ctl))) break;
             if (t == 0 && !(ok = warp_wait(&v_full[stp], php, ctl))) break;
             tc_fence_after();
-            issue_pv(t, stp, i - 1 > 0);
+            issue_pv(t, stp, i - 1 > 0, 0);
+            if (!(ok = warp_wait(&p_full[t], (i - 1) & 1, ctl))) break;
+            tc_fence_after();
+            issue_pv(t, stp, true, 1);
           }
           issue_qk(t, st);
           umma_commit(&s_full[t]);
@@ -275,10 +283,13 @@ __global__ void __launch_bounds__(FwdLayout<D>::THREADS, 1)
         const int il = n_local - 1;
         const int stl = il % NS;
         for (int t = 0; ok && t < QT; ++t) {
-          if (!(ok = warp_wait(&p_full[t], il & 1, ctl))) break;
+          if (!(ok = warp_wait(&p_half[t], il & 1, ctl))) break;
           if (t == 0 && !(ok = warp_wait(&v_full[stl], (il / NS) & 1, ctl))) break;
           tc_fence_after();
-          issue_pv(t, stl, il > 0);
+          issue_pv(t, stl, il > 0, 0);
+          if (!(ok = warp_wait(&p_full[t], il & 1, ctl))) break;
+          tc_fence_after();
+          issue_pv(t, stl, true, 1);
         }
         if (ok) {
           umma_commit(&v_empty[stl]);
@@ -369,12 +380,14 @@ __global__ void __launch_bounds__(FwdLayout<D>::THREADS, 1)
       const float2 sl2x2 = make_float2(sl2, sl2);
       const float2 negm = make_float2(-m_eff, -m_eff);
       float2 acc = make_float2(0.f, 0.f);
+      // P in four 32-key groups, each stored as soon as it is packed; the first
+      // two groups (keys 0..63) are announced while the third is stored
 #pragma unroll
-      for (int h = 0; h < 2; ++h) {
-        uint32_t packed[32];
+      for (int g4 = 0; g4 < 4; ++g4) {
+        uint32_t packed[16];
 #pragma unroll
-        for (int k = 0; k < 32; ++k) {
-          const float2 x = fma2(make_float2(s[64 * h + 2 * k], s[64 * h + 2 * k + 1]), sl2x2, negm);
+        for (int k = 0; k < 16; ++k) {
+          const float2 x = fma2(make_float2(s[32 * g4 + 2 * k], s[32 * g4 + 2 * k + 1]), sl2x2, negm);
           const uint32_t pk = pack_bf16x2(ex2_approx(x.x), ex2_approx(x.y));
           // the row sum uses the bf16 weights the PV MMA consumes, so O is an
           // exact convex combination of them (d = 64: summed by the MMA)
@@ -382,7 +395,13 @@ __global__ void __launch_bounds__(FwdLayout<D>::THREADS, 1)
             acc = add2(acc, make_float2(__uint_as_float(pk << 16), __uint_as_float(pk & 0xffff0000u)));
           packed[k] = pk;
         }
-        tmem_st32(s_addr + 32 * h, packed);
+        if (g4 == 2) {  // the first half has landed: its PV can start
+          tmem_wait_st();
+          tc_fence_before();
+          __syncwarp();
+          if (lane == 0) mbar_arrive(&p_half[t]);
+        }
+        tmem_st16(s_addr + 16 * g4, packed);
       }
       l += acc.x + acc.y;
       tmem_wait_st();
