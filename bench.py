@@ -23,6 +23,7 @@ from __future__ import annotations
 
 import argparse
 import csv
+import datetime
 import io
 import json
 import math
@@ -132,32 +133,41 @@ def aggregate_rate(units_per_rank: float, world: int, seconds_max: float) -> flo
 
 # ------------------------------------------------------------------ clocks
 
-CLOCK_FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+CLOCK_FIELDS = ("timestamp,index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
                 "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
                 "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
 
 
 class ClockSampler:
-    """nvidia-smi sampling (200 ms) while the timed region runs."""
+    """nvidia-smi sampling every 20 ms; the summary keeps the samples taken
+    between mark_start() and mark_end() (the timed region)."""
 
     def __init__(self, gpu_index: int):
         self.gpu_index = gpu_index
         self.proc = None
+        self.t0 = self.t1 = None
 
     def __enter__(self):
         try:
             self.proc = subprocess.Popen(
                 ["nvidia-smi", "-i", str(self.gpu_index), f"--query-gpu={CLOCK_FIELDS}",
-                 "--format=csv,noheader,nounits", "-lms", "200"],
+                 "--format=csv,noheader,nounits", "-lms", "20"],
                 stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+            time.sleep(0.5)  # nvidia-smi is sampling before the timed region starts
         except OSError:
             self.proc = None
         return self
 
+    def mark_start(self):
+        self.t0 = datetime.datetime.now()
+
+    def mark_end(self):
+        self.t1 = datetime.datetime.now()
+
     def __exit__(self, *exc):
         self.text = ""
         if self.proc is not None:
-            time.sleep(0.25)
+            time.sleep(0.1)
             self.proc.terminate()
             try:
                 self.text, _ = self.proc.communicate(timeout=5)
@@ -167,17 +177,38 @@ class ClockSampler:
         return False
 
     def summary(self):
-        rows = [r for r in csv.reader(io.StringIO(getattr(self, "text", ""))) if len(r) >= 9]
+        rows = []
+        for r in csv.reader(io.StringIO(getattr(self, "text", ""))):
+            if len(r) < 10:
+                continue
+            ts = None
+            for fmt in ("%Y/%m/%d %H:%M:%S.%f", "%Y/%m/%d %H:%M:%S"):
+                try:
+                    ts = datetime.datetime.strptime(r[0].strip(), fmt)
+                    break
+                except ValueError:
+                    pass
+            if ts is None:
+                continue
+            rows.append((ts, r[1:]))
         if not rows:
             return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["unsampled"], "samples": 0}
-        sm = [float(r[1]) for r in rows if r[1].strip().replace(".", "").isdigit()]
-        mx = [float(r[2]) for r in rows if r[2].strip().replace(".", "").isdigit()]
+        inside = [r for ts, r in rows if self.t0 is not None and self.t1 is not None
+                  and self.t0 <= ts <= self.t1]
+        window = "timed region"
+        if not inside:  # region shorter than the sampling period
+            inside = [r for _, r in rows]
+            window = "whole run (no sample fell inside the timed region)"
+        num = lambda v: v.strip().replace(".", "").isdigit()
+        sm = [float(r[1]) for r in inside if num(r[1])]
+        mx = [float(r[2]) for r in inside if num(r[2])]
         names = ("hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap")
-        reasons = sorted({n for r in rows for n, v in zip(names, r[5:9]) if "Active" == v.strip()})
-        power = [float(r[3]) for r in rows if r[3].strip().replace(".", "").isdigit()]
+        reasons = sorted({n for r in inside for n, v in zip(names, r[5:9]) if "Active" == v.strip()})
+        power = [float(r[3]) for r in inside if num(r[3])]
         return {"sm_mhz": statistics.median(sm) if sm else None,
                 "sm_max_mhz": max(mx) if mx else None, "reasons": reasons,
-                "samples": len(rows), "power_w_max": max(power) if power else None}
+                "samples": len(inside), "window": window,
+                "power_w_max": max(power) if power else None}
 
 
 # ------------------------------------------------------------------ CPU baseline (oracle)
@@ -294,6 +325,7 @@ def run_ours(args):
     with ClockSampler(local) as clk:
         barrier(world)
         torch.cuda.synchronize()
+        clk.mark_start()
         for _ in range(args.steps):
             flush_buf.zero_()          # L2 flush between steps, outside the events
             s, f, m = Events(), Events(), Events()
@@ -311,6 +343,7 @@ def run_ours(args):
             main_ev.append(m)
             fwd_ev.append(f)
         torch.cuda.synchronize()
+        clk.mark_end()
         barrier(world)
     step_ms = [e.ms() for e in step_ev]
     total_ms = max_over_ranks(sum(step_ms), world, dev)

@@ -44,7 +44,9 @@ def _digest() -> str:
             h.update(name.encode() + f.read())
     with open(os.path.join(INCLUDE, "mw_bca.h"), "rb") as f:
         h.update(f.read())
-    h.update(" ".join(ARCH + CFLAGS).encode())
+    # flags without the include directory, so that the digest names the same
+    # build on every machine (the checkout path differs)
+    h.update(" ".join(ARCH + [f for f in CFLAGS if not f.startswith("-I")]).encode())
     return h.hexdigest()
 
 
