@@ -334,9 +334,11 @@ __global__ void __launch_bounds__(FwdLayout<D>::THREADS, 1)
         for (int c = 0; c < 128; ++c)
           if (c >= limit) s[c] = -INFINITY;
       }
-      float mq[4] = {s[0], s[1], s[2], s[3]};
+      float mq[4];
 #pragma unroll
-      for (int c = 4; c < 128; c += 8) {
+      for (int k = 0; k < 4; ++k) mq[k] = fmaxf(s[k], s[k + 4]);
+#pragma unroll
+      for (int c = 8; c < 128; c += 8) {
         mq[0] = max3(mq[0], s[c], s[c + 1]);
         mq[1] = max3(mq[1], s[c + 2], s[c + 3]);
         mq[2] = max3(mq[2], s[c + 4], s[c + 5]);
