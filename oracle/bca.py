@@ -229,17 +229,25 @@ def ring_logical(ring: torch.Tensor, cap: int, head: int, length: int) -> torch.
 
 def cache_fwd(q: torch.Tensor, k_new: torch.Tensor, v_new: torch.Tensor,
               k_ring: torch.Tensor, v_ring: torch.Tensor, cap: int, head: int,
-              length: int, T: int, scale: float) -> Tuple[torch.Tensor, torch.Tensor]:
+              length: int, T: int, scale: float, k_sink: torch.Tensor = None,
+              v_sink: torch.Tensor = None) -> Tuple[torch.Tensor, torch.Tensor]:
     """(O, LSE) of W in-flight chunks (Q, K_new, V_new [B,H,W*T,d]).
 
     In-flight chunk j sees every cached token (the committed history, in
     logical order) and in-flight chunks 0..j (Sec. 3.5: a future chunk attends
     only to the committed history and to preceding chunks of the active window,
-    itself included as in Sec. 3.2).
+    itself included as in Sec. 3.2).  The committed history is the sink
+    anchor (``k_sink``/``v_sink`` [B,H,S,d], the initial context that is never
+    evicted and always comes first, Sec. 3.5 "Structured Rolling KV Cache"),
+    if given, followed by the ring's ``length`` tokens.
     """
     q, k_new, v_new = q.to(F64), k_new.to(F64), v_new.to(F64)
     kc = ring_logical(k_ring.to(F64), cap, head, length)
     vc = ring_logical(v_ring.to(F64), cap, head, length)
+    if k_sink is not None:
+        kc = torch.cat([k_sink.to(F64), kc], dim=-2)
+        vc = torch.cat([v_sink.to(F64), vc], dim=-2)
+        length = length + k_sink.shape[-2]
     keys = torch.cat([kc, k_new], dim=-2)
     vals = torch.cat([vc, v_new], dim=-2)
     B, H, M, _ = q.shape

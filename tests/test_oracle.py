@@ -282,6 +282,50 @@ def test_cache_equals_unrolled_training_form(W, T, cap_chunks, head):
     assert torch.allclose(o, ref, atol=1e-12, rtol=0)
 
 
+@pytest.mark.parametrize("S,W,T,cap_chunks,head", [(1, 1, 4, 5, 9), (2, 2, 4, 3, 5), (4, 2, 4, 3, 0),
+                                                   (9, 3, 3, 4, 7)])
+def test_sink_anchor_comes_first_and_is_always_visible(S, W, T, cap_chunks, head):
+    """Sec. 3.5: the committed history is the sink anchor (never evicted, first
+    position) followed by the FIFO ring; every in-flight chunk sees all of it."""
+    cap = cap_chunks * T
+    q, kn, vn, kr, vr = _cache_case(W, T, cap, cap, head)
+    ks, vs = _rand(1, 2, S, 8, seed=91), _rand(1, 2, S, 8, seed=92)
+    o, lse = oracle.cache_fwd(q, kn, vn, kr, vr, cap, head, cap, T, 0.5, ks, vs)
+    idx = torch.tensor([(head + t) % cap for t in range(cap)])
+    keys = torch.cat([ks, kr[:, :, idx], kn], dim=-2)
+    vals = torch.cat([vs, vr[:, :, idx], vn], dim=-2)
+    mask = torch.zeros(W * T, S + cap + W * T, dtype=torch.bool)
+    for j in range(W):
+        mask[j * T:(j + 1) * T, :S + cap + (j + 1) * T] = True
+    ref = F.scaled_dot_product_attention(q, keys, vals, attn_mask=mask, scale=0.5)
+    assert torch.allclose(o, ref, atol=1e-12, rtol=0)
+    # LSE from its definition over the visible keys
+    s_all = 0.5 * q @ keys.transpose(-1, -2)
+    lse_ref = torch.logsumexp(s_all.masked_fill(~mask, float("-inf")), dim=-1)
+    assert torch.allclose(lse, lse_ref, atol=1e-12, rtol=0)
+    # a sink of S tokens is the same as S more tokens at the ring's logical front
+    ring2_k = torch.cat([ks, kr[:, :, idx]], dim=-2)
+    ring2_v = torch.cat([vs, vr[:, :, idx]], dim=-2)
+    o2, lse2 = oracle.cache_fwd(q, kn, vn, ring2_k, ring2_v, S + cap, 0, S + cap, T, 0.5)
+    assert torch.equal(o2, o) and torch.equal(lse2, lse)
+
+
+def test_sink_of_whole_chunks_is_training_form():
+    """With a one-chunk sink the cache path equals the training form over
+    [sink ; ring (logical) ; in-flight] (Sec. 3.2 block-causal mask)."""
+    W, T, cap, head = 2, 4, 12, 5
+    q, kn, vn, kr, vr = _cache_case(W, T, cap, cap, head)
+    ks, vs = _rand(1, 2, T, 8, seed=93), _rand(1, 2, T, 8, seed=94)
+    o, lse = oracle.cache_fwd(q, kn, vn, kr, vr, cap, head, cap, T, 0.5, ks, vs)
+    idx = torch.tensor([(head + t) % cap for t in range(cap)])
+    keys = torch.cat([ks, kr[:, :, idx], kn], dim=-2)
+    vals = torch.cat([vs, vr[:, :, idx], vn], dim=-2)
+    qq = torch.cat([torch.zeros_like(ks), torch.zeros_like(kr), q], dim=-2)
+    o_ref, lse_ref = oracle.fwd(qq, keys, vals, T, 0.5)
+    assert torch.allclose(o, o_ref[:, :, T + cap:], atol=1e-13, rtol=0)
+    assert torch.allclose(lse, lse_ref[:, :, T + cap:], atol=1e-13, rtol=0)
+
+
 def test_ring_rotation_is_invisible():
     W, T, cap = 2, 3, 12
     q, kn, vn, kr, vr = _cache_case(W, T, cap, cap, 4)
