@@ -55,10 +55,10 @@ def train_pairs(cfg) -> int:
 
 
 def cache_pairs(cfg) -> int:
-    """Each of the W*T queries sees `length` cached keys plus its causal share
-    of the in-flight keys."""
+    """Each of the W*T queries sees the sink anchor and `length` cached keys
+    plus its causal share of the in-flight keys."""
     inflight = cfg.T * cfg.T * cfg.W * (cfg.W + 1) // 2
-    return cfg.B * cfg.H * (cfg.W * cfg.T * cfg.length + inflight)
+    return cfg.B * cfg.H * (cfg.W * cfg.T * (cfg.sink + cfg.length) + inflight)
 
 
 def fwd_flops(pairs: int, d: int) -> float:
@@ -79,10 +79,10 @@ def bwd_main_bytes(cfg) -> float:
 
 
 def cache_bytes(cfg) -> float:
-    """Read the cached K/V once, the in-flight Q/K/V, write O and LSE, and the
-    commit (read + write of one chunk's K and V)."""
+    """Read the cached K/V (sink anchor and ring) once, the in-flight Q/K/V,
+    write O and LSE, and the commit (read + write of one chunk's K and V)."""
     e_new = cfg.B * cfg.H * cfg.W * cfg.T * cfg.d
-    e_ring = cfg.B * cfg.H * cfg.length * cfg.d
+    e_ring = cfg.B * cfg.H * (cfg.sink + cfg.length) * cfg.d
     commit = 2.0 * 2 * 2 * cfg.B * cfg.H * cfg.T * cfg.d
     return 2.0 * 2 * e_ring + 2.0 * 3 * e_new + 2.0 * e_new + 4.0 * cfg.B * cfg.H * cfg.W * cfg.T + commit
 
@@ -464,6 +464,7 @@ def run_extras(mw, dev, peaks):
     del q, k, v, do, o, lse, ws, grads
     extra["rolling_cache"] = bench_rolling(mw, dev, peaks)
     extra["pipelined"] = bench_pipelined(mw, dev, peaks, flush)
+    extra["sink_anchor"] = bench_sink(mw, dev, peaks, flush)
     return extra
 
 
@@ -559,6 +560,28 @@ def bench_pipelined(mw, dev, peaks, flush):
                        20, flush=flush)
     med = statistics.median(ts) * 1e3
     res = {"us_median": round(med, 2), "l2": "flushed between runs"}
+    res.update(_cache_roofline(cfg, med, peaks))
+    return res
+
+
+def bench_sink(mw, dev, peaks, flush):
+    """Eight in-flight chunks against the 12-chunk ring behind a one-frame sink
+    anchor (the cache forward with its sink segment and split-KV combine)."""
+    cfg = CACHE_CONFIGS["sink_anchor"]
+    x = gen_cache(cfg)
+    kr, vr = x["k_ring"].to(dev), x["v_ring"].to(dev)
+    ks, vs = x["k_sink"].to(dev), x["v_sink"].to(dev)
+    q, kn, vn = x["q"][0].to(dev), x["k_new"][0].to(dev), x["v_new"][0].to(dev)
+    ws_bytes = mw.mw_bca_cache_workspace_size(cfg.B, cfg.H, cfg.W, cfg.T, cfg.d,
+                                              cfg.sink + cfg.length)
+    ws = torch.empty(max(ws_bytes, 1), dtype=torch.uint8, device=dev)
+    o = torch.empty_like(q)
+    ts = time_repeated(lambda: mw.mw_bca_cache_fwd_sink(q, kn, vn, ks, vs, kr, vr, cfg.head,
+                                                        cfg.length, cfg.T, cfg.scale,
+                                                        need_lse=False, workspace=ws, out=o),
+                       20, flush=flush)
+    med = statistics.median(ts) * 1e3
+    res = {"us_median": round(med, 2), "l2": "flushed between runs", "sink_tokens": cfg.sink}
     res.update(_cache_roofline(cfg, med, peaks))
     return res
 

@@ -135,6 +135,25 @@ mw_status mw_bca_cache_fwd(const void* q, const void* k_new, const void* v_new,
                            float scale, void* stream);
 
 /*
+ * The same forward with a sink anchor ahead of the ring (Sec. 3.5, structured
+ * rolling KV cache: the initial clean context is retained permanently as a
+ * sink anchor that occupies the first position and never takes part in the
+ * FIFO eviction).
+ *   k_sink, v_sink  : [B, H, sink_len, d] bf16 (may be NULL when sink_len is 0)
+ * In-flight chunk j sees the sink_len sink tokens, all cache_len cached
+ * tokens and in-flight chunks 0..j.  0 <= sink_len <= 2^24; every other
+ * argument is as for mw_bca_cache_fwd, which is this call with sink_len 0.
+ * The workspace is mw_bca_cache_workspace_size(B, H, n_q_chunks, T_chunk, d,
+ * sink_len + cache_len) bytes.
+ */
+mw_status mw_bca_cache_fwd_sink(const void* q, const void* k_new, const void* v_new,
+                                const void* k_sink, const void* v_sink, int sink_len,
+                                const void* k_cache, const void* v_cache, int cache_cap,
+                                int cache_head, int cache_len, void* o, float* lse,
+                                void* workspace, size_t ws_bytes, int B, int H, int n_q_chunks,
+                                int T_chunk, int d, float scale, void* stream);
+
+/*
  * Commit of finished tokens into the ring (Sec. 3.5: once a chunk reaches the
  * data endpoint its keys/values go to the cache and are never modified).
  * Copies rows r = 0..rows-1 of k_src / v_src ([B, H, rows, d] bf16) to

@@ -10,6 +10,8 @@ Entry points (same names as the C ABI, taking torch tensors):
   mw_bca_bwd(q, k, v, o, lse, dout, T_chunk, scale=None) -> (dq, dk, dv)
   mw_bca_cache_fwd(q, k_new, v_new, k_cache, v_cache, cache_head, cache_len,
                    T_chunk, scale=None, need_lse=True) -> (o, lse)
+  mw_bca_cache_fwd_sink(q, k_new, v_new, k_sink, v_sink, k_cache, v_cache,
+                        cache_head, cache_len, T_chunk, ...) -> (o, lse)
   mw_bca_cache_commit(k_cache, v_cache, slot_start, k_src, v_src)
   mw_device_status(clear=True), mw_set_option(name, value)
 Tensors are contiguous bf16 [B, H, rows, d] on the current CUDA device.
@@ -25,6 +27,7 @@ import torch
 
 __all__ = [
     "MWError", "library", "lib_path", "mw_bca_fwd", "mw_bca_bwd", "mw_bca_cache_fwd",
+    "mw_bca_cache_fwd_sink",
     "mw_bca_cache_commit", "mw_bca_bwd_workspace_size", "mw_bca_cache_workspace_size",
     "mw_device_status", "mw_set_option", "BlockCausalAttention", "EXPORTED_SYMBOLS",
     "RingState",
@@ -37,7 +40,7 @@ EXPORTED_SYMBOLS = (
     "mw_bca_fwd", "mw_bca_bwd_workspace_size", "mw_bca_bwd", "mw_bca_bwd_stage",
     "mw_bca_cache_workspace_size",
     "mw_bca_cache_fwd", "mw_bca_cache_commit", "mw_status_string", "mw_last_error",
-    "mw_device_status", "mw_set_option", "mw_bca_cache_fwd_noalloc",
+    "mw_device_status", "mw_set_option", "mw_bca_cache_fwd_noalloc", "mw_bca_cache_fwd_sink",
 )
 
 STATUS = {0: "MW_OK", 1: "MW_ERR_INVALID_ARG", 2: "MW_ERR_UNSUPPORTED", 3: "MW_ERR_CUDA",
@@ -80,6 +83,8 @@ def library() -> ctypes.CDLL:
         "mw_bca_cache_workspace_size": (_Z, [_I, _I, _I, _I, _I, _I]),
         "mw_bca_cache_fwd": (_I, [_P, _P, _P, _P, _P, _I, _I, _I, _P, _P, _P, _Z,
                                   _I, _I, _I, _I, _I, _F, _P]),
+        "mw_bca_cache_fwd_sink": (_I, [_P, _P, _P, _P, _P, _I, _P, _P, _I, _I, _I, _P, _P, _P,
+                                       _Z, _I, _I, _I, _I, _I, _F, _P]),
         "mw_bca_cache_commit": (_I, [_P, _P, _I, _I, _P, _P, _I, _I, _I, _I, _P]),
         "mw_bca_cache_fwd_noalloc": (_I, [_P, _P, _P, _P, _P, _I, _I, _I, _P, _P,
                                           _I, _I, _I, _I, _I, _F, _P]),
@@ -183,6 +188,22 @@ def mw_bca_cache_fwd(q, k_new, v_new, k_cache, v_cache, cache_head: int, cache_l
                      T_chunk: int, scale: Optional[float] = None, need_lse: bool = True,
                      workspace: Optional[torch.Tensor] = None, out: Optional[torch.Tensor] = None):
     """In-flight chunks against the rolling KV cache (Sec. 3.5); returns (O, LSE or None)."""
+    return _cache_fwd(q, k_new, v_new, None, None, k_cache, v_cache, cache_head, cache_len,
+                      T_chunk, scale, need_lse, workspace, out)
+
+
+def mw_bca_cache_fwd_sink(q, k_new, v_new, k_sink, v_sink, k_cache, v_cache, cache_head: int,
+                          cache_len: int, T_chunk: int, scale: Optional[float] = None,
+                          need_lse: bool = True, workspace: Optional[torch.Tensor] = None,
+                          out: Optional[torch.Tensor] = None):
+    """As mw_bca_cache_fwd with a sink anchor k_sink / v_sink [B, H, S, d] that
+    every in-flight chunk sees ahead of the ring (Sec. 3.5); returns (O, LSE or None)."""
+    return _cache_fwd(q, k_new, v_new, k_sink, v_sink, k_cache, v_cache, cache_head, cache_len,
+                      T_chunk, scale, need_lse, workspace, out)
+
+
+def _cache_fwd(q, k_new, v_new, k_sink, v_sink, k_cache, v_cache, cache_head, cache_len,
+               T_chunk, scale, need_lse, workspace, out):
     B, H, M, d = _bhnd(q, "q")
     for t, n in ((k_new, "k_new"), (v_new, "v_new")):
         if _bhnd(t, n) != (B, H, M, d):
@@ -194,15 +215,28 @@ def mw_bca_cache_fwd(q, k_new, v_new, k_cache, v_cache, cache_head: int, cache_l
     if M % T_chunk != 0:
         raise ValueError(f"{M} query rows is not a multiple of T_chunk={T_chunk}")
     W = M // T_chunk
-    ws_bytes = mw_bca_cache_workspace_size(B, H, W, T_chunk, d, cache_len)
+    sink_len = 0
+    if k_sink is not None:
+        Bs, Hs, sink_len, ds = _bhnd(k_sink, "k_sink")
+        _bhnd(v_sink, "v_sink")
+        if (Bs, Hs, ds) != (B, H, d) or tuple(v_sink.shape) != tuple(k_sink.shape):
+            raise ValueError("k_sink / v_sink must be [B, H, S, d] matching q")
+    ws_bytes = mw_bca_cache_workspace_size(B, H, W, T_chunk, d, sink_len + cache_len)
     if ws_bytes and (workspace is None or workspace.numel() < ws_bytes):
         workspace = torch.empty(ws_bytes, dtype=torch.uint8, device=q.device)
     o = torch.empty_like(q) if out is None else out
     lse = torch.empty((B, H, M), dtype=torch.float32, device=q.device) if need_lse else None
-    _check(library().mw_bca_cache_fwd(
-        _ptr(q), _ptr(k_new), _ptr(v_new), _ptr(k_cache), _ptr(v_cache), cap, cache_head,
-        cache_len, _ptr(o), _ptr(lse), _ptr(workspace) if ws_bytes else None, ws_bytes,
-        B, H, W, T_chunk, d, _scale(scale, d), _stream()))
+    if k_sink is None:
+        _check(library().mw_bca_cache_fwd(
+            _ptr(q), _ptr(k_new), _ptr(v_new), _ptr(k_cache), _ptr(v_cache), cap, cache_head,
+            cache_len, _ptr(o), _ptr(lse), _ptr(workspace) if ws_bytes else None, ws_bytes,
+            B, H, W, T_chunk, d, _scale(scale, d), _stream()))
+    else:
+        _check(library().mw_bca_cache_fwd_sink(
+            _ptr(q), _ptr(k_new), _ptr(v_new), _ptr(k_sink), _ptr(v_sink), sink_len,
+            _ptr(k_cache), _ptr(v_cache), cap, cache_head, cache_len, _ptr(o), _ptr(lse),
+            _ptr(workspace) if ws_bytes else None, ws_bytes, B, H, W, T_chunk, d,
+            _scale(scale, d), _stream()))
     return o, lse
 
 

@@ -256,14 +256,14 @@ mw_status launch_status(cudaError_t e, const char* what) {
 }
 
 mw_status fwd_common(const void* q, const void* k, const void* v, const void* kr, const void* vr,
-                     int cap, int head, int len, void* o, float* lse, void* ws, size_t ws_bytes,
-                     int BH, int rows_q, int T, int d, float scale, int splits,
-                     cudaStream_t stream) {
+                     int cap, int head, int len, const void* ks, const void* vs, int sink_len,
+                     void* o, float* lse, void* ws, size_t ws_bytes, int BH, int rows_q, int T,
+                     int d, float scale, int splits, cudaStream_t stream) {
   DeviceScope scope(stream);
   MW_TRY(scope.status());
   unsigned* status = nullptr;
   MW_TRY(status_ptr(&status));
-  CUtensorMap tq, tk, tv, tkr, tvr;
+  CUtensorMap tq, tk, tv, tkr, tvr, tks, tvs;
   MW_TRY(make_map(&tq, q, rows_q, BH, d, "q"));
   MW_TRY(make_map(&tk, k, rows_q, BH, d, "k"));
   MW_TRY(make_map(&tv, v, rows_q, BH, d, "v"));
@@ -274,6 +274,13 @@ mw_status fwd_common(const void* q, const void* k, const void* v, const void* kr
     tkr = tk;
     tvr = tv;
   }
+  if (sink_len > 0) {
+    MW_TRY(make_map(&tks, ks, sink_len, BH, d, "k_sink"));
+    MW_TRY(make_map(&tvs, vs, sink_len, BH, d, "v_sink"));
+  } else {
+    tks = tk;
+    tvs = tv;
+  }
   mw::FwdParams p{};
   p.BH = BH;
   p.rows_q = rows_q;
@@ -282,6 +289,7 @@ mw_status fwd_common(const void* q, const void* k, const void* v, const void* kr
   p.ring_cap = len > 0 ? cap : 1;
   p.ring_head = len > 0 ? head : 0;
   p.ring_len = len;
+  p.sink_len = sink_len;
   p.num_splits = splits;
   p.scale_log2 = scale * 1.4426950408889634f;
   p.o = static_cast<__nv_bfloat16*>(o);
@@ -298,7 +306,7 @@ mw_status fwd_common(const void* q, const void* k, const void* v, const void* kr
     p.lse_part = reinterpret_cast<float*>(
         base + align256(static_cast<size_t>(p.num_splits) * BH * rows_q * d * sizeof(float)));
   }
-  MW_TRY(launch_status(mw::launch_fwd(d, tq, tk, tv, tkr, tvr, p, stream), "forward kernel launch"));
+  MW_TRY(launch_status(mw::launch_fwd(d, tq, tk, tv, tkr, tvr, tks, tvs, p, stream), "forward kernel launch"));
   if (p.num_splits > 1)
     MW_TRY(launch_status(mw::launch_combine(d, p.o_part, p.lse_part, p.o, lse, p.num_splits, BH,
                                             rows_q, stream),
@@ -355,7 +363,7 @@ mw_status mw_bca_fwd(const void* q, const void* k, const void* v, void* o, float
   MW_TRY(check_ptr(o, "o"));
   if (lse && (reinterpret_cast<uintptr_t>(lse) & 3u))
     return fail(MW_ERR_INVALID_ARG, "lse is not 4-byte aligned");
-  return fwd_common(q, k, v, nullptr, nullptr, 1, 0, 0, o, lse, nullptr, 0, B * H,
+  return fwd_common(q, k, v, nullptr, nullptr, 1, 0, 0, nullptr, nullptr, 0, o, lse, nullptr, 0, B * H,
                     static_cast<int>(N), T_chunk, d, scale, 1, static_cast<cudaStream_t>(stream));
 }
 
@@ -469,6 +477,17 @@ mw_status mw_bca_cache_fwd(const void* q, const void* k_new, const void* v_new,
                            int cache_head, int cache_len, void* o, float* lse, void* workspace,
                            size_t ws_bytes, int B, int H, int n_q_chunks, int T_chunk, int d,
                            float scale, void* stream) {
+  return mw_bca_cache_fwd_sink(q, k_new, v_new, nullptr, nullptr, 0, k_cache, v_cache, cache_cap,
+                               cache_head, cache_len, o, lse, workspace, ws_bytes, B, H,
+                               n_q_chunks, T_chunk, d, scale, stream);
+}
+
+mw_status mw_bca_cache_fwd_sink(const void* q, const void* k_new, const void* v_new,
+                                const void* k_sink, const void* v_sink, int sink_len,
+                                const void* k_cache, const void* v_cache, int cache_cap,
+                                int cache_head, int cache_len, void* o, float* lse,
+                                void* workspace, size_t ws_bytes, int B, int H, int n_q_chunks,
+                                int T_chunk, int d, float scale, void* stream) {
   MW_TRY(check_dims(B, H, d));
   if (n_q_chunks < 1 || T_chunk < 1)
     return fail(MW_ERR_INVALID_ARG, "n_q_chunks=%d and T_chunk=%d must be >= 1", n_q_chunks, T_chunk);
@@ -480,6 +499,8 @@ mw_status mw_bca_cache_fwd(const void* q, const void* k_new, const void* v_new,
     return fail(MW_ERR_INVALID_ARG, "cache_head=%d not in [0, cache_cap=%d)", cache_head, cache_cap);
   if (cache_len < 0 || cache_len > cache_cap)
     return fail(MW_ERR_INVALID_ARG, "cache_len=%d not in [0, cache_cap=%d]", cache_len, cache_cap);
+  if (sink_len < 0 || sink_len > (1 << 24))
+    return fail(MW_ERR_INVALID_ARG, "sink_len=%d out of range [0, 2^24]", sink_len);
   if (!(scale > 0.f)) return fail(MW_ERR_INVALID_ARG, "scale must be > 0");
   MW_TRY(check_ptr(q, "q"));
   MW_TRY(check_ptr(k_new, "k_new"));
@@ -489,10 +510,15 @@ mw_status mw_bca_cache_fwd(const void* q, const void* k_new, const void* v_new,
     MW_TRY(check_ptr(k_cache, "k_cache"));
     MW_TRY(check_ptr(v_cache, "v_cache"));
   }
+  if (sink_len > 0) {
+    MW_TRY(check_ptr(k_sink, "k_sink"));
+    MW_TRY(check_ptr(v_sink, "v_sink"));
+  }
   if (lse && (reinterpret_cast<uintptr_t>(lse) & 3u))
     return fail(MW_ERR_INVALID_ARG, "lse is not 4-byte aligned");
   const int BH = B * H;
-  const int splits = plan_splits(BH, static_cast<int>(rows), cache_len);
+  // the split plan counts every cached key (sink and ring alike)
+  const int splits = plan_splits(BH, static_cast<int>(rows), sink_len + cache_len);
   const size_t need = cache_ws_bytes(splits, BH, static_cast<int>(rows), d);
   if (need > 0) {
     if (workspace == nullptr || ws_bytes < need)
@@ -500,9 +526,10 @@ mw_status mw_bca_cache_fwd(const void* q, const void* k_new, const void* v_new,
     if (reinterpret_cast<uintptr_t>(workspace) & 255u)
       return fail(MW_ERR_INVALID_ARG, "workspace is not 256-byte aligned");
   }
-  return fwd_common(q, k_new, v_new, k_cache, v_cache, cache_cap, cache_head, cache_len, o, lse,
-                    need > 0 ? workspace : nullptr, ws_bytes, BH, static_cast<int>(rows), T_chunk,
-                    d, scale, splits, static_cast<cudaStream_t>(stream));
+  return fwd_common(q, k_new, v_new, k_cache, v_cache, cache_cap, cache_head, cache_len, k_sink,
+                    v_sink, sink_len, o, lse, need > 0 ? workspace : nullptr, ws_bytes, BH,
+                    static_cast<int>(rows), T_chunk, d, scale, splits,
+                    static_cast<cudaStream_t>(stream));
 }
 
 mw_status mw_bca_cache_commit(void* k_cache, void* v_cache, int cache_cap, int slot_start,

@@ -54,30 +54,41 @@ struct FwdLayout {
                 "register re-split must hand out exactly the launch's registers");
 };
 
-// Where key tile j of a query block comes from.
+// Where key tile j of a query block comes from.  Keys are visited in logical
+// order: the sink anchor (segment S), the ring from its head to the end of
+// the buffer (A) and from the start after wrapping (B), then the queries' own
+// chunks (C).
+enum : int { kSegOwn = 0, kSegRing = 1, kSegSink = 2 };
 struct TileSrc {
-  bool ring;   // ring buffer (segments A, B) or the queries' own keys (C)
+  int seg;     // kSegOwn, kSegRing or kSegSink: which tensor maps hold the tile
   int row0;    // first physical row of the tile
-  int end;     // ring: exclusive end of the valid rows; C: unused
+  int end;     // ring and sink: exclusive end of the valid rows; own: unused
 };
 
 struct Segs {
-  int nA, nB, nC;
-  int headA, endA, endB;
+  int nS, nA, nB, nC;
+  int endS, headA, endA, endB;
 };
 
 __device__ __forceinline__ TileSrc tile_src(const Segs& g, int j) {
   TileSrc s;
+  if (j < g.nS) {
+    s.seg = kSegSink;
+    s.row0 = j * kTileRows;
+    s.end = g.endS;
+    return s;
+  }
+  j -= g.nS;
   if (j < g.nA) {
-    s.ring = true;
+    s.seg = kSegRing;
     s.row0 = g.headA + j * kTileRows;
     s.end = g.endA;
   } else if (j < g.nA + g.nB) {
-    s.ring = true;
+    s.seg = kSegRing;
     s.row0 = (j - g.nA) * kTileRows;
     s.end = g.endB;
   } else {
-    s.ring = false;
+    s.seg = kSegOwn;
     s.row0 = (j - g.nA - g.nB) * kTileRows;
     s.end = 0;
   }
@@ -88,7 +99,8 @@ template <int D>
 __global__ void __launch_bounds__(FwdLayout<D>::THREADS, 1)
     bca_fwd_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_k,
                    const __grid_constant__ CUtensorMap tm_v, const __grid_constant__ CUtensorMap tm_kr,
-                   const __grid_constant__ CUtensorMap tm_vr, const FwdParams p) {
+                   const __grid_constant__ CUtensorMap tm_vr, const __grid_constant__ CUtensorMap tm_ks,
+                   const __grid_constant__ CUtensorMap tm_vs, const FwdParams p) {
   using L = FwdLayout<D>;
   constexpr int QT = L::QT;
   constexpr int NS = L::STAGES;
@@ -124,6 +136,8 @@ __global__ void __launch_bounds__(FwdLayout<D>::THREADS, 1)
   const int c_end = (last_row / p.T + 1) * p.T;  // keys of segment C visible to the block
 
   Segs g;
+  g.nS = (p.sink_len + kTileRows - 1) / kTileRows;
+  g.endS = p.sink_len;
   const int lenA = min(p.ring_len, p.ring_cap - p.ring_head);
   const int lenB = p.ring_len - lenA;
   g.nA = (lenA + kTileRows - 1) / kTileRows;
@@ -132,7 +146,7 @@ __global__ void __launch_bounds__(FwdLayout<D>::THREADS, 1)
   g.headA = p.ring_head;
   g.endA = p.ring_head + lenA;
   g.endB = lenB;
-  const int n_all = g.nA + g.nB + g.nC;
+  const int n_all = g.nS + g.nA + g.nB + g.nC;
   const int j0 = (int)((long long)split * n_all / p.num_splits);
   const int j1 = (int)((long long)(split + 1) * n_all / p.num_splits);
   const int n_local = j1 - j0;
@@ -199,13 +213,15 @@ __global__ void __launch_bounds__(FwdLayout<D>::THREADS, 1)
         if (!mbar_wait(&k_empty[st], ph ^ 1, ctl)) break;
         mbar_arrive_expect_tx(&k_full[st], L::TILE_BYTES);
         for (int r = 0; r < L::REG; ++r)
-          tma_load_3d(sK + st * L::TILE_BYTES + r * L::REGION_BYTES, src.ring ? &tm_kr : &tm_k,
+          tma_load_3d(sK + st * L::TILE_BYTES + r * L::REGION_BYTES,
+                      src.seg == kSegRing ? &tm_kr : src.seg == kSegSink ? &tm_ks : &tm_k,
                       &k_full[st], 64 * r, src.row0, bh);
         ++issued_k;
         if (!mbar_wait(&v_empty[st], ph ^ 1, ctl)) break;
         mbar_arrive_expect_tx(&v_full[st], L::TILE_BYTES);
         for (int r = 0; r < L::REG; ++r)
-          tma_load_3d(sV + st * L::TILE_BYTES + r * L::REGION_BYTES, src.ring ? &tm_vr : &tm_v,
+          tma_load_3d(sV + st * L::TILE_BYTES + r * L::REGION_BYTES,
+                      src.seg == kSegRing ? &tm_vr : src.seg == kSegSink ? &tm_vs : &tm_v,
                       &v_full[st], 64 * r, src.row0, bh);
         ++issued_v;
       }
@@ -328,7 +344,7 @@ __global__ void __launch_bounds__(FwdLayout<D>::THREADS, 1)
 #pragma unroll
         for (int k = 0; k < 32; ++k) s[32 * c + k] = __uint_as_float(r[k]);
       }
-      const int limit = (src.ring ? src.end : c_limit) - src.row0;
+      const int limit = (src.seg != kSegOwn ? src.end : c_limit) - src.row0;
       if (limit < kTileRows) {
 #pragma unroll
         for (int c = 0; c < 128; ++c)
@@ -509,8 +525,8 @@ __global__ void __launch_bounds__(256) combine_kernel(const float* __restrict__ 
 
 template <int D>
 cudaError_t launch_fwd_t(const CUtensorMap& tq, const CUtensorMap& tk, const CUtensorMap& tv,
-                         const CUtensorMap& tkr, const CUtensorMap& tvr, const FwdParams& p,
-                         cudaStream_t s) {
+                         const CUtensorMap& tkr, const CUtensorMap& tvr, const CUtensorMap& tks,
+                         const CUtensorMap& tvs, const FwdParams& p, cudaStream_t s) {
   using L = FwdLayout<D>;
   static bool attr_set = false;  // per process; the attribute is per function
   if (!attr_set) {
@@ -526,17 +542,17 @@ cudaError_t launch_fwd_t(const CUtensorMap& tq, const CUtensorMap& tk, const CUt
     attr_set = true;
   }
   const unsigned grid = static_cast<unsigned>(p.BH) * p.n_qblocks * p.num_splits;
-  bca_fwd_kernel<D><<<grid, L::THREADS, L::BYTES, s>>>(tq, tk, tv, tkr, tvr, p);
+  bca_fwd_kernel<D><<<grid, L::THREADS, L::BYTES, s>>>(tq, tk, tv, tkr, tvr, tks, tvs, p);
   return cudaGetLastError();
 }
 
 }  // namespace
 
 cudaError_t launch_fwd(int d, const CUtensorMap& tq, const CUtensorMap& tk, const CUtensorMap& tv,
-                       const CUtensorMap& tkr, const CUtensorMap& tvr, const FwdParams& p,
-                       cudaStream_t s) {
-  if (d == 64) return launch_fwd_t<64>(tq, tk, tv, tkr, tvr, p, s);
-  return launch_fwd_t<128>(tq, tk, tv, tkr, tvr, p, s);
+                       const CUtensorMap& tkr, const CUtensorMap& tvr, const CUtensorMap& tks,
+                       const CUtensorMap& tvs, const FwdParams& p, cudaStream_t s) {
+  if (d == 64) return launch_fwd_t<64>(tq, tk, tv, tkr, tvr, tks, tvs, p, s);
+  return launch_fwd_t<128>(tq, tk, tv, tkr, tvr, tks, tvs, p, s);
 }
 
 cudaError_t launch_combine(int d, const float* o_part, const float* lse_part, __nv_bfloat16* o,

@@ -31,6 +31,7 @@ struct FwdParams {
   int ring_cap;
   int ring_head;
   int ring_len;
+  int sink_len;     // tokens of the sink anchor, visited before the ring
   int num_splits;   // 1: write bf16 O + LSE; >1: fp32 partials for the combine
   float scale_log2; // softmax scale * log2(e)
   __nv_bfloat16* o;
@@ -59,9 +60,11 @@ struct BwdParams {
 };
 
 // Launchers (return cudaGetLastError() of the launch).
+// tkr/tvr: ring buffer maps; tks/tvs: sink anchor maps (any valid map when
+// the segment is empty)
 cudaError_t launch_fwd(int d, const CUtensorMap& tq, const CUtensorMap& tk, const CUtensorMap& tv,
-                       const CUtensorMap& tkr, const CUtensorMap& tvr, const FwdParams& p,
-                       cudaStream_t s);
+                       const CUtensorMap& tkr, const CUtensorMap& tvr, const CUtensorMap& tks,
+                       const CUtensorMap& tvs, const FwdParams& p, cudaStream_t s);
 cudaError_t launch_combine(int d, const float* o_part, const float* lse_part, __nv_bfloat16* o,
                            float* lse, int splits, int BH, int rows, cudaStream_t s);
 cudaError_t launch_bwd_pre(int d, const __nv_bfloat16* o, const __nv_bfloat16* dout,

@@ -111,6 +111,21 @@ def test_cache_rejects_bad_ring_state(mw):
     assert call(T=0) == INVALID
 
 
+def test_sink_entry_rejects_bad_sink(mw):
+    lib = mw.library()
+
+    def call(sink_len=440, ks=FAKE, vs=FAKE, head=0):
+        return lib.mw_bca_cache_fwd_sink(FAKE, FAKE, FAKE, ks, vs, sink_len, FAKE, FAKE, 1024,
+                                         head, 1024, FAKE, None, None, 0, 1, 2, 1, 64, 128, 0.1,
+                                         None)
+
+    assert call(sink_len=-1) == INVALID
+    assert call(sink_len=(1 << 24) + 1) == INVALID
+    assert call(ks=None) == INVALID
+    assert call(vs=None) == INVALID
+    assert call(head=1024) == INVALID  # the ring checks still apply
+
+
 def test_commit_rejects_bad_slots(mw):
     lib = mw.library()
 

@@ -283,6 +283,61 @@ def test_pipelined_config(mw):
     check_lse(lse, lse_ref, "pipelined")
 
 
+SINK_SMALL = [
+    # B, H, W, T, cap, length, head, sink, d, splits (0 = automatic)
+    (1, 2, 1, 64, 512, 512, 100, 32, 128, 0),     # half-chunk sink, wrapped ring
+    (1, 2, 3, 100, 1000, 300, 900, 1, 64, 0),     # one sink token, partial ring
+    (2, 1, 2, 64, 640, 0, 0, 200, 128, 0),        # sink only (empty ring), ragged tile
+    (1, 2, 2, 96, 960, 960, 480, 128, 64, 4),     # sink of exactly one tile, forced splits
+    (1, 1, 1, 880, 1760, 1760, 1759, 440, 128, 1),  # one latent frame, single pass
+]
+
+
+@pytest.mark.parametrize("B,H,W,T,cap,length,head,sink,d,splits", SINK_SMALL)
+def test_cache_forward_with_sink(mw, B, H, W, T, cap, length, head, sink, d, splits):
+    q, kn, vn, kr, vr = _ring_case(B, H, W, T, cap, d, seed=cap + head + sink)
+    g = torch.Generator().manual_seed(sink + 7)
+    ks, vs = (torch.randn(B, H, sink, d, generator=g).to(torch.bfloat16) for _ in range(2))
+    sc = 1.0 / math.sqrt(d)
+    mw.mw_set_option("cache_splits", splits)
+    try:
+        o, lse = mw.mw_bca_cache_fwd_sink(q.cuda(), kn.cuda(), vn.cuda(), ks.cuda(), vs.cuda(),
+                                          kr.cuda(), vr.cuda(), head, length, T, sc)
+    finally:
+        mw.mw_set_option("cache_splits", 0)
+    o_ref, lse_ref = oracle.cache_fwd(q, kn, vn, kr, vr, cap, head, length, T, sc, ks, vs)
+    tag = f"sink{sink} W{W} T{T} cap{cap} len{length} head{head} splits{splits}"
+    check_o(o, o_ref, tag)
+    check_lse(lse, lse_ref, tag)
+
+
+def test_empty_sink_is_the_plain_cache_path(mw):
+    """sink_len = 0 is exactly mw_bca_cache_fwd (same kernels, same bits)."""
+    q, kn, vn, kr, vr = (t.cuda() for t in _ring_case(1, 2, 2, 128, 1024, 128, seed=31))
+    o0, l0 = mw.mw_bca_cache_fwd(q, kn, vn, kr, vr, 300, 1024, 128)
+    empty = torch.empty(1, 2, 0, 128, dtype=torch.bfloat16, device="cuda")
+    o1, l1 = mw.mw_bca_cache_fwd_sink(q, kn, vn, empty, empty, kr, vr, 300, 1024, 128)
+    assert torch.equal(o0, o1) and torch.equal(l0, l1)
+
+
+def test_sink_anchor_config(mw):
+    """Eight in-flight chunks against a wrapped 12-chunk ring behind a one-frame
+    (440-token) sink anchor; the oracle checks two of the 16 heads."""
+    cfg = CACHE_CONFIGS["sink_anchor"]
+    x = gen_cache(cfg)
+    q, kn, vn = x["q"][0], x["k_new"][0], x["v_new"][0]
+    o, lse = mw.mw_bca_cache_fwd_sink(q.cuda(), kn.cuda(), vn.cuda(), x["k_sink"].cuda(),
+                                      x["v_sink"].cuda(), x["k_ring"].cuda(), x["v_ring"].cuda(),
+                                      cfg.head, cfg.length, cfg.T, cfg.scale)
+    heads = [0, 11]
+    sel = lambda t: t[:, heads]
+    o_ref, lse_ref = oracle.cache_fwd(sel(q), sel(kn), sel(vn), sel(x["k_ring"]), sel(x["v_ring"]),
+                                      cfg.cap, cfg.head, cfg.length, cfg.T, cfg.scale,
+                                      sel(x["k_sink"]), sel(x["v_sink"]))
+    check_o(o[:, heads], o_ref, "sink_anchor")
+    check_lse(lse[:, heads], lse_ref, "sink_anchor")
+
+
 def test_device_status_is_clean(mw):
     torch.cuda.synchronize()
     assert mw.mw_device_status() == 0

@@ -74,6 +74,7 @@ class CacheConfig:
     seed: int
     std_lo: float = 1.0    # per-chunk std on K and V, U[std_lo, std_hi]
     std_hi: float = 1.0
+    sink: int = 0          # tokens of the sink anchor ahead of the ring (Sec. 3.5)
 
     @property
     def scale(self) -> float:
@@ -102,6 +103,11 @@ CACHE_CONFIGS: Dict[str, CacheConfig] = {
     "pipelined": CacheConfig("pipelined", B=1, H=16, d=128, W=4, T=880,
                              cap=12 * 880, length=12 * 880, head=7 * 880,
                              steps=1, seed=4, std_lo=0.5, std_hi=1.5),
+    # 8 in-flight chunks, a 12-chunk ring and a resident sink of one latent
+    # frame (half a 2-frame chunk), the shape of the paper's cache ablation
+    "sink_anchor": CacheConfig("sink_anchor", B=1, H=16, d=128, W=8, T=880,
+                               cap=12 * 880, length=12 * 880, head=3 * 880,
+                               steps=1, seed=5, sink=440),
 }
 
 
@@ -147,6 +153,8 @@ def gen_cache(cfg: CacheConfig, device: str = "cpu",
     followed by the ``W`` in-flight chunks, shared by K and V, B and H.
     Only the first ``steps`` (default ``cfg.steps``) steps are materialised; the
     draws of earlier steps never depend on how many are kept after them.
+    The sink anchor (``cfg.sink`` > 0) comes from its own generator, seeded
+    ``cfg.seed + 10000``: K then V ``[B,H,sink,d]``.
     """
     n_steps = cfg.steps if steps is None else steps
     g = torch.Generator("cpu").manual_seed(cfg.seed)
@@ -179,10 +187,16 @@ def gen_cache(cfg: CacheConfig, device: str = "cpu",
         new_std = new_std.view(1, 1, cfg.W * cfg.T, 1)
         ks = [k * new_std for k in ks]
         vs = [v * new_std for v in vs]
-    out = {
+    out = {}
+    if cfg.sink > 0:
+        gs = torch.Generator("cpu").manual_seed(cfg.seed + 10000)
+        sshape = (cfg.B, cfg.H, cfg.sink, cfg.d)
+        out["k_sink"] = _bf16(torch.randn(sshape, generator=gs, dtype=torch.float32))
+        out["v_sink"] = _bf16(torch.randn(sshape, generator=gs, dtype=torch.float32))
+    out.update({
         "k_ring": _bf16(k_ring), "v_ring": _bf16(v_ring),
         "q": torch.stack([_bf16(x) for x in qs]),
         "k_new": torch.stack([_bf16(x) for x in ks]),
         "v_new": torch.stack([_bf16(x) for x in vs]),
-    }
+    })
     return {n: t.to(device) for n, t in out.items()}
