@@ -444,24 +444,28 @@ def run_extras(mw, dev, peaks):
     flush_buf = torch.empty(L2_FLUSH_BYTES, dtype=torch.uint8, device=dev)
     flush = flush_buf.zero_
     extra = {}
-    # forward / backward of the d=128 peaky workload
-    cfg = TRAIN_CONFIGS["train_h16_d128_peaky"]
-    x = gen_train(cfg)
-    q, k, v, do = (x[n].to(dev) for n in ("q", "k", "v", "do"))
-    o, lse = mw.mw_bca_fwd(q, k, v, cfg.T, cfg.scale)
-    ws = torch.empty(mw.mw_bca_bwd_workspace_size(cfg.B, cfg.H, cfg.n_chunks, cfg.T, cfg.d),
-                     dtype=torch.uint8, device=dev)
-    grads = tuple(torch.empty_like(q) for _ in range(3))
-    pairs = train_pairs(cfg)
-    tf = time_repeated(lambda: mw.mw_bca_fwd(q, k, v, cfg.T, cfg.scale), 10, flush=flush)
-    tb = time_repeated(lambda: mw.mw_bca_bwd(q, k, v, o, lse, do, cfg.T, cfg.scale, workspace=ws,
-                                             out=grads), 10, flush=flush)
-    fm, bm = statistics.median(tf), statistics.median(tb)
-    extra["train_h16_d128_peaky"] = {
-        "fwd_ms": round(fm, 4), "bwd_ms": round(bm, 4),
-        "fwd_tflops": round(fwd_flops(pairs, cfg.d) / fm / 1e9, 2),
-        "fwd_bwd_tflops": round((fwd_flops(pairs, cfg.d) + bwd_flops(pairs, cfg.d)) / (fm + bm) / 1e9, 2)}
-    del q, k, v, do, o, lse, ws, grads
+    # forward / backward of the other training workloads: d=128 with peaky
+    # logits, and the paper's 32-chunk window of 600-token chunks at the
+    # MiniWorld-1B head layout (12 heads of 128)
+    for name in ("train_h16_d128_peaky", "train_1b_32x600"):
+        cfg = TRAIN_CONFIGS[name]
+        x = gen_train(cfg)
+        q, k, v, do = (x[n].to(dev) for n in ("q", "k", "v", "do"))
+        o, lse = mw.mw_bca_fwd(q, k, v, cfg.T, cfg.scale)
+        ws = torch.empty(mw.mw_bca_bwd_workspace_size(cfg.B, cfg.H, cfg.n_chunks, cfg.T, cfg.d),
+                         dtype=torch.uint8, device=dev)
+        grads = tuple(torch.empty_like(q) for _ in range(3))
+        pairs = train_pairs(cfg)
+        tf = time_repeated(lambda: mw.mw_bca_fwd(q, k, v, cfg.T, cfg.scale), 10, flush=flush)
+        tb = time_repeated(lambda: mw.mw_bca_bwd(q, k, v, o, lse, do, cfg.T, cfg.scale,
+                                                 workspace=ws, out=grads), 10, flush=flush)
+        fm, bm = statistics.median(tf), statistics.median(tb)
+        extra[name] = {
+            "fwd_ms": round(fm, 4), "bwd_ms": round(bm, 4),
+            "fwd_tflops": round(fwd_flops(pairs, cfg.d) / fm / 1e9, 2),
+            "fwd_bwd_tflops": round((fwd_flops(pairs, cfg.d) + bwd_flops(pairs, cfg.d))
+                                    / (fm + bm) / 1e9, 2)}
+        del q, k, v, do, o, lse, ws, grads
     extra["rolling_cache"] = bench_rolling(mw, dev, peaks)
     extra["pipelined"] = bench_pipelined(mw, dev, peaks, flush)
     extra["sink_anchor"] = bench_sink(mw, dev, peaks, flush)

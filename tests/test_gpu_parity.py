@@ -84,6 +84,7 @@ SMALL = [
     (1, 1, 2, 880, 128, 4.0),    # one latent frame per chunk, peaky logits
     (1, 3, 5, 200, 64, 1.0),
     (2, 2, 1, 600, 128, 1.0),    # a single chunk: full bidirectional attention
+    (1, 20, 3, 96, 128, 1.0),    # the 3B head layout (20 heads of 128)
 ]
 
 
@@ -104,7 +105,7 @@ def test_small_shapes_forward_backward(mw, B, H, n, T, d, gain):
     check_grad(dv, dv_r, tag + " dV")
 
 
-@pytest.mark.parametrize("name", ["train_b12_d64", "train_h16_d128_peaky"])
+@pytest.mark.parametrize("name", ["train_b12_d64", "train_h16_d128_peaky", "train_1b_32x600"])
 def test_full_size_training_configs(mw, name):
     """Full-size launch; the oracle recomputes two sampled (b, h) heads in full."""
     cfg = TRAIN_CONFIGS[name]

@@ -92,6 +92,10 @@ TRAIN_CONFIGS: Dict[str, TrainConfig] = {
     "train_h16_d128_peaky": TrainConfig("train_h16_d128_peaky", B=1, H=16, d=128,
                                         n_chunks=21, T=880, seed=2,
                                         gain_lo=1.0, gain_hi=4.0),
+    # the paper's 32-chunk training window with 600-token chunks (15 x 20
+    # latent positions x 2 frames) at the MiniWorld-1B head layout (1536 / 12)
+    "train_1b_32x600": TrainConfig("train_1b_32x600", B=1, H=12, d=128, n_chunks=32,
+                                   T=600, seed=6),
 }
 
 CACHE_CONFIGS: Dict[str, CacheConfig] = {
