@@ -227,10 +227,30 @@ def ring_logical(ring: torch.Tensor, cap: int, head: int, length: int) -> torch.
     return ring.index_select(-2, idx)
 
 
+def rope_rotate(x: torch.Tensor, frames: torch.Tensor, rope_dims: int,
+                base: float) -> torch.Tensor:
+    """Temporal rotary embedding of the rows of ``x`` [..., N, d] (fp64 copy).
+
+    Row n sits at temporal position ``frames[n]``; channel pair (2i, 2i+1)
+    for i < rope_dims / 2 turns by the angle frames[n] * base^(-2i/rope_dims);
+    the other channels are unchanged.  (The paper implies RoPE on the latent
+    tokens and re-shifts the temporal positions of cached keys, Sec. 3.5, but
+    states neither the channel layout nor the frequencies: both are inputs.)
+    """
+    x = x.to(F64).clone()
+    for i in range(rope_dims // 2):
+        theta = frames.to(F64) * (float(base) ** (-2.0 * i / rope_dims))
+        c, s = torch.cos(theta), torch.sin(theta)
+        a, b = x[..., 2 * i].clone(), x[..., 2 * i + 1].clone()
+        x[..., 2 * i] = a * c - b * s
+        x[..., 2 * i + 1] = a * s + b * c
+    return x
+
+
 def cache_fwd(q: torch.Tensor, k_new: torch.Tensor, v_new: torch.Tensor,
               k_ring: torch.Tensor, v_ring: torch.Tensor, cap: int, head: int,
               length: int, T: int, scale: float, k_sink: torch.Tensor = None,
-              v_sink: torch.Tensor = None) -> Tuple[torch.Tensor, torch.Tensor]:
+              v_sink: torch.Tensor = None, rope=None) -> Tuple[torch.Tensor, torch.Tensor]:
     """(O, LSE) of W in-flight chunks (Q, K_new, V_new [B,H,W*T,d]).
 
     In-flight chunk j sees every cached token (the committed history, in
@@ -240,10 +260,22 @@ def cache_fwd(q: torch.Tensor, k_new: torch.Tensor, v_new: torch.Tensor,
     anchor (``k_sink``/``v_sink`` [B,H,S,d], the initial context that is never
     evicted and always comes first, Sec. 3.5 "Structured Rolling KV Cache"),
     if given, followed by the ring's ``length`` tokens.
+
+    RoPE re-shifting (Sec. 3.5: after evictions the retained keys are
+    re-indexed from the start of the window; the sink keeps the first
+    position and is not re-shifted): with ``rope = (rope_dims, base,
+    tokens_per_frame, first_frame)`` the ring holds keys without their
+    temporal rotation, and ring token t (logical order) is rotated to frame
+    first_frame + t // tokens_per_frame before it is used.  Sink and
+    in-flight keys are used as given.
     """
     q, k_new, v_new = q.to(F64), k_new.to(F64), v_new.to(F64)
     kc = ring_logical(k_ring.to(F64), cap, head, length)
     vc = ring_logical(v_ring.to(F64), cap, head, length)
+    if rope is not None and rope[0] > 0:
+        rope_dims, base, per_frame, first_frame = rope
+        frames = first_frame + torch.arange(length) // per_frame
+        kc = rope_rotate(kc, frames, rope_dims, base)
     if k_sink is not None:
         kc = torch.cat([k_sink.to(F64), kc], dim=-2)
         vc = torch.cat([v_sink.to(F64), vc], dim=-2)

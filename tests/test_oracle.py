@@ -326,6 +326,76 @@ def test_sink_of_whole_chunks_is_training_form():
     assert torch.allclose(lse, lse_ref[:, :, T + cap:], atol=1e-13, rtol=0)
 
 
+def test_rope_rotate_hand_values():
+    """d = 4 with both pairs rotated, base 100: pair 0 turns by the frame index,
+    pair 1 by frame / 10."""
+    x = torch.tensor([[1.0, 0.0, 0.0, 1.0]], dtype=F64)
+    y = oracle.rope_rotate(x, torch.tensor([2]), 4, 100.0)
+    want = torch.tensor([[math.cos(2.0), math.sin(2.0), -math.sin(0.2), math.cos(0.2)]], dtype=F64)
+    assert torch.allclose(y, want, atol=1e-15, rtol=0)
+    # frame 0 and rope_dims 0 leave the rows unchanged; the last channels never move
+    assert torch.equal(oracle.rope_rotate(x, torch.tensor([0]), 4, 100.0), x)
+    assert torch.equal(oracle.rope_rotate(x, torch.tensor([5]), 0, 100.0), x)
+    z = oracle.rope_rotate(torch.ones(1, 6, dtype=F64), torch.tensor([3]), 2, 10.0)
+    assert torch.equal(z[:, 2:], torch.ones(1, 4, dtype=F64))
+
+
+def test_rope_rotate_is_a_complex_phase():
+    """Channel pairs as complex numbers: rotation multiplies pair i by
+    exp(1j * frame * base^(-2i/rope_dims)) and keeps every pair's norm."""
+    x = _rand(1, 2, 9, 12, seed=95).to(F64)
+    frames = torch.tensor([0, 1, 1, 2, 3, 5, 8, 13, 21])
+    y = oracle.rope_rotate(x, frames, 8, 500.0)
+    zx = torch.view_as_complex(x[..., :8].reshape(1, 2, 9, 4, 2).contiguous())
+    freq = 500.0 ** (-2.0 * torch.arange(4, dtype=F64) / 8)
+    phase = torch.polar(torch.ones(9, 4, dtype=F64), frames.to(F64)[:, None] * freq[None, :])
+    zy = torch.view_as_real(zx * phase).reshape(1, 2, 9, 8)
+    assert torch.allclose(y[..., :8], zy, atol=1e-13, rtol=0)
+    assert torch.equal(y[..., 8:], x[..., 8:])
+
+
+def test_rope_reshift_keeps_relative_positions():
+    """Scores of rotated queries and keys depend on frame differences only:
+    moving every position (sink, ring, in-flight chunks) by the same offset
+    changes nothing (the re-indexing of Sec. 3.5 is lossless)."""
+    W, T, cap, head, P = 2, 4, 12, 5, 2
+    q, kn, vn, kr, vr = _cache_case(W, T, cap, cap, head)
+    ks, vs = _rand(1, 2, 2, 8, seed=96), _rand(1, 2, 2, 8, seed=97)
+
+    def run(first):
+        new_frames = first + cap // P + torch.arange(W * T) // P
+        qr = oracle.rope_rotate(q, new_frames, 6, 50.0)
+        knr = oracle.rope_rotate(kn, new_frames, 6, 50.0)
+        ksr = oracle.rope_rotate(ks, torch.full((2,), first - 1), 6, 50.0)  # one frame ahead
+        return oracle.cache_fwd(qr, knr, vn, kr, vr, cap, head, cap, T, 0.5, ksr, vs,
+                                rope=(6, 50.0, P, first))
+
+    o1, l1 = run(1)
+    o2, l2 = run(7)
+    assert torch.allclose(o1, o2, atol=1e-12, rtol=0) and torch.allclose(l1, l2, atol=1e-12, rtol=0)
+    # and the rotation really is applied: other offsets between ring and queries differ
+    new_frames = 1 + cap // P + torch.arange(W * T) // P
+    qr = oracle.rope_rotate(q, new_frames, 6, 50.0)
+    knr = oracle.rope_rotate(kn, new_frames, 6, 50.0)
+    o3, _ = oracle.cache_fwd(qr, knr, vn, kr, vr, cap, head, cap, T, 0.5,
+                             oracle.rope_rotate(ks, torch.zeros(2, dtype=torch.long), 6, 50.0),
+                             vs, rope=(6, 50.0, P, 4))
+    assert (o3 - o1).abs().max() > 1e-3
+
+
+def test_rope_ring_equals_prerotated_ring():
+    """Rotating the ring on read equals handing over the logically ordered,
+    already rotated keys with no RoPE (the ring rewrite the fused read avoids)."""
+    W, T, cap, head, P = 1, 4, 8, 3, 4
+    q, kn, vn, kr, vr = _cache_case(W, T, cap, cap, head)
+    o, lse = oracle.cache_fwd(q, kn, vn, kr, vr, cap, head, cap, T, 0.5, rope=(8, 1e4, P, 2))
+    logical = oracle.ring_logical(kr.to(F64), cap, head, cap)
+    rotated = oracle.rope_rotate(logical, 2 + torch.arange(cap) // P, 8, 1e4)
+    o2, lse2 = oracle.cache_fwd(q, kn, vn, rotated, oracle.ring_logical(vr.to(F64), cap, head, cap),
+                                cap, 0, cap, T, 0.5)
+    assert torch.equal(o, o2) and torch.equal(lse, lse2)
+
+
 def test_ring_rotation_is_invisible():
     W, T, cap = 2, 3, 12
     q, kn, vn, kr, vr = _cache_case(W, T, cap, cap, 4)
