@@ -587,6 +587,17 @@ def bench_sink(mw, dev, peaks, flush):
     med = statistics.median(ts) * 1e3
     res = {"us_median": round(med, 2), "l2": "flushed between runs", "sink_tokens": cfg.sink}
     res.update(_cache_roofline(cfg, med, peaks))
+    # the same call with the ring's RoPE re-shift fused into its read: the
+    # first 32 channels carry the temporal rotation, 440 tokens per frame, the
+    # ring starting at frame 1 behind the one-frame sink
+    ts = time_repeated(lambda: mw.mw_bca_cache_fwd_rope(q, kn, vn, ks, vs, kr, vr, cfg.head,
+                                                        cfg.length, cfg.T, 32, 10000.0, 440, 1,
+                                                        cfg.scale, need_lse=False, workspace=ws,
+                                                        out=o),
+                       20, flush=flush)
+    med_r = statistics.median(ts) * 1e3
+    res["rope_reshift"] = {"us_median": round(med_r, 2), "rope_dims": 32,
+                           "tokens_per_frame": 440, **_cache_roofline(cfg, med_r, peaks)}
     return res
 
 

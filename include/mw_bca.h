@@ -154,6 +154,37 @@ mw_status mw_bca_cache_fwd_sink(const void* q, const void* k_new, const void* v_
                                 int T_chunk, int d, float scale, void* stream);
 
 /*
+ * The same forward with RoPE re-shifting of the ring fused into its read
+ * (Sec. 3.5, RoPE re-shifting: after each cache update the retained keys are
+ * re-indexed from the start of the window by subtracting the temporal offset
+ * of the evicted chunks; the sink anchor keeps the first position).  Instead
+ * of rewriting the ring, the ring holds keys without their temporal rotation
+ * and each is rotated as it is read:
+ *   ring token t (logical order, oldest = 0) is at frame
+ *       f(t) = first_frame + t / tokens_per_frame   (integer division)
+ *   channel pair (2i, 2i+1), 0 <= i < rope_dims / 2, of its key turns by
+ *       f(t) * rope_base^(-2i / rope_dims):
+ *       (x, y) -> (x cos - y sin, x sin + y cos)
+ * The rotated key is rounded to bf16 before QK^T.  Sink and in-flight keys
+ * (and all queries) are used as given: the caller rotates them to their
+ * window positions.  The paper states neither the channel layout nor the
+ * frequencies of its RoPE, so they are arguments.
+ *   rope_dims        : even, 0 <= rope_dims <= d (0: no rotation, i.e.
+ *                      mw_bca_cache_fwd_sink)
+ *   rope_base        : > 1
+ *   tokens_per_frame : >= 1
+ *   first_frame      : 0 <= first_frame <= 2^24
+ * Every other argument is as for mw_bca_cache_fwd_sink.
+ */
+mw_status mw_bca_cache_fwd_rope(const void* q, const void* k_new, const void* v_new,
+                                const void* k_sink, const void* v_sink, int sink_len,
+                                const void* k_cache, const void* v_cache, int cache_cap,
+                                int cache_head, int cache_len, int rope_dims, float rope_base,
+                                int tokens_per_frame, int first_frame, void* o, float* lse,
+                                void* workspace, size_t ws_bytes, int B, int H, int n_q_chunks,
+                                int T_chunk, int d, float scale, void* stream);
+
+/*
  * Commit of finished tokens into the ring (Sec. 3.5: once a chunk reaches the
  * data endpoint its keys/values go to the cache and are never modified).
  * Copies rows r = 0..rows-1 of k_src / v_src ([B, H, rows, d] bf16) to

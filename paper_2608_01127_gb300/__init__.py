@@ -12,6 +12,7 @@ Entry points (same names as the C ABI, taking torch tensors):
                    T_chunk, scale=None, need_lse=True) -> (o, lse)
   mw_bca_cache_fwd_sink(q, k_new, v_new, k_sink, v_sink, k_cache, v_cache,
                         cache_head, cache_len, T_chunk, ...) -> (o, lse)
+  mw_bca_cache_fwd_rope(..., rope_dims, rope_base, tokens_per_frame, first_frame)
   mw_bca_cache_commit(k_cache, v_cache, slot_start, k_src, v_src)
   mw_device_status(clear=True), mw_set_option(name, value)
 Tensors are contiguous bf16 [B, H, rows, d] on the current CUDA device.
@@ -27,7 +28,7 @@ import torch
 
 __all__ = [
     "MWError", "library", "lib_path", "mw_bca_fwd", "mw_bca_bwd", "mw_bca_cache_fwd",
-    "mw_bca_cache_fwd_sink",
+    "mw_bca_cache_fwd_sink", "mw_bca_cache_fwd_rope",
     "mw_bca_cache_commit", "mw_bca_bwd_workspace_size", "mw_bca_cache_workspace_size",
     "mw_device_status", "mw_set_option", "BlockCausalAttention", "EXPORTED_SYMBOLS",
     "RingState",
@@ -41,6 +42,7 @@ EXPORTED_SYMBOLS = (
     "mw_bca_cache_workspace_size",
     "mw_bca_cache_fwd", "mw_bca_cache_commit", "mw_status_string", "mw_last_error",
     "mw_device_status", "mw_set_option", "mw_bca_cache_fwd_noalloc", "mw_bca_cache_fwd_sink",
+    "mw_bca_cache_fwd_rope",
 )
 
 STATUS = {0: "MW_OK", 1: "MW_ERR_INVALID_ARG", 2: "MW_ERR_UNSUPPORTED", 3: "MW_ERR_CUDA",
@@ -85,6 +87,8 @@ def library() -> ctypes.CDLL:
                                   _I, _I, _I, _I, _I, _F, _P]),
         "mw_bca_cache_fwd_sink": (_I, [_P, _P, _P, _P, _P, _I, _P, _P, _I, _I, _I, _P, _P, _P,
                                        _Z, _I, _I, _I, _I, _I, _F, _P]),
+        "mw_bca_cache_fwd_rope": (_I, [_P, _P, _P, _P, _P, _I, _P, _P, _I, _I, _I, _I, _F, _I, _I,
+                                       _P, _P, _P, _Z, _I, _I, _I, _I, _I, _F, _P]),
         "mw_bca_cache_commit": (_I, [_P, _P, _I, _I, _P, _P, _I, _I, _I, _I, _P]),
         "mw_bca_cache_fwd_noalloc": (_I, [_P, _P, _P, _P, _P, _I, _I, _I, _P, _P,
                                           _I, _I, _I, _I, _I, _F, _P]),
@@ -202,8 +206,21 @@ def mw_bca_cache_fwd_sink(q, k_new, v_new, k_sink, v_sink, k_cache, v_cache, cac
                       T_chunk, scale, need_lse, workspace, out)
 
 
+def mw_bca_cache_fwd_rope(q, k_new, v_new, k_sink, v_sink, k_cache, v_cache, cache_head: int,
+                          cache_len: int, T_chunk: int, rope_dims: int, rope_base: float,
+                          tokens_per_frame: int, first_frame: int, scale: Optional[float] = None,
+                          need_lse: bool = True, workspace: Optional[torch.Tensor] = None,
+                          out: Optional[torch.Tensor] = None):
+    """As mw_bca_cache_fwd_sink (k_sink may be None) with the ring's keys rotated
+    on read to window frames first_frame + t // tokens_per_frame (RoPE
+    re-shifting, Sec. 3.5); returns (O, LSE or None)."""
+    return _cache_fwd(q, k_new, v_new, k_sink, v_sink, k_cache, v_cache, cache_head, cache_len,
+                      T_chunk, scale, need_lse, workspace, out,
+                      rope=(rope_dims, rope_base, tokens_per_frame, first_frame))
+
+
 def _cache_fwd(q, k_new, v_new, k_sink, v_sink, k_cache, v_cache, cache_head, cache_len,
-               T_chunk, scale, need_lse, workspace, out):
+               T_chunk, scale, need_lse, workspace, out, rope=None):
     B, H, M, d = _bhnd(q, "q")
     for t, n in ((k_new, "k_new"), (v_new, "v_new")):
         if _bhnd(t, n) != (B, H, M, d):
@@ -226,7 +243,14 @@ def _cache_fwd(q, k_new, v_new, k_sink, v_sink, k_cache, v_cache, cache_head, ca
         workspace = torch.empty(ws_bytes, dtype=torch.uint8, device=q.device)
     o = torch.empty_like(q) if out is None else out
     lse = torch.empty((B, H, M), dtype=torch.float32, device=q.device) if need_lse else None
-    if k_sink is None:
+    if rope is not None:
+        _check(library().mw_bca_cache_fwd_rope(
+            _ptr(q), _ptr(k_new), _ptr(v_new), _ptr(k_sink), _ptr(v_sink), sink_len,
+            _ptr(k_cache), _ptr(v_cache), cap, cache_head, cache_len, int(rope[0]),
+            float(rope[1]), int(rope[2]), int(rope[3]), _ptr(o), _ptr(lse),
+            _ptr(workspace) if ws_bytes else None, ws_bytes, B, H, W, T_chunk, d,
+            _scale(scale, d), _stream()))
+    elif k_sink is None:
         _check(library().mw_bca_cache_fwd(
             _ptr(q), _ptr(k_new), _ptr(v_new), _ptr(k_cache), _ptr(v_cache), cap, cache_head,
             cache_len, _ptr(o), _ptr(lse), _ptr(workspace) if ws_bytes else None, ws_bytes,

@@ -7,6 +7,7 @@
 #include <climits>
 #include <cstdarg>
 #include <cstdio>
+#include <cmath>
 #include <cstring>
 #include <mutex>
 #include <string>
@@ -255,10 +256,17 @@ mw_status launch_status(cudaError_t e, const char* what) {
   return ok();
 }
 
+struct RopeArgs {
+  int dims = 0;          // 0: off
+  float log2_base = 0.f;
+  int per_frame = 1;
+  int first_frame = 0;
+};
+
 mw_status fwd_common(const void* q, const void* k, const void* v, const void* kr, const void* vr,
                      int cap, int head, int len, const void* ks, const void* vs, int sink_len,
-                     void* o, float* lse, void* ws, size_t ws_bytes, int BH, int rows_q, int T,
-                     int d, float scale, int splits, cudaStream_t stream) {
+                     const RopeArgs& rope, void* o, float* lse, void* ws, size_t ws_bytes, int BH,
+                     int rows_q, int T, int d, float scale, int splits, cudaStream_t stream) {
   DeviceScope scope(stream);
   MW_TRY(scope.status());
   unsigned* status = nullptr;
@@ -290,6 +298,10 @@ mw_status fwd_common(const void* q, const void* k, const void* v, const void* kr
   p.ring_head = len > 0 ? head : 0;
   p.ring_len = len;
   p.sink_len = sink_len;
+  p.rope_dims = len > 0 ? rope.dims : 0;
+  p.rope_log2_base = rope.log2_base;
+  p.rope_per_frame = rope.per_frame;
+  p.rope_first_frame = rope.first_frame;
   p.num_splits = splits;
   p.scale_log2 = scale * 1.4426950408889634f;
   p.o = static_cast<__nv_bfloat16*>(o);
@@ -363,7 +375,7 @@ mw_status mw_bca_fwd(const void* q, const void* k, const void* v, void* o, float
   MW_TRY(check_ptr(o, "o"));
   if (lse && (reinterpret_cast<uintptr_t>(lse) & 3u))
     return fail(MW_ERR_INVALID_ARG, "lse is not 4-byte aligned");
-  return fwd_common(q, k, v, nullptr, nullptr, 1, 0, 0, nullptr, nullptr, 0, o, lse, nullptr, 0, B * H,
+  return fwd_common(q, k, v, nullptr, nullptr, 1, 0, 0, nullptr, nullptr, 0, RopeArgs{}, o, lse, nullptr, 0, B * H,
                     static_cast<int>(N), T_chunk, d, scale, 1, static_cast<cudaStream_t>(stream));
 }
 
@@ -488,6 +500,18 @@ mw_status mw_bca_cache_fwd_sink(const void* q, const void* k_new, const void* v_
                                 int cache_head, int cache_len, void* o, float* lse,
                                 void* workspace, size_t ws_bytes, int B, int H, int n_q_chunks,
                                 int T_chunk, int d, float scale, void* stream) {
+  return mw_bca_cache_fwd_rope(q, k_new, v_new, k_sink, v_sink, sink_len, k_cache, v_cache,
+                               cache_cap, cache_head, cache_len, 0, 0.f, 1, 0, o, lse, workspace,
+                               ws_bytes, B, H, n_q_chunks, T_chunk, d, scale, stream);
+}
+
+mw_status mw_bca_cache_fwd_rope(const void* q, const void* k_new, const void* v_new,
+                                const void* k_sink, const void* v_sink, int sink_len,
+                                const void* k_cache, const void* v_cache, int cache_cap,
+                                int cache_head, int cache_len, int rope_dims, float rope_base,
+                                int tokens_per_frame, int first_frame, void* o, float* lse,
+                                void* workspace, size_t ws_bytes, int B, int H, int n_q_chunks,
+                                int T_chunk, int d, float scale, void* stream) {
   MW_TRY(check_dims(B, H, d));
   if (n_q_chunks < 1 || T_chunk < 1)
     return fail(MW_ERR_INVALID_ARG, "n_q_chunks=%d and T_chunk=%d must be >= 1", n_q_chunks, T_chunk);
@@ -502,6 +526,21 @@ mw_status mw_bca_cache_fwd_sink(const void* q, const void* k_new, const void* v_
   if (sink_len < 0 || sink_len > (1 << 24))
     return fail(MW_ERR_INVALID_ARG, "sink_len=%d out of range [0, 2^24]", sink_len);
   if (!(scale > 0.f)) return fail(MW_ERR_INVALID_ARG, "scale must be > 0");
+  RopeArgs rope;
+  if (rope_dims != 0) {
+    if (rope_dims < 0 || rope_dims > d || (rope_dims & 1))
+      return fail(MW_ERR_INVALID_ARG, "rope_dims=%d must be even and in [0, d=%d]", rope_dims, d);
+    if (!(rope_base > 1.f) || !(rope_base < 1e30f))
+      return fail(MW_ERR_INVALID_ARG, "rope_base must be > 1 and finite");
+    if (tokens_per_frame < 1)
+      return fail(MW_ERR_INVALID_ARG, "tokens_per_frame=%d must be >= 1", tokens_per_frame);
+    if (first_frame < 0 || first_frame > (1 << 24))
+      return fail(MW_ERR_INVALID_ARG, "first_frame=%d out of range [0, 2^24]", first_frame);
+    rope.dims = rope_dims;
+    rope.log2_base = std::log2(rope_base);
+    rope.per_frame = tokens_per_frame;
+    rope.first_frame = first_frame;
+  }
   MW_TRY(check_ptr(q, "q"));
   MW_TRY(check_ptr(k_new, "k_new"));
   MW_TRY(check_ptr(v_new, "v_new"));
@@ -527,7 +566,7 @@ mw_status mw_bca_cache_fwd_sink(const void* q, const void* k_new, const void* v_
       return fail(MW_ERR_INVALID_ARG, "workspace is not 256-byte aligned");
   }
   return fwd_common(q, k_new, v_new, k_cache, v_cache, cache_cap, cache_head, cache_len, k_sink,
-                    v_sink, sink_len, o, lse, need > 0 ? workspace : nullptr, ws_bytes, BH,
+                    v_sink, sink_len, rope, o, lse, need > 0 ? workspace : nullptr, ws_bytes, BH,
                     static_cast<int>(rows), T_chunk, d, scale, splits,
                     static_cast<cudaStream_t>(stream));
 }

@@ -11,7 +11,9 @@
 //   warps 0-3 / 4-7  softmax of query tile 0 / 1 (one thread per row = TMEM lane)
 //   warp 8           TMA producer (Q once, then K/V tiles through a ring of stages)
 //   warp 9           tcgen05 issuer (S = Q K^T into TMEM, O += P V with P in TMEM)
-//   warps 10-11      idle (they complete warpgroup 2 for the register re-split)
+//   warps 10-11      RoPE re-shift of ring key tiles in shared memory when it
+//                    is enabled (otherwise idle; they complete warpgroup 2 for
+//                    the register re-split)
 // TMEM (512 columns): S_t at column 128 t (P_t, bf16, overwrites its first 64
 // columns), O_t at 256 + D t.
 #include "mw_internal.h"
@@ -37,8 +39,10 @@ struct FwdLayout {
   static constexpr int OW = SUM_MMA ? D + 16 : D;     // O columns in TMEM
   static constexpr int OFF_ONES = OFF_V + STAGES * TILE_BYTES;
   static constexpr int ONES_BYTES = SUM_MMA ? REGION_BYTES : 0;
-  static constexpr int OFF_BAR = OFF_ONES + ONES_BYTES;
-  static constexpr int NBAR = 1 + 4 * STAGES + 3 * QT + 1;
+  static constexpr int OFF_ROPE = OFF_ONES + ONES_BYTES;   // per-pair RoPE frequencies
+  static constexpr int ROPE_BYTES = D / 2 * 4;
+  static constexpr int OFF_BAR = OFF_ROPE + ROPE_BYTES;
+  static constexpr int NBAR = 1 + 5 * STAGES + 3 * QT + 1;
   static constexpr int OFF_MISC = OFF_BAR + NBAR * 8;
   static constexpr int BYTES = OFF_MISC + 16;
   static constexpr uint32_t S_COL(int t) { return 128u * t; }
@@ -63,15 +67,17 @@ struct TileSrc {
   int seg;     // kSegOwn, kSegRing or kSegSink: which tensor maps hold the tile
   int row0;    // first physical row of the tile
   int end;     // ring and sink: exclusive end of the valid rows; own: unused
+  int t0;      // ring: logical index (oldest = 0) of the tile's first row
 };
 
 struct Segs {
   int nS, nA, nB, nC;
-  int endS, headA, endA, endB;
+  int endS, headA, endA, endB, lenA;
 };
 
 __device__ __forceinline__ TileSrc tile_src(const Segs& g, int j) {
   TileSrc s;
+  s.t0 = 0;
   if (j < g.nS) {
     s.seg = kSegSink;
     s.row0 = j * kTileRows;
@@ -83,10 +89,12 @@ __device__ __forceinline__ TileSrc tile_src(const Segs& g, int j) {
     s.seg = kSegRing;
     s.row0 = g.headA + j * kTileRows;
     s.end = g.endA;
+    s.t0 = j * kTileRows;
   } else if (j < g.nA + g.nB) {
     s.seg = kSegRing;
     s.row0 = (j - g.nA) * kTileRows;
     s.end = g.endB;
+    s.t0 = g.lenA + (j - g.nA) * kTileRows;
   } else {
     s.seg = kSegOwn;
     s.row0 = (j - g.nA - g.nB) * kTileRows;
@@ -95,7 +103,10 @@ __device__ __forceinline__ TileSrc tile_src(const Segs& g, int j) {
   return s;
 }
 
-template <int D>
+// ROPE: the cache form with the ring's RoPE re-shift (warps 10-11 rotate ring
+// key tiles before the MMAs read them); the training and plain cache forms
+// are compiled without it.
+template <int D, bool ROPE>
 __global__ void __launch_bounds__(FwdLayout<D>::THREADS, 1)
     bca_fwd_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_k,
                    const __grid_constant__ CUtensorMap tm_v, const __grid_constant__ CUtensorMap tm_kr,
@@ -115,7 +126,8 @@ __global__ void __launch_bounds__(FwdLayout<D>::THREADS, 1)
   uint64_t* k_empty = k_full + NS;
   uint64_t* v_full = k_empty + NS;
   uint64_t* v_empty = v_full + NS;
-  uint64_t* s_full = v_empty + NS;
+  uint64_t* k_rdy = v_empty + NS;  // K tile in shared memory, RoPE re-shift applied
+  uint64_t* s_full = k_rdy + NS;
   uint64_t* p_full = s_full + QT;
   uint64_t* p_half = p_full + QT;  // first 64 keys of P in TMEM
   uint64_t* o_full = p_half + QT;
@@ -136,6 +148,7 @@ __global__ void __launch_bounds__(FwdLayout<D>::THREADS, 1)
   const int c_end = (last_row / p.T + 1) * p.T;  // keys of segment C visible to the block
 
   Segs g;
+  g.lenA = 0;
   g.nS = (p.sink_len + kTileRows - 1) / kTileRows;
   g.endS = p.sink_len;
   const int lenA = min(p.ring_len, p.ring_cap - p.ring_head);
@@ -145,6 +158,7 @@ __global__ void __launch_bounds__(FwdLayout<D>::THREADS, 1)
   g.nC = (c_end + kTileRows - 1) / kTileRows;
   g.headA = p.ring_head;
   g.endA = p.ring_head + lenA;
+  g.lenA = lenA;
   g.endB = lenB;
   const int n_all = g.nS + g.nA + g.nB + g.nC;
   const int j0 = (int)((long long)split * n_all / p.num_splits);
@@ -158,6 +172,7 @@ __global__ void __launch_bounds__(FwdLayout<D>::THREADS, 1)
       mbar_init(&k_empty[s], 1);
       mbar_init(&v_full[s], 1);
       mbar_init(&v_empty[s], 1);
+      mbar_init(&k_rdy[s], 2);
     }
     for (int t = 0; t < QT; ++t) {
       mbar_init(&s_full[t], 1);
@@ -275,7 +290,7 @@ __global__ void __launch_bounds__(FwdLayout<D>::THREADS, 1)
         const uint32_t ph = (i / NS) & 1;
         const int stp = (i + NS - 1) % NS;
         const uint32_t php = ((i - 1) / NS) & 1;
-        if (!(ok = warp_wait(&k_full[st], ph, ctl))) break;
+        if (!(ok = warp_wait(ROPE ? &k_rdy[st] : &k_full[st], ph, ctl))) break;
         tc_fence_after();
         for (int t = 0; t < QT; ++t) {
           if (i > 0) {
@@ -312,6 +327,52 @@ __global__ void __launch_bounds__(FwdLayout<D>::THREADS, 1)
           umma_commit(o_full);
         }
       }
+    }
+  } else if (ROPE && (warp == 10 || warp == 11) && n_local > 0) {
+    // ------------------------------------------------------------ RoPE re-shift
+    // Ring keys are stored without their temporal rotation; after evictions the
+    // window is re-indexed from its start (Sec. 3.5), so ring token t (logical
+    // order) is rotated to frame first_frame + t / per_frame here, in shared
+    // memory, between the TMA copy and the MMAs that read the tile.  Channel
+    // pair (2i, 2i+1), i < rope_dims / 2, turns by frame * base^(-2i/rope_dims).
+    const int tid = threadIdx.x - 320;  // 0..63
+    float* omega = reinterpret_cast<float*>(smem + L::OFF_ROPE);
+    const int pairs = p.rope_dims / 2;
+    for (int i = tid; i < pairs; i += 64)
+      omega[i] = exp2f(-(2.f * i / p.rope_dims) * p.rope_log2_base);
+    asm volatile("barrier.cta.sync 1, 64;" ::: "memory");
+    const float inv_2pi = 0.15915494309189535f;
+    const float two_pi = 6.283185307179586f;
+    for (int i = 0; i < n_local; ++i) {
+      const int st = i % NS;
+      if (!warp_wait(&k_full[st], (i / NS) & 1, ctl)) break;
+      const TileSrc src = tile_src(g, j0 + i);
+      if (src.seg == kSegRing) {
+        uint8_t* tile = sK + st * L::TILE_BYTES;
+#pragma unroll 1
+        for (int rr = 0; rr < 2; ++rr) {
+          const int r = 2 * tid + rr;
+          if (src.row0 + r >= src.end) continue;  // rows past the ring's valid end
+          const float f = static_cast<float>(p.rope_first_frame + (src.t0 + r) / p.rope_per_frame);
+#pragma unroll 1
+          for (int pi = 0; pi < pairs; ++pi) {
+            const int c = 2 * pi;  // 128-byte swizzle: 16-byte chunk index ^ (row mod 8)
+            uint32_t* a = reinterpret_cast<uint32_t*>(
+                tile + (c >> 6) * L::REGION_BYTES + r * 128 +
+                (((((c & 63) * 2) >> 4) ^ (r & 7)) << 4) + ((c * 2) & 15));
+            float th = f * omega[pi];
+            th = fmaf(-two_pi, rintf(th * inv_2pi), th);
+            float sn, cs;
+            __sincosf(th, &sn, &cs);
+            const uint32_t v = *a;
+            const float x0 = __uint_as_float(v << 16), x1 = __uint_as_float(v & 0xffff0000u);
+            *a = pack_bf16x2(x0 * cs - x1 * sn, x0 * sn + x1 * cs);
+          }
+        }
+        fence_proxy_async_smem();  // the tensor core reads the tile next
+      }
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&k_rdy[st]);
     }
   }
   } else {
@@ -523,7 +584,7 @@ __global__ void __launch_bounds__(256) combine_kernel(const float* __restrict__ 
   if (lse && lane == 0) lse[row] = wsum > 0.f ? m + __logf(wsum) : -INFINITY;
 }
 
-template <int D>
+template <int D, bool ROPE>
 cudaError_t launch_fwd_t(const CUtensorMap& tq, const CUtensorMap& tk, const CUtensorMap& tv,
                          const CUtensorMap& tkr, const CUtensorMap& tvr, const CUtensorMap& tks,
                          const CUtensorMap& tvs, const FwdParams& p, cudaStream_t s) {
@@ -533,16 +594,16 @@ cudaError_t launch_fwd_t(const CUtensorMap& tq, const CUtensorMap& tk, const CUt
     // The in-kernel register re-split assumes the launch register count; with
     // any other count its setmaxnreg.inc could never be satisfied, so refuse.
     cudaFuncAttributes fa;
-    cudaError_t e = cudaFuncGetAttributes(&fa, bca_fwd_kernel<D>);
+    cudaError_t e = cudaFuncGetAttributes(&fa, bca_fwd_kernel<D, ROPE>);
     if (e != cudaSuccess) return e;
     if (fa.numRegs != L::REGS_LAUNCH) return cudaErrorInvalidKernelImage;
-    e = cudaFuncSetAttribute(bca_fwd_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+    e = cudaFuncSetAttribute(bca_fwd_kernel<D, ROPE>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                              L::BYTES);
     if (e != cudaSuccess) return e;
     attr_set = true;
   }
   const unsigned grid = static_cast<unsigned>(p.BH) * p.n_qblocks * p.num_splits;
-  bca_fwd_kernel<D><<<grid, L::THREADS, L::BYTES, s>>>(tq, tk, tv, tkr, tvr, tks, tvs, p);
+  bca_fwd_kernel<D, ROPE><<<grid, L::THREADS, L::BYTES, s>>>(tq, tk, tv, tkr, tvr, tks, tvs, p);
   return cudaGetLastError();
 }
 
@@ -551,8 +612,12 @@ cudaError_t launch_fwd_t(const CUtensorMap& tq, const CUtensorMap& tk, const CUt
 cudaError_t launch_fwd(int d, const CUtensorMap& tq, const CUtensorMap& tk, const CUtensorMap& tv,
                        const CUtensorMap& tkr, const CUtensorMap& tvr, const CUtensorMap& tks,
                        const CUtensorMap& tvs, const FwdParams& p, cudaStream_t s) {
-  if (d == 64) return launch_fwd_t<64>(tq, tk, tv, tkr, tvr, tks, tvs, p, s);
-  return launch_fwd_t<128>(tq, tk, tv, tkr, tvr, tks, tvs, p, s);
+  if (p.rope_dims > 0) {
+    if (d == 64) return launch_fwd_t<64, true>(tq, tk, tv, tkr, tvr, tks, tvs, p, s);
+    return launch_fwd_t<128, true>(tq, tk, tv, tkr, tvr, tks, tvs, p, s);
+  }
+  if (d == 64) return launch_fwd_t<64, false>(tq, tk, tv, tkr, tvr, tks, tvs, p, s);
+  return launch_fwd_t<128, false>(tq, tk, tv, tkr, tvr, tks, tvs, p, s);
 }
 
 cudaError_t launch_combine(int d, const float* o_part, const float* lse_part, __nv_bfloat16* o,

@@ -126,6 +126,23 @@ def test_sink_entry_rejects_bad_sink(mw):
     assert call(head=1024) == INVALID  # the ring checks still apply
 
 
+def test_rope_entry_rejects_bad_rope(mw):
+    lib = mw.library()
+
+    def call(dims=32, base=1e4, per_frame=440, first=1):
+        return lib.mw_bca_cache_fwd_rope(FAKE, FAKE, FAKE, None, None, 0, FAKE, FAKE, 1024, 0,
+                                         1024, dims, base, per_frame, first, FAKE, None, None, 0,
+                                         1, 2, 1, 64, 128, 0.1, None)
+
+    assert call(dims=-2) == INVALID
+    assert call(dims=31) == INVALID       # odd
+    assert call(dims=130) == INVALID      # more than d
+    assert call(base=1.0) == INVALID
+    assert call(base=float("nan")) == INVALID
+    assert call(per_frame=0) == INVALID
+    assert call(first=-1) == INVALID
+
+
 def test_commit_rejects_bad_slots(mw):
     lib = mw.library()
 

@@ -339,6 +339,72 @@ def test_sink_anchor_config(mw):
     check_lse(lse[:, heads], lse_ref, "sink_anchor")
 
 
+ROPE_SMALL = [
+    # B, H, W, T, cap, length, head, sink, d, rope_dims, per_frame, first_frame, splits
+    (1, 2, 1, 64, 512, 512, 100, 0, 128, 32, 64, 1, 0),      # tiles span two frames
+    (1, 2, 2, 100, 1000, 300, 900, 32, 64, 64, 7, 0, 0),     # every channel, many frames per tile
+    (1, 1, 1, 880, 1760, 1760, 1759, 440, 128, 16, 440, 1, 3),  # one-frame sink, frames of 440
+    (2, 1, 2, 64, 640, 640, 0, 0, 64, 2, 1, 5, 0),           # one token per frame
+]
+
+
+@pytest.mark.parametrize("B,H,W,T,cap,length,head,sink,d,rope_dims,per_frame,first,splits",
+                         ROPE_SMALL)
+def test_cache_forward_rope_reshift(mw, B, H, W, T, cap, length, head, sink, d, rope_dims,
+                                    per_frame, first, splits):
+    q, kn, vn, kr, vr = _ring_case(B, H, W, T, cap, d, seed=cap + rope_dims + per_frame)
+    g = torch.Generator().manual_seed(sink + 11)
+    ks, vs = (torch.randn(B, H, sink, d, generator=g).to(torch.bfloat16) for _ in range(2))
+    sc, base = 1.0 / math.sqrt(d), 10000.0
+    mw.mw_set_option("cache_splits", splits)
+    try:
+        o, lse = mw.mw_bca_cache_fwd_rope(q.cuda(), kn.cuda(), vn.cuda(),
+                                          ks.cuda() if sink else None, vs.cuda() if sink else None,
+                                          kr.cuda(), vr.cuda(), head, length, T, rope_dims, base,
+                                          per_frame, first, sc)
+    finally:
+        mw.mw_set_option("cache_splits", 0)
+    o_ref, lse_ref = oracle.cache_fwd(q, kn, vn, kr, vr, cap, head, length, T, sc,
+                                      ks if sink else None, vs if sink else None,
+                                      rope=(rope_dims, base, per_frame, first))
+    tag = f"rope{rope_dims} P{per_frame} first{first} sink{sink} len{length} splits{splits}"
+    check_o(o, o_ref, tag)
+    check_lse(lse, lse_ref, tag)
+
+
+def test_rope_reshift_streaming(mw):
+    """Streaming with a sink and a FIFO ring whose keys are stored without their
+    temporal rotation: each step the in-flight chunk is rotated to the frames
+    after the window (test side), attends, and its unrotated keys are
+    committed; evictions re-index the window without rewriting the ring."""
+    B, H, T, d, P, cap, sink = 1, 2, 64, 128, 32, 256, 32
+    rope_dims, base, sc = 32, 10000.0, 1.0 / math.sqrt(d)
+    g = torch.Generator().manual_seed(41)
+    ks, vs = (torch.randn(B, H, sink, d, generator=g).to(torch.bfloat16) for _ in range(2))
+    ks = oracle.rope_rotate(ks, torch.zeros(sink, dtype=torch.long), rope_dims, base).to(torch.bfloat16)
+    kr = torch.zeros(B, H, cap, d, dtype=torch.bfloat16)
+    vr = torch.zeros(B, H, cap, d, dtype=torch.bfloat16)
+    ring = mw.RingState(cap, 0, 0)
+    kr_g, vr_g = kr.cuda(), vr.cuda()
+    first = sink // P  # the ring starts right after the sink frame(s)
+    for step in range(7):  # the ring fills after 4 steps, then evicts
+        q_raw, k_raw, v_new = (torch.randn(B, H, T, d, generator=g).to(torch.bfloat16)
+                               for _ in range(3))
+        frames = first + ring.length // P + torch.arange(T) // P
+        q = oracle.rope_rotate(q_raw, frames, rope_dims, base).to(torch.bfloat16)
+        k = oracle.rope_rotate(k_raw, frames, rope_dims, base).to(torch.bfloat16)
+        o, lse = mw.mw_bca_cache_fwd_rope(q.cuda(), k.cuda(), v_new.cuda(), ks.cuda(), vs.cuda(),
+                                          kr_g, vr_g, ring.head, ring.length, T, rope_dims, base,
+                                          P, first, sc)
+        o_ref, lse_ref = oracle.cache_fwd(q, k, v_new, kr, vr, cap, ring.head, ring.length, T, sc,
+                                          ks, vs, rope=(rope_dims, base, P, first))
+        check_o(o, o_ref, f"stream step {step}")
+        check_lse(lse, lse_ref, f"stream step {step}")
+        slot = ring.commit(T)
+        mw.mw_bca_cache_commit(kr_g, vr_g, slot, k_raw.cuda(), v_new.cuda())
+        kr, vr = oracle.cache_commit(kr, vr, cap, slot, k_raw, v_new)
+
+
 def test_device_status_is_clean(mw):
     torch.cuda.synchronize()
     assert mw.mw_device_status() == 0
