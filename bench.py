@@ -445,9 +445,10 @@ def run_extras(mw, dev, peaks):
     flush = flush_buf.zero_
     extra = {}
     # forward / backward of the other training workloads: d=128 with peaky
-    # logits, and the paper's 32-chunk window of 600-token chunks at the
-    # MiniWorld-1B head layout (12 heads of 128)
-    for name in ("train_h16_d128_peaky", "train_1b_32x600"):
+    # logits, the paper's 32-chunk window of 600-token chunks at the
+    # MiniWorld-1B head layout (12 heads of 128), and the 0.5B head dim (72,
+    # run on the 128-wide kernels with zero-filled columns)
+    for name in ("train_h16_d128_peaky", "train_1b_32x600", "train_05b_d72"):
         cfg = TRAIN_CONFIGS[name]
         x = gen_train(cfg)
         q, k, v, do = (x[n].to(dev) for n in ("q", "k", "v", "do"))

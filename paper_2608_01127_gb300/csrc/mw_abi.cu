@@ -55,11 +55,18 @@ mw_status check_ptr(const void* p, const char* name) {
   return MW_OK;
 }
 
+// Head dims: the kernels are built for 64 and 128; a head dim in between (a
+// multiple of 8, e.g. 72) runs on the 128 kernels, whose TMA maps read the
+// caller's d columns and fill the rest of each 128-column tile with zeros.
+bool d_supported(int d) { return d >= 64 && d <= 128 && d % 8 == 0; }
+int kernel_d(int d) { return d == 64 ? 64 : 128; }
+
 mw_status check_dims(int B, int H, int d) {
   if (B < 1 || H < 1) return fail(MW_ERR_INVALID_ARG, "B and H must be >= 1 (B=%d H=%d)", B, H);
   if (static_cast<long long>(B) * H > (1 << 20))
     return fail(MW_ERR_INVALID_ARG, "B*H=%lld exceeds 2^20", static_cast<long long>(B) * H);
-  if (d != 64 && d != 128) return fail(MW_ERR_UNSUPPORTED, "head dim d=%d (supported: 64, 128)", d);
+  if (!d_supported(d))
+    return fail(MW_ERR_UNSUPPORTED, "head dim d=%d (supported: multiples of 8 from 64 to 128)", d);
   return MW_OK;
 }
 
@@ -289,9 +296,11 @@ mw_status fwd_common(const void* q, const void* k, const void* v, const void* kr
     tks = tk;
     tvs = tv;
   }
+  const int D = kernel_d(d);
   mw::FwdParams p{};
   p.BH = BH;
   p.rows_q = rows_q;
+  p.d_io = d;
   p.T = T;
   p.n_qblocks = ceil_div(rows_q, mw::kFwdBlockRows);
   p.ring_cap = len > 0 ? cap : 1;
@@ -310,17 +319,17 @@ mw_status fwd_common(const void* q, const void* k, const void* v, const void* kr
   p.budget_ns = budget_ns();
   p.debug_skip_q = static_cast<int>(g_opt_skip_q);
   if (p.num_splits > 1) {
-    const size_t need = cache_ws_bytes(p.num_splits, BH, rows_q, d);
+    const size_t need = cache_ws_bytes(p.num_splits, BH, rows_q, D);
     if (ws_bytes < need)
       return fail(MW_ERR_WORKSPACE, "workspace %zu bytes, need %zu", ws_bytes, need);
     char* base = static_cast<char*>(ws);
     p.o_part = reinterpret_cast<float*>(base);
     p.lse_part = reinterpret_cast<float*>(
-        base + align256(static_cast<size_t>(p.num_splits) * BH * rows_q * d * sizeof(float)));
+        base + align256(static_cast<size_t>(p.num_splits) * BH * rows_q * D * sizeof(float)));
   }
-  MW_TRY(launch_status(mw::launch_fwd(d, tq, tk, tv, tkr, tvr, tks, tvs, p, stream), "forward kernel launch"));
+  MW_TRY(launch_status(mw::launch_fwd(D, tq, tk, tv, tkr, tvr, tks, tvs, p, stream), "forward kernel launch"));
   if (p.num_splits > 1)
-    MW_TRY(launch_status(mw::launch_combine(d, p.o_part, p.lse_part, p.o, lse, p.num_splits, BH,
+    MW_TRY(launch_status(mw::launch_combine(D, d, p.o_part, p.lse_part, p.o, lse, p.num_splits, BH,
                                             rows_q, stream),
                          "combine kernel launch"));
   return ok();
@@ -380,11 +389,11 @@ mw_status mw_bca_fwd(const void* q, const void* k, const void* v, void* o, float
 }
 
 size_t mw_bca_bwd_workspace_size(int B, int H, int n_chunks, int T_chunk, int d) {
-  if (B < 1 || H < 1 || n_chunks < 1 || T_chunk < 1 || (d != 64 && d != 128)) return 0;
+  if (B < 1 || H < 1 || n_chunks < 1 || T_chunk < 1 || !d_supported(d)) return 0;
   const long long N = static_cast<long long>(n_chunks) * T_chunk;
   if (N > (1 << 24)) return 0;
   const int N_pad = ceil_div(N, mw::kTileRows) * mw::kTileRows;
-  return bwd_ws_layout(B * H, N_pad, d).total;
+  return bwd_ws_layout(B * H, N_pad, kernel_d(d)).total;
 }
 
 mw_status mw_bca_bwd_stage(int stage, const void* q, const void* k, const void* v, const void* o,
@@ -416,7 +425,7 @@ mw_status mw_bca_bwd_stage(int stage, const void* q, const void* k, const void* 
   if (post) MW_TRY(check_ptr(dq, "dq"));
   const int BH = B * H;
   const int N_pad = ceil_div(N, mw::kTileRows) * mw::kTileRows;
-  const BwdWs w = bwd_ws_layout(BH, N_pad, d);
+  const BwdWs w = bwd_ws_layout(BH, N_pad, kernel_d(d));
   if (workspace == nullptr || ws_bytes < w.total)
     return fail(MW_ERR_WORKSPACE, "workspace %zu bytes, need %zu", ws_bytes, w.total);
   if (reinterpret_cast<uintptr_t>(workspace) & 255u)
@@ -429,7 +438,7 @@ mw_status mw_bca_bwd_stage(int stage, const void* q, const void* k, const void* 
   float* lse2 = reinterpret_cast<float*>(base + w.lse2);
   float* delta = reinterpret_cast<float*>(base + w.delta);
   if (pre)
-    MW_TRY(launch_status(mw::launch_bwd_pre(d, static_cast<const __nv_bfloat16*>(o),
+    MW_TRY(launch_status(mw::launch_bwd_pre(kernel_d(d), d, static_cast<const __nv_bfloat16*>(o),
                                             static_cast<const __nv_bfloat16*>(dout), lse, lse2,
                                             delta, dq_acc, BH, static_cast<int>(N), N_pad, s),
                          "backward pre kernel launch"));
@@ -437,16 +446,18 @@ mw_status mw_bca_bwd_stage(int stage, const void* q, const void* k, const void* 
     unsigned* status = nullptr;
     MW_TRY(status_ptr(&status));
     CUtensorMap tq, tk, tv, tdo, tdq;
-    const int qrows = mw::bwd_q_rows(d);  // query rows per backward step
+    const int D = kernel_d(d);
+    const int qrows = mw::bwd_q_rows(D);  // query rows per backward step
     MW_TRY(make_map(&tq, q, static_cast<int>(N), BH, d, "q", qrows));
     MW_TRY(make_map(&tk, k, static_cast<int>(N), BH, d, "k"));
     MW_TRY(make_map(&tv, v, static_cast<int>(N), BH, d, "v"));
     MW_TRY(make_map(&tdo, dout, static_cast<int>(N), BH, d, "dout", qrows));
-    MW_TRY(make_map(&tdq, dq_acc, N_pad, BH, d, "dq_acc", 32, true));
+    MW_TRY(make_map(&tdq, dq_acc, N_pad, BH, D, "dq_acc", 32, true));
     mw::BwdParams p{};
     p.BH = BH;
     p.N = static_cast<int>(N);
     p.N_pad = N_pad;
+    p.d_io = d;
     p.T = T_chunk;
     p.scale_log2 = scale * 1.4426950408889634f;
     p.scale = scale;
@@ -457,10 +468,10 @@ mw_status mw_bca_bwd_stage(int stage, const void* q, const void* k, const void* 
     p.dv = static_cast<__nv_bfloat16*>(dv);
     p.status = status;
     p.budget_ns = budget_ns();
-    MW_TRY(launch_status(mw::launch_bwd_main(d, tq, tk, tv, tdo, tdq, p, s), "backward kernel launch"));
+    MW_TRY(launch_status(mw::launch_bwd_main(D, tq, tk, tv, tdo, tdq, p, s), "backward kernel launch"));
   }
   if (post)
-    MW_TRY(launch_status(mw::launch_bwd_post(d, dq_acc, static_cast<__nv_bfloat16*>(dq), scale, BH,
+    MW_TRY(launch_status(mw::launch_bwd_post(kernel_d(d), d, dq_acc, static_cast<__nv_bfloat16*>(dq), scale, BH,
                                              static_cast<int>(N), N_pad, s),
                          "backward post kernel launch"));
   return ok();
@@ -476,12 +487,12 @@ mw_status mw_bca_bwd(const void* q, const void* k, const void* v, const void* o,
 
 size_t mw_bca_cache_workspace_size(int B, int H, int n_q_chunks, int T_chunk, int d,
                                    int cache_len) {
-  if (B < 1 || H < 1 || n_q_chunks < 1 || T_chunk < 1 || cache_len < 0 || (d != 64 && d != 128))
+  if (B < 1 || H < 1 || n_q_chunks < 1 || T_chunk < 1 || cache_len < 0 || !d_supported(d))
     return 0;
   const long long rows = static_cast<long long>(n_q_chunks) * T_chunk;
   if (rows > (1 << 24)) return 0;
   const int splits = plan_splits(B * H, static_cast<int>(rows), cache_len);
-  return cache_ws_bytes(splits, B * H, static_cast<int>(rows), d);
+  return cache_ws_bytes(splits, B * H, static_cast<int>(rows), kernel_d(d));
 }
 
 mw_status mw_bca_cache_fwd(const void* q, const void* k_new, const void* v_new,
@@ -558,7 +569,7 @@ mw_status mw_bca_cache_fwd_rope(const void* q, const void* k_new, const void* v_
   const int BH = B * H;
   // the split plan counts every cached key (sink and ring alike)
   const int splits = plan_splits(BH, static_cast<int>(rows), sink_len + cache_len);
-  const size_t need = cache_ws_bytes(splits, BH, static_cast<int>(rows), d);
+  const size_t need = cache_ws_bytes(splits, BH, static_cast<int>(rows), kernel_d(d));
   if (need > 0) {
     if (workspace == nullptr || ws_bytes < need)
       return fail(MW_ERR_WORKSPACE, "workspace %zu bytes, need %zu", ws_bytes, need);
@@ -670,7 +681,7 @@ extern "C" mw_status mw_bca_cache_fwd_noalloc(const void* q, const void* k_new, 
   if (cache_len < 0 || cache_len > cache_cap)
     return fail(MW_ERR_INVALID_ARG, "cache_len=%d not in [0, cache_cap=%d]", cache_len, cache_cap);
   const int splits = plan_splits(B * H, static_cast<int>(rows), cache_len);
-  const size_t need = cache_ws_bytes(splits, B * H, static_cast<int>(rows), d);
+  const size_t need = cache_ws_bytes(splits, B * H, static_cast<int>(rows), kernel_d(d));
   if (need > MW_NOALLOC_SCRATCH_BYTES)
     return fail(MW_ERR_WORKSPACE,
                 "these sizes need %zu bytes of split-KV scratch; the static scratch holds %u "

@@ -510,17 +510,21 @@ __global__ void __launch_bounds__(BwdLayout<D>::THREADS, 1)
       const uint32_t col0 = wg == 0 ? L::DK_COL : L::DV_COL;
       const float mul = wg == 0 ? p.scale : 1.f;
       __nv_bfloat16* out = wg == 0 ? p.dk : p.dv;
-      const size_t row_off = (static_cast<size_t>(bh) * p.N + krow) * D;
+      // the caller's rows hold d_io <= D columns (multiples of 8); only the
+      // 128-wide kernel serves padded head dims
+      const int d_io = (D == 64) ? D : p.d_io;
+      const size_t row_off = (static_cast<size_t>(bh) * p.N + krow) * d_io;
 #pragma unroll
       for (int c = 0; c < D / 32; ++c) {
         uint32_t r[32];
         tmem_ld32(lane_base + col0 + 32 * c, r);
         tmem_wait_ld();
-        if (k_valid) {
+        if (k_valid && 32 * c < d_io) {
+          const int n16 = min(4, (d_io - 32 * c) / 8);
           uint4* dst = reinterpret_cast<uint4*>(out + row_off + 32 * c);
 #pragma unroll
           for (int k = 0; k < 4; ++k)
-            dst[k] = make_uint4(pack_bf16x2(__uint_as_float(r[8 * k]) * mul, __uint_as_float(r[8 * k + 1]) * mul),
+            if (k < n16) dst[k] = make_uint4(pack_bf16x2(__uint_as_float(r[8 * k]) * mul, __uint_as_float(r[8 * k + 1]) * mul),
                                 pack_bf16x2(__uint_as_float(r[8 * k + 2]) * mul, __uint_as_float(r[8 * k + 3]) * mul),
                                 pack_bf16x2(__uint_as_float(r[8 * k + 4]) * mul, __uint_as_float(r[8 * k + 5]) * mul),
                                 pack_bf16x2(__uint_as_float(r[8 * k + 6]) * mul, __uint_as_float(r[8 * k + 7]) * mul));
@@ -612,7 +616,8 @@ __global__ void __launch_bounds__(256) bwd_pre_kernel(const __nv_bfloat16* __res
                                                       float* __restrict__ lse2,
                                                       float* __restrict__ delta,
                                                       float* __restrict__ dq_acc, int BH, int N,
-                                                      int N_pad) {
+                                                      int N_pad, int d_io_arg) {
+  const int d_io = (D == 64) ? D : d_io_arg;  // padded head dims use the 128-wide kernels
   const int gw = blockIdx.x * 8 + (threadIdx.x >> 5);  // one warp per padded row
   const int lane = threadIdx.x & 31;
   if (gw >= BH * N_pad) return;
@@ -622,8 +627,8 @@ __global__ void __launch_bounds__(256) bwd_pre_kernel(const __nv_bfloat16* __res
   float4* acc = reinterpret_cast<float4*>(dq_acc + static_cast<size_t>(gw) * D);
   for (int k = lane; k < D / 4; k += 32) acc[k] = make_float4(0.f, 0.f, 0.f, 0.f);
   float sum = 0.f;
-  if (i < N) {
-    const size_t off = (static_cast<size_t>(bh) * N + i) * D + lane * PER;
+  if (i < N && lane * PER < d_io) {  // d_io is a multiple of 8, PER divides it
+    const size_t off = (static_cast<size_t>(bh) * N + i) * d_io + lane * PER;
 #pragma unroll
     for (int k = 0; k < PER; ++k) sum += __bfloat162float(o[off + k]) * __bfloat162float(dout[off + k]);
   }
@@ -638,13 +643,14 @@ __global__ void __launch_bounds__(256) bwd_pre_kernel(const __nv_bfloat16* __res
 template <int D>
 __global__ void __launch_bounds__(256) bwd_post_kernel(const float* __restrict__ dq_acc,
                                                        __nv_bfloat16* __restrict__ dq, float scale,
-                                                       int BH, int N, int N_pad) {
+                                                       int BH, int N, int N_pad, int d_io_arg) {
+  const int d_io = (D == 64) ? D : d_io_arg;  // padded head dims use the 128-wide kernels
   const size_t idx = (static_cast<size_t>(blockIdx.x) * blockDim.x + threadIdx.x);  // 4 elements
-  const size_t total = static_cast<size_t>(BH) * N * D / 4;
+  const size_t total = static_cast<size_t>(BH) * N * d_io / 4;
   if (idx >= total) return;
-  const size_t e = idx * 4;
-  const size_t row = e / D;  // over BH * N
-  const int c = static_cast<int>(e % D);
+  const size_t e = idx * 4;  // element of dq [BH, N, d_io]
+  const size_t row = e / d_io;  // over BH * N
+  const int c = static_cast<int>(e % d_io);
   const size_t bh = row / N;
   const size_t i = row % N;
   const float4 v = *reinterpret_cast<const float4*>(dq_acc + (bh * N_pad + i) * D + c);
@@ -673,14 +679,14 @@ cudaError_t launch_bwd_main_t(const CUtensorMap& tq, const CUtensorMap& tk, cons
 
 }  // namespace
 
-cudaError_t launch_bwd_pre(int d, const __nv_bfloat16* o, const __nv_bfloat16* dout,
+cudaError_t launch_bwd_pre(int d, int d_io, const __nv_bfloat16* o, const __nv_bfloat16* dout,
                            const float* lse, float* lse2, float* delta, float* dq_acc, int BH,
                            int N, int N_pad, cudaStream_t s) {
   const unsigned grid = static_cast<unsigned>((static_cast<size_t>(BH) * N_pad + 7) / 8);
   if (d == 64)
-    bwd_pre_kernel<64><<<grid, 256, 0, s>>>(o, dout, lse, lse2, delta, dq_acc, BH, N, N_pad);
+    bwd_pre_kernel<64><<<grid, 256, 0, s>>>(o, dout, lse, lse2, delta, dq_acc, BH, N, N_pad, d_io);
   else
-    bwd_pre_kernel<128><<<grid, 256, 0, s>>>(o, dout, lse, lse2, delta, dq_acc, BH, N, N_pad);
+    bwd_pre_kernel<128><<<grid, 256, 0, s>>>(o, dout, lse, lse2, delta, dq_acc, BH, N, N_pad, d_io);
   return cudaGetLastError();
 }
 
@@ -691,15 +697,15 @@ cudaError_t launch_bwd_main(int d, const CUtensorMap& tq, const CUtensorMap& tk,
   return launch_bwd_main_t<128>(tq, tk, tv, tdo, tdq, p, s);
 }
 
-cudaError_t launch_bwd_post(int d, const float* dq_acc, __nv_bfloat16* dq, float scale, int BH,
-                            int N, int N_pad, cudaStream_t s) {
-  const size_t total = static_cast<size_t>(BH) * N * d / 4;
+cudaError_t launch_bwd_post(int d, int d_io, const float* dq_acc, __nv_bfloat16* dq, float scale,
+                            int BH, int N, int N_pad, cudaStream_t s) {
+  const size_t total = static_cast<size_t>(BH) * N * d_io / 4;
   const unsigned grid = static_cast<unsigned>((total + 255) / 256);
   if (total == 0) return cudaSuccess;
   if (d == 64)
-    bwd_post_kernel<64><<<grid, 256, 0, s>>>(dq_acc, dq, scale, BH, N, N_pad);
+    bwd_post_kernel<64><<<grid, 256, 0, s>>>(dq_acc, dq, scale, BH, N, N_pad, d_io);
   else
-    bwd_post_kernel<128><<<grid, 256, 0, s>>>(dq_acc, dq, scale, BH, N, N_pad);
+    bwd_post_kernel<128><<<grid, 256, 0, s>>>(dq_acc, dq, scale, BH, N, N_pad, d_io);
   return cudaGetLastError();
 }
 

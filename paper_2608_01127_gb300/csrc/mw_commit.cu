@@ -7,24 +7,24 @@
 namespace mw {
 namespace {
 
-// One thread per 16-byte piece of a row; both K and V.
-template <int D>
+// One thread per 16-byte piece of a row (d / 8 pieces, d a multiple of 8);
+// both K and V.
 __global__ void __launch_bounds__(256) commit_kernel(__nv_bfloat16* __restrict__ kc,
                                                      __nv_bfloat16* __restrict__ vc,
                                                      const __nv_bfloat16* __restrict__ ks,
                                                      const __nv_bfloat16* __restrict__ vs, int cap,
-                                                     int slot, int rows, int BH) {
-  constexpr int PIECES = D / 8;  // 16-byte pieces per row
-  // grid: x covers rows * PIECES of one head, y strides over the heads
+                                                     int slot, int rows, int BH, int d) {
+  const int pieces = d / 8;
+  // grid: x covers rows * pieces of one head, y strides over the heads
   const int idx = blockIdx.x * blockDim.x + threadIdx.x;
-  if (idx >= rows * PIECES) return;
-  const int piece = idx % PIECES;
-  const int r = idx / PIECES;
+  if (idx >= rows * pieces) return;
+  const int piece = idx % pieces;
+  const int r = idx / pieces;
   int dst = slot + r;
   if (dst >= cap) dst -= cap;  // slot < cap and rows <= cap
   for (int bh = blockIdx.y; bh < BH; bh += gridDim.y) {
-    const size_t so = (static_cast<size_t>(bh) * rows + r) * D + piece * 8;
-    const size_t dso = (static_cast<size_t>(bh) * cap + dst) * D + piece * 8;
+    const size_t so = (static_cast<size_t>(bh) * rows + r) * d + piece * 8;
+    const size_t dso = (static_cast<size_t>(bh) * cap + dst) * d + piece * 8;
     *reinterpret_cast<uint4*>(kc + dso) = *reinterpret_cast<const uint4*>(ks + so);
     *reinterpret_cast<uint4*>(vc + dso) = *reinterpret_cast<const uint4*>(vs + so);
   }
@@ -39,10 +39,7 @@ cudaError_t launch_commit(int d, __nv_bfloat16* kc, __nv_bfloat16* vc, const __n
   if (per_head == 0 || BH == 0) return cudaSuccess;
   const dim3 grid(static_cast<unsigned>((per_head + 255) / 256),
                   static_cast<unsigned>(BH < 65535 ? BH : 65535));
-  if (d == 64)
-    commit_kernel<64><<<grid, 256, 0, s>>>(kc, vc, ks, vs, cap, slot, rows, BH);
-  else
-    commit_kernel<128><<<grid, 256, 0, s>>>(kc, vc, ks, vs, cap, slot, rows, BH);
+  commit_kernel<<<grid, 256, 0, s>>>(kc, vc, ks, vs, cap, slot, rows, BH, d);
   return cudaGetLastError();
 }
 

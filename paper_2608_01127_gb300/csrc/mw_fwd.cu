@@ -517,10 +517,15 @@ __global__ void __launch_bounds__(FwdLayout<D>::THREADS, 1)
 #pragma unroll
       for (int k = 0; k < 32; ++k) v[k] = nonzero ? __uint_as_float(r[k]) * inv_l : 0.f;
       if (p.num_splits == 1) {
-        uint4* dst = reinterpret_cast<uint4*>(p.o + row_off * D + 32 * c);
+        // the caller's rows hold d_io <= D columns (multiples of 8); only the
+        // 128-wide kernel serves padded head dims
+        const int d_io = (D == 64) ? D : p.d_io;
+        if (32 * c >= d_io) continue;
+        const int n16 = min(4, (d_io - 32 * c) / 8);
+        uint4* dst = reinterpret_cast<uint4*>(p.o + row_off * d_io + 32 * c);
 #pragma unroll
         for (int k = 0; k < 4; ++k)
-          dst[k] = make_uint4(pack_bf16x2(v[8 * k], v[8 * k + 1]), pack_bf16x2(v[8 * k + 2], v[8 * k + 3]),
+          if (k < n16) dst[k] = make_uint4(pack_bf16x2(v[8 * k], v[8 * k + 1]), pack_bf16x2(v[8 * k + 2], v[8 * k + 3]),
                               pack_bf16x2(v[8 * k + 4], v[8 * k + 5]),
                               pack_bf16x2(v[8 * k + 6], v[8 * k + 7]));
       } else {
@@ -555,7 +560,8 @@ __global__ void __launch_bounds__(256) combine_kernel(const float* __restrict__ 
                                                       const float* __restrict__ lse_part,
                                                       __nv_bfloat16* __restrict__ o,
                                                       float* __restrict__ lse, int splits,
-                                                      int n_rows) {
+                                                      int n_rows, int d_io_arg) {
+  const int d_io = (D == 64) ? D : d_io_arg;  // padded head dims use the 128-wide kernels
   const int row = blockIdx.x * 8 + (threadIdx.x >> 5);
   const int lane = threadIdx.x & 31;
   if (row >= n_rows) return;
@@ -576,10 +582,11 @@ __global__ void __launch_bounds__(256) combine_kernel(const float* __restrict__ 
     for (int k = 0; k < PER; ++k) acc[k] += w * src[k];
   }
   const float inv = wsum > 0.f ? 1.f / wsum : 0.f;
-  __nv_bfloat16* dst = o + static_cast<size_t>(row) * D + lane * PER;
+  __nv_bfloat16* dst = o + static_cast<size_t>(row) * d_io + lane * PER;
 #pragma unroll
   for (int k = 0; k < PER; k += 2) {
-    *reinterpret_cast<uint32_t*>(dst + k) = pack_bf16x2(acc[k] * inv, acc[k + 1] * inv);
+    if (lane * PER + k < d_io)
+      *reinterpret_cast<uint32_t*>(dst + k) = pack_bf16x2(acc[k] * inv, acc[k + 1] * inv);
   }
   if (lse && lane == 0) lse[row] = wsum > 0.f ? m + __logf(wsum) : -INFINITY;
 }
@@ -620,14 +627,15 @@ cudaError_t launch_fwd(int d, const CUtensorMap& tq, const CUtensorMap& tk, cons
   return launch_fwd_t<128, false>(tq, tk, tv, tkr, tvr, tks, tvs, p, s);
 }
 
-cudaError_t launch_combine(int d, const float* o_part, const float* lse_part, __nv_bfloat16* o,
-                           float* lse, int splits, int BH, int rows, cudaStream_t s) {
+cudaError_t launch_combine(int d, int d_io, const float* o_part, const float* lse_part,
+                           __nv_bfloat16* o, float* lse, int splits, int BH, int rows,
+                           cudaStream_t s) {
   const int n_rows = BH * rows;
   const unsigned grid = static_cast<unsigned>((n_rows + 7) / 8);
   if (d == 64)
-    combine_kernel<64><<<grid, 256, 0, s>>>(o_part, lse_part, o, lse, splits, n_rows);
+    combine_kernel<64><<<grid, 256, 0, s>>>(o_part, lse_part, o, lse, splits, n_rows, d_io);
   else
-    combine_kernel<128><<<grid, 256, 0, s>>>(o_part, lse_part, o, lse, splits, n_rows);
+    combine_kernel<128><<<grid, 256, 0, s>>>(o_part, lse_part, o, lse, splits, n_rows, d_io);
   return cudaGetLastError();
 }
 

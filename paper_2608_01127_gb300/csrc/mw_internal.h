@@ -26,6 +26,8 @@ __host__ __device__ constexpr int bwd_q_rows(int) { return 128; }
 struct FwdParams {
   int BH;
   int rows_q;       // query rows (= rows of segment C) per (b,h)
+  int d_io;         // head dim of the caller's tensors (<= the kernel's D; the
+                    // TMA maps zero-fill the columns in between)
   int T;            // chunk length in tokens
   int n_qblocks;    // ceil(rows_q / kFwdBlockRows)
   int ring_cap;
@@ -53,6 +55,7 @@ struct BwdParams {
   int BH;
   int N;            // tokens per (b,h)
   int N_pad;        // N rounded up to kTileRows
+  int d_io;         // head dim of the caller's tensors (<= the kernel's D)
   int T;
   float scale_log2;
   float scale;
@@ -71,9 +74,11 @@ struct BwdParams {
 cudaError_t launch_fwd(int d, const CUtensorMap& tq, const CUtensorMap& tk, const CUtensorMap& tv,
                        const CUtensorMap& tkr, const CUtensorMap& tvr, const CUtensorMap& tks,
                        const CUtensorMap& tvs, const FwdParams& p, cudaStream_t s);
-cudaError_t launch_combine(int d, const float* o_part, const float* lse_part, __nv_bfloat16* o,
-                           float* lse, int splits, int BH, int rows, cudaStream_t s);
-cudaError_t launch_bwd_pre(int d, const __nv_bfloat16* o, const __nv_bfloat16* dout,
+// d: the kernels' head dim (64 or 128); d_io: the caller's (a multiple of 8, <= d)
+cudaError_t launch_combine(int d, int d_io, const float* o_part, const float* lse_part,
+                           __nv_bfloat16* o, float* lse, int splits, int BH, int rows,
+                           cudaStream_t s);
+cudaError_t launch_bwd_pre(int d, int d_io, const __nv_bfloat16* o, const __nv_bfloat16* dout,
                            const float* lse, float* lse2, float* delta, float* dq_acc, int BH,
                            int N, int N_pad, cudaStream_t s);
 // tdq: f32 map over dQacc [BH, N_pad, d] with 32 x 32 boxes (128-byte
@@ -81,8 +86,9 @@ cudaError_t launch_bwd_pre(int d, const __nv_bfloat16* o, const __nv_bfloat16* d
 cudaError_t launch_bwd_main(int d, const CUtensorMap& tq, const CUtensorMap& tk,
                             const CUtensorMap& tv, const CUtensorMap& tdo, const CUtensorMap& tdq,
                             const BwdParams& p, cudaStream_t s);
-cudaError_t launch_bwd_post(int d, const float* dq_acc, __nv_bfloat16* dq, float scale, int BH,
-                            int N, int N_pad, cudaStream_t s);
+cudaError_t launch_bwd_post(int d, int d_io, const float* dq_acc, __nv_bfloat16* dq, float scale,
+                            int BH, int N, int N_pad, cudaStream_t s);
+// d: any multiple of 8 (rows are copied in 16-byte pieces)
 cudaError_t launch_commit(int d, __nv_bfloat16* kc, __nv_bfloat16* vc, const __nv_bfloat16* ks,
                           const __nv_bfloat16* vs, int cap, int slot, int rows, int BH,
                           cudaStream_t s);

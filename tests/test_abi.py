@@ -64,7 +64,9 @@ def test_fwd_rejects_bad_arguments(mw):
     assert call(q=None) == INVALID
     assert call(o=None) == INVALID
     assert call(k=MISALIGNED) == INVALID
-    assert call(d=96) == UNSUPPORTED
+    assert call(d=100) == UNSUPPORTED   # not a multiple of 8
+    assert call(d=136) == UNSUPPORTED
+    assert call(d=56) == UNSUPPORTED
     assert call(d=0) == UNSUPPORTED
     assert call(B=0) == INVALID
     assert call(T=0) == INVALID
@@ -81,7 +83,9 @@ def test_bwd_rejects_bad_arguments_and_workspace(mw):
     need = lib.mw_bca_bwd_workspace_size(B, H, n, T, d)
     # dQ accumulator (fp32, rows padded to 128) + two fp32 row vectors, 256-byte aligned
     assert need == 2 * 256 * 64 * 4 + 2 * 256 * 4 + 2 * 256 * 4
-    assert lib.mw_bca_bwd_workspace_size(B, H, n, T, 96) == 0
+    assert lib.mw_bca_bwd_workspace_size(B, H, n, T, 100) == 0
+    # a padded head dim (72) keeps a 128-wide fp32 accumulator
+    assert lib.mw_bca_bwd_workspace_size(B, H, n, T, 72) == 2 * 256 * 128 * 4 + 2 * 256 * 4 + 2 * 256 * 4
 
     def call(ws=FAKE, ws_bytes=need, lse=FAKE, d=d):
         return lib.mw_bca_bwd(FAKE, FAKE, FAKE, FAKE, lse, FAKE, FAKE, FAKE, FAKE, ws, ws_bytes,
@@ -107,7 +111,7 @@ def test_cache_rejects_bad_ring_state(mw):
     assert call(length=-1) == INVALID
     assert call(cap=0, head=0, length=0) == INVALID
     assert call(kc=None) == INVALID
-    assert call(d=80) == UNSUPPORTED
+    assert call(d=84) == UNSUPPORTED
     assert call(T=0) == INVALID
 
 

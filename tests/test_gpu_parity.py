@@ -85,6 +85,8 @@ SMALL = [
     (1, 3, 5, 200, 64, 1.0),
     (2, 2, 1, 600, 128, 1.0),    # a single chunk: full bidirectional attention
     (1, 20, 3, 96, 128, 1.0),    # the 3B head layout (20 heads of 128)
+    (1, 2, 3, 100, 72, 1.0),     # the 0.5B head dim (72: zero-padded to 128 in the kernels)
+    (2, 1, 2, 130, 96, 2.0),     # another padded head dim
 ]
 
 
@@ -105,7 +107,8 @@ def test_small_shapes_forward_backward(mw, B, H, n, T, d, gain):
     check_grad(dv, dv_r, tag + " dV")
 
 
-@pytest.mark.parametrize("name", ["train_b12_d64", "train_h16_d128_peaky", "train_1b_32x600"])
+@pytest.mark.parametrize("name", ["train_b12_d64", "train_h16_d128_peaky", "train_1b_32x600",
+                                  "train_05b_d72"])
 def test_full_size_training_configs(mw, name):
     """Full-size launch; the oracle recomputes two sampled (b, h) heads in full."""
     cfg = TRAIN_CONFIGS[name]
@@ -179,6 +182,7 @@ CACHE_SMALL = [
     (1, 2, 4, 96, 1152, 1152, 576, 64, 5),     # forced split-KV
     (1, 2, 2, 130, 780, 780, 390, 128, 1),     # forced single pass
     (1, 1, 1, 16, 48, 40, 30, 64, 3),          # tiny ring, more splits than needed
+    (1, 2, 2, 64, 640, 640, 320, 72, 3),       # padded head dim with split-KV
 ]
 
 
@@ -234,8 +238,9 @@ def test_ring_rotation_matches(mw):
         check_lse(lse, lse_ref, f"rotation {r}")
 
 
-def test_commit_is_bit_exact(mw):
-    B, H, d, cap, rows = 2, 3, 128, 1000, 300
+@pytest.mark.parametrize("d", [128, 72])
+def test_commit_is_bit_exact(mw, d):
+    B, H, cap, rows = 2, 3, 1000, 300
     g = torch.Generator().manual_seed(3)
     kr, vr, ks, vs = (torch.randn(B, H, n, d, generator=g).to(torch.bfloat16)
                       for n in (cap, cap, rows, rows))
@@ -345,6 +350,7 @@ ROPE_SMALL = [
     (1, 2, 2, 100, 1000, 300, 900, 32, 64, 64, 7, 0, 0),     # every channel, many frames per tile
     (1, 1, 1, 880, 1760, 1760, 1759, 440, 128, 16, 440, 1, 3),  # one-frame sink, frames of 440
     (2, 1, 2, 64, 640, 640, 0, 0, 64, 2, 1, 5, 0),           # one token per frame
+    (1, 2, 1, 64, 512, 512, 200, 16, 72, 24, 64, 1, 2),     # padded head dim, sink, splits
 ]
 
 

@@ -96,6 +96,9 @@ TRAIN_CONFIGS: Dict[str, TrainConfig] = {
     # latent positions x 2 frames) at the MiniWorld-1B head layout (1536 / 12)
     "train_1b_32x600": TrainConfig("train_1b_32x600", B=1, H=12, d=128, n_chunks=32,
                                    T=600, seed=6),
+    # the MiniWorld-0.5B head layout (1152 / 16 = 72 channels per head)
+    "train_05b_d72": TrainConfig("train_05b_d72", B=1, H=16, d=72, n_chunks=16, T=880,
+                                 seed=7),
 }
 
 CACHE_CONFIGS: Dict[str, CacheConfig] = {
