@@ -21,8 +21,11 @@
  *     [B, H, rows, d] of bf16 (raw 16-bit bfloat16 bits; nv_bfloat16 in CUDA),
  *     16-byte aligned.  LSE arrays are fp32 [B, H, rows].  The caller owns every
  *     buffer; the library keeps no pointer after a call returns.
- *   - d must be 64 or 128 (the head dims of the paper's model table,
- *     Sec. 4.1); anything else returns MW_ERR_UNSUPPORTED.
+ *   - d is a multiple of 8 from 64 to 128.  The kernels are built for 64
+ *     and 128 (the head dims of most of the paper's model table, Sec. 4.1);
+ *     a head dim in between (the 0.5B layout's 72) runs on the 128-wide
+ *     kernels, whose loads fill the missing columns with zeros.  Anything
+ *     else returns MW_ERR_UNSUPPORTED.
  *   - `stream` is a cudaStream_t (NULL = legacy default stream).  Every call
  *     validates its arguments on the host, then enqueues kernels on `stream`
  *     and returns without synchronising.  Outputs are ready when the stream
@@ -49,7 +52,7 @@ extern "C" {
 typedef enum {
   MW_OK = 0,
   MW_ERR_INVALID_ARG = 1,  /* null pointer, bad size, misalignment, bad ring state */
-  MW_ERR_UNSUPPORTED = 2,  /* valid but not implemented (d not in {64,128}) */
+  MW_ERR_UNSUPPORTED = 2,  /* valid but not implemented (d outside 64..128 or not a multiple of 8) */
   MW_ERR_CUDA = 3,         /* a CUDA runtime / driver call failed */
   MW_ERR_TIMEOUT = 4,      /* a kernel's bounded wait expired (mw_device_status) */
   MW_ERR_WORKSPACE = 5     /* workspace missing or smaller than *_workspace_size() */
