@@ -39,8 +39,13 @@ struct FwdLayout {
   static constexpr int OW = SUM_MMA ? D + 16 : D;     // O columns in TMEM
   static constexpr int OFF_ONES = OFF_V + STAGES * TILE_BYTES;
   static constexpr int ONES_BYTES = SUM_MMA ? REGION_BYTES : 0;
-  static constexpr int OFF_ROPE = OFF_ONES + ONES_BYTES;   // per-pair RoPE frequencies
-  static constexpr int ROPE_BYTES = D / 2 * 4;
+  // RoPE re-shift: per-pair frequencies, then (cos, sin) per (frame, pair) for
+  // up to ROPE_FRAMES frames of the tile being rotated
+  // (one copy per rotating warp)
+  static constexpr int ROPE_FRAMES = 4;
+  static constexpr int OFF_ROPE = OFF_ONES + ONES_BYTES;
+  static constexpr int ROPE_WARP_BYTES = D / 2 * 4 + ROPE_FRAMES * (D / 2) * 8;
+  static constexpr int ROPE_BYTES = 2 * ROPE_WARP_BYTES;
   static constexpr int OFF_BAR = OFF_ROPE + ROPE_BYTES;
   static constexpr int NBAR = 1 + 5 * STAGES + 3 * QT + 1;
   static constexpr int OFF_MISC = OFF_BAR + NBAR * 8;
@@ -335,41 +340,98 @@ __global__ void __launch_bounds__(FwdLayout<D>::THREADS, 1)
     // order) is rotated to frame first_frame + t / per_frame here, in shared
     // memory, between the TMA copy and the MMAs that read the tile.  Channel
     // pair (2i, 2i+1), i < rope_dims / 2, turns by frame * base^(-2i/rope_dims).
-    const int tid = threadIdx.x - 320;  // 0..63
-    float* omega = reinterpret_cast<float*>(smem + L::OFF_ROPE);
+    // Each of the two warps turns its own half of every ring tile (rows
+    // [64 h, 64 h + 64)), so they never wait for each other.
+    const int half = warp - 10;
+    float* omega = reinterpret_cast<float*>(smem + L::OFF_ROPE + half * L::ROPE_WARP_BYTES);
+    float2* table = reinterpret_cast<float2*>(omega + D / 2);  // [ROPE_FRAMES][4 n_ch]
     const int pairs = p.rope_dims / 2;
-    for (int i = tid; i < pairs; i += 64)
+    for (int i = lane; i < pairs; i += 32)
       omega[i] = exp2f(-(2.f * i / p.rope_dims) * p.rope_log2_base);
-    asm volatile("barrier.cta.sync 1, 64;" ::: "memory");
+    __syncwarp();
+    // lane -> (row within a pass, 16-byte chunk of 8 channels = 4 pairs)
+    const int n_ch = (pairs + 3) / 4;
+    const int rpp = 32 / n_ch;
+    const int my_r = lane / n_ch, my_ch = lane % n_ch;
+    const bool active = my_r < rpp;
+    const int c0 = 8 * my_ch;
+    const int np = min(4, pairs - 4 * my_ch);        // pairs of the chunk that turn
+    const int region_off = (c0 >> 6) * L::REGION_BYTES;
+    const int cidx = (c0 & 63) >> 3;                 // chunk index within the 128-byte row
     const float inv_2pi = 0.15915494309189535f;
     const float two_pi = 6.283185307179586f;
+    auto angle_cs = [&](int f, int pi) {  // (cos, sin) of f * omega_pi
+      float th = static_cast<float>(f) * omega[pi];
+      th = fmaf(-two_pi, rintf(th * inv_2pi), th);
+      float sn, cs;
+      __sincosf(th, &sn, &cs);
+      return make_float2(cs, sn);
+    };
+    auto turn = [](uint32_t w, float2 csn) {  // bf16 pair (x0, x1) -> rotated pair
+      const float x0 = __uint_as_float(w << 16), x1 = __uint_as_float(w & 0xffff0000u);
+      // (x0 c - x1 s, x0 s + x1 c) as two packed operations
+      const float2 y = fma2(make_float2(-x1, x1), make_float2(csn.y, csn.x),
+                            mul2(make_float2(x0, x0), csn));
+      return pack_bf16x2(y.x, y.y);
+    };
     for (int i = 0; i < n_local; ++i) {
       const int st = i % NS;
       if (!warp_wait(&k_full[st], (i / NS) & 1, ctl)) break;
       const TileSrc src = tile_src(g, j0 + i);
-      if (src.seg == kSegRing) {
-        uint8_t* tile = sK + st * L::TILE_BYTES;
+      const int r_lo = 64 * half;
+      const int nrows = min(64, src.end - src.row0 - r_lo);  // valid rows of this half
+      if (src.seg == kSegRing && nrows > 0) {
+        uint8_t* tile = sK + st * L::TILE_BYTES + region_off;
+        const int t_lo = src.t0 + r_lo;
+        const int f_lo = p.rope_first_frame + t_lo / p.rope_per_frame;
+        const int nf = p.rope_first_frame + (t_lo + nrows - 1) / p.rope_per_frame - f_lo + 1;
+        const bool tabled = nf <= L::ROPE_FRAMES;
+        if (tabled) {  // (cos, sin) once per frame and pair; rows of 4 n_ch pairs (32-byte aligned)
+          for (int e = lane; e < nf * pairs; e += 32)
+            table[(e / pairs) * (4 * n_ch) + e % pairs] = angle_cs(f_lo + e / pairs, e % pairs);
+          __syncwarp();
+        }
+        if (active && tabled) {
+          // rows before the first frame boundary use table row 0, the next
+          // per_frame rows row 1, ... (no division per row)
+          const int b0 = (f_lo + 1 - p.rope_first_frame) * p.rope_per_frame - t_lo;
+          const int P = p.rope_per_frame;
+          const int pi0 = 4 * my_ch;
+#pragma unroll 2
+          for (int rr = my_r; rr < nrows; rr += rpp) {
+            const int r = r_lo + rr;
+            const int fi = (rr >= b0) + (rr >= b0 + P) + (rr >= b0 + 2 * P);
+            const float4* cs = reinterpret_cast<const float4*>(table + fi * (4 * n_ch) + pi0);
+            // 128-byte swizzle: 16-byte chunk index ^ (row mod 8)
+            uint4* a = reinterpret_cast<uint4*>(tile + r * 128 + ((cidx ^ (r & 7)) << 4));
+            uint4 v = *a;
+            const float4 c01 = cs[0];
+            v.x = turn(v.x, make_float2(c01.x, c01.y));
+            if (np > 1) v.y = turn(v.y, make_float2(c01.z, c01.w));
+            if (np > 2) {
+              const float4 c23 = cs[1];
+              v.z = turn(v.z, make_float2(c23.x, c23.y));
+              if (np > 3) v.w = turn(v.w, make_float2(c23.z, c23.w));
+            }
+            *a = v;
+          }
+        } else if (active) {  // many frames in one tile (short frames): angles per row
 #pragma unroll 1
-        for (int rr = 0; rr < 2; ++rr) {
-          const int r = 2 * tid + rr;
-          if (src.row0 + r >= src.end) continue;  // rows past the ring's valid end
-          const float f = static_cast<float>(p.rope_first_frame + (src.t0 + r) / p.rope_per_frame);
-#pragma unroll 1
-          for (int pi = 0; pi < pairs; ++pi) {
-            const int c = 2 * pi;  // 128-byte swizzle: 16-byte chunk index ^ (row mod 8)
-            uint32_t* a = reinterpret_cast<uint32_t*>(
-                tile + (c >> 6) * L::REGION_BYTES + r * 128 +
-                (((((c & 63) * 2) >> 4) ^ (r & 7)) << 4) + ((c * 2) & 15));
-            float th = f * omega[pi];
-            th = fmaf(-two_pi, rintf(th * inv_2pi), th);
-            float sn, cs;
-            __sincosf(th, &sn, &cs);
-            const uint32_t v = *a;
-            const float x0 = __uint_as_float(v << 16), x1 = __uint_as_float(v & 0xffff0000u);
-            *a = pack_bf16x2(x0 * cs - x1 * sn, x0 * sn + x1 * cs);
+          for (int rr = my_r; rr < nrows; rr += rpp) {
+            const int r = r_lo + rr;
+            const int f = p.rope_first_frame + (t_lo + rr) / p.rope_per_frame;
+            const int pi0 = 4 * my_ch;
+            uint4* a = reinterpret_cast<uint4*>(tile + r * 128 + ((cidx ^ (r & 7)) << 4));
+            uint4 v = *a;
+            v.x = turn(v.x, angle_cs(f, pi0));
+            if (np > 1) v.y = turn(v.y, angle_cs(f, pi0 + 1));
+            if (np > 2) v.z = turn(v.z, angle_cs(f, pi0 + 2));
+            if (np > 3) v.w = turn(v.w, angle_cs(f, pi0 + 3));
+            *a = v;
           }
         }
         fence_proxy_async_smem();  // the tensor core reads the tile next
+        __syncwarp();              // every lane is done with the table
       }
       __syncwarp();
       if (lane == 0) mbar_arrive(&k_rdy[st]);
