@@ -549,6 +549,26 @@ def bench_rolling(mw, dev, peaks):
                    "replayed as one CUDA graph. The ring (57.7 MB) stays L2-resident across "
                    "steps, as in streaming"}
     res.update(_cache_roofline(cfg, g_us, peaks))
+    # the same stream with the ring's RoPE re-shift fused into its read (32
+    # rotated channels, 440 tokens per frame; the ring holds unrotated keys)
+    def step_rope(s):
+        h, ln, slot = plan[s]
+        mw.mw_bca_cache_fwd_rope(qs[s], ks[s], vs[s], None, None, kr, vr, h, ln, cfg.T, 32,
+                                 10000.0, 440, 0, cfg.scale, need_lse=False, workspace=ws, out=o)
+        mw.mw_bca_cache_commit(kr, vr, slot, ks[s], vs[s])
+
+    for s in range(3):
+        step_rope(s)
+    torch.cuda.synchronize()
+    evs = []
+    for s in range(cfg.steps):
+        e = Events()
+        e.start()
+        step_rope(s)
+        e.stop()
+        evs.append(e)
+    torch.cuda.synchronize()
+    res["rope_reshift_us_per_step_median"] = round(statistics.median(e.ms() * 1e3 for e in evs), 2)
     return res
 
 
