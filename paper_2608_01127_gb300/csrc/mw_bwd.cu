@@ -608,7 +608,9 @@ __global__ void __launch_bounds__(BwdLayout<D>::THREADS, 1)
 }
 
 // D_i = <dO_i, O_i>, LSE2_i = LSE_i log2(e) for i < N; padding rows get
-// D = 0, LSE2 = +inf (so their P is exactly 0).  Also zeroes dQacc.
+// D = 0, LSE2 = +inf (so their P is exactly 0).  Also zeroes dQacc.  A group
+// of D / 8 lanes covers one row with 16-byte loads and stores (4 rows per
+// warp at d = 64, 2 at d = 128).
 template <int D>
 __global__ void __launch_bounds__(256) bwd_pre_kernel(const __nv_bfloat16* __restrict__ o,
                                                       const __nv_bfloat16* __restrict__ dout,
@@ -618,25 +620,36 @@ __global__ void __launch_bounds__(256) bwd_pre_kernel(const __nv_bfloat16* __res
                                                       float* __restrict__ dq_acc, int BH, int N,
                                                       int N_pad, int d_io_arg) {
   const int d_io = (D == 64) ? D : d_io_arg;  // padded head dims use the 128-wide kernels
-  const int gw = blockIdx.x * 8 + (threadIdx.x >> 5);  // one warp per padded row
+  constexpr int G = D / 8;                     // lanes per row (8 bf16 = 16 bytes each)
   const int lane = threadIdx.x & 31;
-  if (gw >= BH * N_pad) return;
-  const int bh = gw / N_pad;
-  const int i = gw % N_pad;
-  constexpr int PER = D / 32;
-  float4* acc = reinterpret_cast<float4*>(dq_acc + static_cast<size_t>(gw) * D);
-  for (int k = lane; k < D / 4; k += 32) acc[k] = make_float4(0.f, 0.f, 0.f, 0.f);
-  float sum = 0.f;
-  if (i < N && lane * PER < d_io) {  // d_io is a multiple of 8, PER divides it
-    const size_t off = (static_cast<size_t>(bh) * N + i) * d_io + lane * PER;
+  const long long gr = (static_cast<long long>(blockIdx.x) * blockDim.x + threadIdx.x) / G;  // padded row
+  const int sub = lane % G;
+  // (the grid covers whole rows; lanes past the end stay for the shuffles)
+  const bool valid = gr < static_cast<long long>(BH) * N_pad;
+  const int bh = static_cast<int>(gr / N_pad);
+  const int i = static_cast<int>(gr % N_pad);
+  if (valid) {  // dQacc row: D fp32 = 2 D / 8 float4 stores, G lanes
+    float4* acc = reinterpret_cast<float4*>(dq_acc + gr * D);
 #pragma unroll
-    for (int k = 0; k < PER; ++k) sum += __bfloat162float(o[off + k]) * __bfloat162float(dout[off + k]);
+    for (int k = 0; k < 2; ++k) acc[sub + k * G] = make_float4(0.f, 0.f, 0.f, 0.f);
+  }
+  float sum = 0.f;
+  if (valid && i < N && 8 * sub < d_io) {  // d_io is a multiple of 8
+    const size_t off = (static_cast<size_t>(bh) * N + i) * d_io + 8 * sub;
+    const uint4 a = *reinterpret_cast<const uint4*>(o + off);
+    const uint4 b = *reinterpret_cast<const uint4*>(dout + off);
+    const uint32_t av[4] = {a.x, a.y, a.z, a.w}, bv[4] = {b.x, b.y, b.z, b.w};
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+      sum = fmaf(__uint_as_float(av[k] << 16), __uint_as_float(bv[k] << 16), sum);
+      sum = fmaf(__uint_as_float(av[k] & 0xffff0000u), __uint_as_float(bv[k] & 0xffff0000u), sum);
+    }
   }
 #pragma unroll
-  for (int s = 16; s > 0; s >>= 1) sum += __shfl_xor_sync(0xffffffffu, sum, s);
-  if (lane == 0) {
-    delta[gw] = sum;
-    lse2[gw] = (i < N) ? lse[static_cast<size_t>(bh) * N + i] * 1.4426950408889634f : INFINITY;
+  for (int s = G / 2; s > 0; s >>= 1) sum += __shfl_xor_sync(0xffffffffu, sum, s);
+  if (valid && sub == 0) {
+    delta[gr] = sum;
+    lse2[gr] = (i < N) ? lse[static_cast<size_t>(bh) * N + i] * 1.4426950408889634f : INFINITY;
   }
 }
 
@@ -682,7 +695,8 @@ cudaError_t launch_bwd_main_t(const CUtensorMap& tq, const CUtensorMap& tk, cons
 cudaError_t launch_bwd_pre(int d, int d_io, const __nv_bfloat16* o, const __nv_bfloat16* dout,
                            const float* lse, float* lse2, float* delta, float* dq_acc, int BH,
                            int N, int N_pad, cudaStream_t s) {
-  const unsigned grid = static_cast<unsigned>((static_cast<size_t>(BH) * N_pad + 7) / 8);
+  const size_t threads = static_cast<size_t>(BH) * N_pad * (d / 8);  // d / 8 lanes per row
+  const unsigned grid = static_cast<unsigned>((threads + 255) / 256);
   if (d == 64)
     bwd_pre_kernel<64><<<grid, 256, 0, s>>>(o, dout, lse, lse2, delta, dq_acc, BH, N, N_pad, d_io);
   else
