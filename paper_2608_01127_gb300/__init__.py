@@ -134,17 +134,24 @@ def _scale(scale: Optional[float], d: int) -> float:
 
 
 def mw_bca_fwd(q: torch.Tensor, k: torch.Tensor, v: torch.Tensor, T_chunk: int,
-               scale: Optional[float] = None, need_lse: bool = True
+               scale: Optional[float] = None, need_lse: bool = True,
+               out: Optional[Tuple[torch.Tensor, Optional[torch.Tensor]]] = None
                ) -> Tuple[torch.Tensor, Optional[torch.Tensor]]:
-    """Block-causal attention forward (Sec. 3.2); returns (O, LSE or None)."""
+    """Block-causal attention forward (Sec. 3.2); returns (O, LSE or None).
+
+    ``out`` = (o, lse) reuses caller buffers (lse may be None)."""
     B, H, N, d = _bhnd(q, "q")
     for t, n in ((k, "k"), (v, "v")):
         if _bhnd(t, n) != (B, H, N, d):
             raise ValueError(f"{n} shape {tuple(t.shape)} != q shape {(B, H, N, d)}")
     if N % T_chunk != 0:
         raise ValueError(f"sequence length {N} is not a multiple of T_chunk={T_chunk}")
-    o = torch.empty_like(q)
-    lse = torch.empty((B, H, N), dtype=torch.float32, device=q.device) if need_lse else None
+    if out is not None:
+        o, lse = out
+        _bhnd(o, "o")
+    else:
+        o = torch.empty_like(q)
+        lse = torch.empty((B, H, N), dtype=torch.float32, device=q.device) if need_lse else None
     _check(library().mw_bca_fwd(_ptr(q), _ptr(k), _ptr(v), _ptr(o), _ptr(lse), B, H,
                                 N // T_chunk, T_chunk, d, _scale(scale, d), _stream()))
     return o, lse
