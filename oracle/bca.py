@@ -213,6 +213,26 @@ def fwd_rows(q: torch.Tensor, k: torch.Tensor, v: torch.Tensor, T: int,
     return torch.stack(outs), torch.stack(lses)
 
 
+def dq_rows(q: torch.Tensor, k: torch.Tensor, v: torch.Tensor, do: torch.Tensor, T: int,
+            scale: float, rows: Sequence[int]) -> torch.Tensor:
+    """dQ of selected query rows of one head (Q,K,V,dO [N,d]), row by row.
+
+    Row i needs only its own visible scores: P_i = exp(s_i - LSE_i),
+    O_i = P_i V, D_i = <dO_i, O_i>, dS_ij = P_ij (<dO_i, v_j> - D_i),
+    dQ_i = scale * sum_j dS_ij k_j.
+    """
+    q, k, v, do = q.to(F64), k.to(F64), v.to(F64), do.to(F64)
+    out = []
+    for i in rows:
+        end = (chunk_of(i, T) + 1) * T
+        s = scale * (k[:end] @ q[i])
+        p = torch.exp(s - _row_lse(s.unsqueeze(0))[0])
+        o_i = p @ v[:end]
+        ds = p * (v[:end] @ do[i] - do[i] @ o_i)
+        out.append(scale * (ds @ k[:end]))
+    return torch.stack(out)
+
+
 # --------------------------------------------------------------------------
 # rolling KV cache (Sec. 3.5): ring of committed chunks + in-flight chunks
 # --------------------------------------------------------------------------

@@ -76,6 +76,15 @@ mw_status check_rows(long long rows, const char* what) {
   return MW_OK;
 }
 
+// B*H*rows (plus padding to whole tiles) bounds every grid and element index
+// the launches derive: keep it within 2^31 tokens.
+mw_status check_tokens(long long BH, long long rows) {
+  const long long padded = (rows + 255) / 256 * 256;
+  if (BH * padded > (1ll << 31))
+    return fail(MW_ERR_INVALID_ARG, "B*H*rows=%lld exceeds 2^31 tokens", BH * rows);
+  return MW_OK;
+}
+
 #define MW_TRY(expr)                 \
   do {                               \
     mw_status _s = (expr);           \
@@ -377,6 +386,7 @@ mw_status mw_bca_fwd(const void* q, const void* k, const void* v, void* o, float
     return fail(MW_ERR_INVALID_ARG, "n_chunks=%d and T_chunk=%d must be >= 1", n_chunks, T_chunk);
   const long long N = static_cast<long long>(n_chunks) * T_chunk;
   MW_TRY(check_rows(N, "n_chunks*T_chunk"));
+  MW_TRY(check_tokens(static_cast<long long>(B) * H, N));
   if (!(scale > 0.f)) return fail(MW_ERR_INVALID_ARG, "scale must be > 0");
   MW_TRY(check_ptr(q, "q"));
   MW_TRY(check_ptr(k, "k"));
@@ -409,6 +419,7 @@ mw_status mw_bca_bwd_stage(int stage, const void* q, const void* k, const void* 
     return fail(MW_ERR_INVALID_ARG, "n_chunks=%d and T_chunk=%d must be >= 1", n_chunks, T_chunk);
   const long long N = static_cast<long long>(n_chunks) * T_chunk;
   MW_TRY(check_rows(N, "n_chunks*T_chunk"));
+  MW_TRY(check_tokens(static_cast<long long>(B) * H, N));
   if (!(scale > 0.f)) return fail(MW_ERR_INVALID_ARG, "scale must be > 0");
   if (main) {
     MW_TRY(check_ptr(q, "q"));
@@ -528,6 +539,7 @@ mw_status mw_bca_cache_fwd_rope(const void* q, const void* k_new, const void* v_
     return fail(MW_ERR_INVALID_ARG, "n_q_chunks=%d and T_chunk=%d must be >= 1", n_q_chunks, T_chunk);
   const long long rows = static_cast<long long>(n_q_chunks) * T_chunk;
   MW_TRY(check_rows(rows, "n_q_chunks*T_chunk"));
+  MW_TRY(check_tokens(static_cast<long long>(B) * H, rows));
   if (cache_cap < 1 || cache_cap > (1 << 24))
     return fail(MW_ERR_INVALID_ARG, "cache_cap=%d out of range [1, 2^24]", cache_cap);
   if (cache_head < 0 || cache_head >= cache_cap)
@@ -678,6 +690,7 @@ extern "C" mw_status mw_bca_cache_fwd_noalloc(const void* q, const void* k_new, 
     return fail(MW_ERR_INVALID_ARG, "n_q_chunks=%d and T_chunk=%d must be >= 1", n_q_chunks, T_chunk);
   const long long rows = static_cast<long long>(n_q_chunks) * T_chunk;
   MW_TRY(check_rows(rows, "n_q_chunks*T_chunk"));
+  MW_TRY(check_tokens(static_cast<long long>(B) * H, rows));
   if (cache_len < 0 || cache_len > cache_cap)
     return fail(MW_ERR_INVALID_ARG, "cache_len=%d not in [0, cache_cap=%d]", cache_len, cache_cap);
   const int splits = plan_splits(B * H, static_cast<int>(rows), cache_len);

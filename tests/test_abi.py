@@ -72,6 +72,7 @@ def test_fwd_rejects_bad_arguments(mw):
     assert call(T=0) == INVALID
     assert call(n=0) == INVALID
     assert call(n=1 << 15, T=1 << 10) == INVALID   # 2^25 tokens
+    assert call(B=1 << 10, H=1 << 10, n=1, T=1 << 12) == INVALID   # 2^32 tokens over all heads
     assert call(s=0.0) == INVALID
     assert call(s=-1.0) == INVALID
     assert "scale" in lib.mw_last_error().decode()

@@ -249,6 +249,18 @@ def test_finite_differences():
         assert err < 1e-6, (which, float(err))
 
 
+def test_dq_rows_matches_the_full_backward():
+    """The row-by-row dQ (used for long sequences) equals the full backward's
+    dQ rows, itself pinned by finite differences and autograd."""
+    N, T, d = 25, 5, 6
+    q, k, v, do = (_rand(1, 1, N, d, seed=s)[0, 0] for s in (120, 121, 122, 123))
+    dq, _, _ = oracle.bwd(q.view(1, 1, N, d), k.view(1, 1, N, d), v.view(1, 1, N, d),
+                          do.view(1, 1, N, d), T, 0.7)
+    rows = [0, 3, 4, 5, 11, 19, 24]
+    got = oracle.dq_rows(q, k, v, do, T, 0.7, rows)
+    assert torch.allclose(got, dq[0, 0, rows], atol=1e-13, rtol=0)
+
+
 # ---------------------------------------------------------------- rolling cache
 
 def _cache_case(W, T, cap, length, head, d=8, seed=70, B=1, H=2):
