@@ -131,6 +131,32 @@ def test_full_size_training_configs(mw, name):
     assert mw.mw_device_status() == 0
 
 
+@pytest.mark.parametrize("d,N,T", [(64, 65536, 4096), (128, 32768, 2048)])
+def test_long_sequence_sampled_rows_and_invariants(mw, d, N, T):
+    """A long sequence (16 chunks): O, LSE and dQ on sampled rows against the
+    oracle's row-by-row forms; dK and dV through identities that hold at any
+    size: sum_j dK_j = 0 (each row of dS sums to zero) and sum_j dV_j =
+    sum_i dO_i (each row of P sums to one)."""
+    q, k, v, do = _inputs(1, 1, N // T, T, d, seed=55)
+    sc = 1.0 / math.sqrt(d)
+    qc, kc, vc, doc = (t.cuda() for t in (q, k, v, do))
+    o, lse = mw.mw_bca_fwd(qc, kc, vc, T, sc)
+    dq, dk, dv = mw.mw_bca_bwd(qc, kc, vc, o, lse, doc, T, sc)
+    torch.cuda.synchronize()
+    g = torch.Generator().manual_seed(9)
+    rows = sorted(set([0, T - 1, T, N // 2, N - T, N - 1] +
+                      torch.randint(0, N, (26,), generator=g).tolist()))
+    q1, k1, v1, do1 = (t[0, 0] for t in (q, k, v, do))
+    o_ref, lse_ref = oracle.fwd_rows(q1, k1, v1, T, sc, rows)
+    check_o(o[0, 0, rows], o_ref, f"long d{d} sampled O")
+    check_lse(lse[0, 0, rows], lse_ref, f"long d{d} sampled LSE")
+    check_grad(dq[0, 0, rows], oracle.dq_rows(q1, k1, v1, do1, T, sc, rows), f"long d{d} sampled dQ")
+    dk64, dv64 = dk[0, 0].double().cpu(), dv[0, 0].double().cpu()
+    assert float(dk64.sum(0).norm() / dk64.norm()) < 2e-2
+    sum_do = do1.double().sum(0)
+    assert float((dv64.sum(0) - sum_do).norm() / sum_do.norm()) < 2e-2
+
+
 def test_forward_is_deterministic_and_stays_in_bounds(mw):
     B, H, n, T, d = 1, 2, 3, 100, 64
     q, k, v, _ = _inputs(B, H, n, T, d, seed=7)
