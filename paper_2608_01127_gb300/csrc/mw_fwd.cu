@@ -149,6 +149,8 @@ __global__ void __launch_bounds__(FwdLayout<D>::THREADS, 1)
   const int bh = x % p.BH;
   const int qb = p.n_qblocks - 1 - x / p.BH;
   const int r0 = qb * kFwdBlockRows;
+  // query tiles of the block that hold rows (the last block may hold one)
+  const int qt_n = (r0 + kTileRows < p.rows_q) ? QT : 1;
   const int last_row = min(r0 + kFwdBlockRows - 1, p.rows_q - 1);
   const int c_end = (last_row / p.T + 1) * p.T;  // keys of segment C visible to the block
 
@@ -297,7 +299,7 @@ __global__ void __launch_bounds__(FwdLayout<D>::THREADS, 1)
         const uint32_t php = ((i - 1) / NS) & 1;
         if (!(ok = warp_wait(ROPE ? &k_rdy[st] : &k_full[st], ph, ctl))) break;
         tc_fence_after();
-        for (int t = 0; t < QT; ++t) {
+        for (int t = 0; t < qt_n; ++t) {
           if (i > 0) {
             // PV of the first 64 keys while the softmax warps store the rest of P
             if (!(ok = warp_wait(&p_half[t], (i - 1) & 1, ctl))) break;
@@ -318,7 +320,7 @@ __global__ void __launch_bounds__(FwdLayout<D>::THREADS, 1)
       if (ok) {
         const int il = n_local - 1;
         const int stl = il % NS;
-        for (int t = 0; ok && t < QT; ++t) {
+        for (int t = 0; ok && t < qt_n; ++t) {
           if (!(ok = warp_wait(&p_half[t], il & 1, ctl))) break;
           if (t == 0 && !(ok = warp_wait(&v_full[stl], (il / NS) & 1, ctl))) break;
           tc_fence_after();
@@ -454,7 +456,8 @@ __global__ void __launch_bounds__(FwdLayout<D>::THREADS, 1)
     float m_used = -INFINITY;
     float l = 0.f;
     bool ok = true;
-    for (int i = 0; i < n_local; ++i) {
+    const int n_steps = t < qt_n ? n_local : 0;  // an empty query tile does nothing
+    for (int i = 0; i < n_steps; ++i) {
       const TileSrc src = tile_src(g, j0 + i);
       if (!(ok = warp_wait(&s_full[t], i & 1, ctl))) break;
       tc_fence_after();
@@ -552,7 +555,7 @@ __global__ void __launch_bounds__(FwdLayout<D>::THREADS, 1)
     }
 
     // ---- epilogue
-    const bool have = __all_sync(0xffffffffu, ok) && n_local > 0 && warp_wait(o_full, 0, ctl);
+    const bool have = __all_sync(0xffffffffu, ok) && n_steps > 0 && warp_wait(o_full, 0, ctl);
     tc_fence_after();
     if constexpr (L::SUM_MMA) {
       if (have) {
