@@ -85,6 +85,17 @@ struct BwdLayout {
   static constexpr uint32_t PDS_COL = SHARED_X ? S_COL : 384u;
   static constexpr uint32_t DQ_COL = SHARED_X ? 384u : 448u;
   static constexpr int THREADS = 512;
+  // registers per thread after the re-split: the P/dS warpgroups get more
+  // (at d = 64, room to prefetch the step's LSE and D rows), the drain
+  // warpgroup and the control warpgroup (TMA, MMA) less; the three shares
+  // add up to exactly the launch's 512 threads x 128 registers
+  static constexpr bool PREFETCH = (D == 64);
+  static constexpr int REGS_LAUNCH = 128;
+  static constexpr int REGS_PDS = (D == 64) ? 176 : 152;
+  static constexpr int REGS_DRAIN = (D == 64) ? 80 : 104;
+  static constexpr int REGS_CONTROL = (D == 64) ? 80 : 104;
+  static_assert(256 * REGS_PDS + 128 * REGS_DRAIN + 128 * REGS_CONTROL == THREADS * REGS_LAUNCH,
+                "register re-split must hand out exactly the launch's registers");
   static_assert(SHARED_X ? (2 * D + QN <= 384) : (2 * D + 2 * QN <= 384), "TMEM columns");
   static_assert(BYTES <= 232448, "shared memory");
 };
@@ -184,6 +195,9 @@ __global__ void __launch_bounds__(BwdLayout<D>::THREADS, 1)
   float* sLSE = reinterpret_cast<float*>(smem + L::OFF_LSE);
   float* sDelta = reinterpret_cast<float*>(smem + L::OFF_DELTA);
 
+  if (warp >= 12) {
+  // warpgroup 3 (TMA, MMA issuers, one idle warp): one re-split for all four
+  regs_dec<L::REGS_CONTROL>();
   if (warp == 12) {
     // ------------------------------------------------------------ TMA producer
     if (lane == 0) {
@@ -361,7 +375,9 @@ __global__ void __launch_bounds__(BwdLayout<D>::THREADS, 1)
       }
       if (ok) umma_commit(dkv_full);  // one arrival per issuing warp
     }
+  }
   } else if (warp < 8) {
+    regs_inc<L::REGS_PDS>();
     // ------------------------------------------------------------ P / dS (thread = key row)
     const int wg = warp >> 2;            // query columns [CW wg, CW wg + CW)
     const int wq = warp & 3;             // TMEM lane quadrant
@@ -390,6 +406,18 @@ __global__ void __launch_bounds__(BwdLayout<D>::THREADS, 1)
       const float* delta = sDelta + st * QN + c0;
       if (!(ok = warp_wait(s_full, j & 1, ctl))) break;
       tc_fence_after();
+      // the step's LSE row (16 bytes per load); at d = 64 read while S^T comes
+      // out of TMEM
+      float2 nl[CW / 2];
+      auto load_lse = [&]() {
+#pragma unroll
+        for (int c = 0; c < CW / 4; ++c) {
+          const float4 v = reinterpret_cast<const float4*>(lse2)[c];
+          nl[2 * c] = make_float2(-v.x, -v.y);
+          nl[2 * c + 1] = make_float2(-v.z, -v.w);
+        }
+      };
+      if constexpr (L::PREFETCH) load_lse();
       float pr[CW];
       {
         uint32_t r[CW / 32][32];
@@ -405,14 +433,7 @@ __global__ void __launch_bounds__(BwdLayout<D>::THREADS, 1)
       __syncwarp();
       if (lane == 0) mbar_arrive(s_free);
       const int lim = q_start - q0 - c0;  // columns c < lim are masked
-      // row vectors of this step from shared memory, 16 bytes per load
-      float2 nl[CW / 2];
-#pragma unroll
-      for (int c = 0; c < CW / 4; ++c) {
-        const float4 v = reinterpret_cast<const float4*>(lse2)[c];
-        nl[2 * c] = make_float2(-v.x, -v.y);
-        nl[2 * c + 1] = make_float2(-v.z, -v.w);
-      }
+      if constexpr (!L::PREFETCH) load_lse();
       const float2 sl2x2 = make_float2(sl2, sl2);
 #pragma unroll
       for (int c = 0; c < CW / 2; ++c) {
@@ -447,6 +468,12 @@ __global__ void __launch_bounds__(BwdLayout<D>::THREADS, 1)
         }
         store_pt();
       }
+      // the step's D row (d = 64: read before dP^T is ready)
+      float4 dvv[L::PREFETCH ? CW / 4 : 1];
+      if constexpr (L::PREFETCH) {
+#pragma unroll
+        for (int c = 0; c < CW / 4; ++c) dvv[c] = reinterpret_cast<const float4*>(delta)[c];
+      }
       if (!(ok = warp_wait(dp_full, j & 1, ctl))) break;
       tc_fence_after();
 #pragma unroll
@@ -462,7 +489,8 @@ __global__ void __launch_bounds__(BwdLayout<D>::THREADS, 1)
         }
 #pragma unroll
         for (int k = 0; k < 8; ++k) {
-          const float4 dv = reinterpret_cast<const float4*>(delta)[8 * h + k];
+          const float4 dv = L::PREFETCH ? dvv[L::PREFETCH ? 8 * h + k : 0]
+                                        : reinterpret_cast<const float4*>(delta)[8 * h + k];
           const int c = 32 * h + 4 * k;
           // dS = P (dP - D), two columns per instruction
           const float2 t0 = add2(make_float2(__uint_as_float(r[4 * k]), __uint_as_float(r[4 * k + 1])),
@@ -531,7 +559,8 @@ __global__ void __launch_bounds__(BwdLayout<D>::THREADS, 1)
         }
       }
     }
-  } else if (warp < 12) {
+  } else {
+    regs_dec<L::REGS_DRAIN>();
     // ------------------------------------------------------------ dQ drain
     const int wq = warp & 3;
     const uint32_t lane_base = tmem + (static_cast<uint32_t>(wq * 32) << 16);
@@ -596,6 +625,7 @@ __global__ void __launch_bounds__(BwdLayout<D>::THREADS, 1)
       if (lane == 0) bulk_wait_all();
       __syncwarp();
     }
+
   }
 
   __syncwarp();
@@ -680,6 +710,12 @@ cudaError_t launch_bwd_main_t(const CUtensorMap& tq, const CUtensorMap& tk, cons
   using L = BwdLayout<D>;
   static bool attr_set = false;
   if (!attr_set) {
+    // The in-kernel register re-split assumes the launch register count; with
+    // any other count its setmaxnreg.inc could never be satisfied, so refuse.
+    cudaFuncAttributes fa;
+    cudaError_t e0 = cudaFuncGetAttributes(&fa, bca_bwd_kernel<D>);
+    if (e0 != cudaSuccess) return e0;
+    if (fa.numRegs != L::REGS_LAUNCH) return cudaErrorInvalidKernelImage;
     cudaError_t e = cudaFuncSetAttribute(bca_bwd_kernel<D>,
                                          cudaFuncAttributeMaxDynamicSharedMemorySize, L::BYTES);
     if (e != cudaSuccess) return e;
