@@ -643,15 +643,26 @@ __global__ void __launch_bounds__(256) combine_kernel(const float* __restrict__ 
     const float w = __expf(ls - m);
     wsum += w;
     const float* src = o_part + (static_cast<size_t>(s) * n_rows + row) * D + lane * PER;
-#pragma unroll
-    for (int k = 0; k < PER; ++k) acc[k] += w * src[k];
+    if constexpr (PER == 4) {  // one 16-byte load per lane
+      const float4 x = *reinterpret_cast<const float4*>(src);
+      acc[0] += w * x.x;
+      acc[1] += w * x.y;
+      acc[2] += w * x.z;
+      acc[3] += w * x.w;
+    } else {  // PER == 2: one 8-byte load per lane
+      const float2 x = *reinterpret_cast<const float2*>(src);
+      acc[0] += w * x.x;
+      acc[1] += w * x.y;
+    }
   }
   const float inv = wsum > 0.f ? 1.f / wsum : 0.f;
   __nv_bfloat16* dst = o + static_cast<size_t>(row) * d_io + lane * PER;
-#pragma unroll
-  for (int k = 0; k < PER; k += 2) {
-    if (lane * PER + k < d_io)
-      *reinterpret_cast<uint32_t*>(dst + k) = pack_bf16x2(acc[k] * inv, acc[k + 1] * inv);
+  if (lane * PER < d_io) {  // d_io is a multiple of 8, so a lane's PER columns are all in range
+    if constexpr (PER == 4)
+      *reinterpret_cast<uint2*>(dst) = make_uint2(pack_bf16x2(acc[0] * inv, acc[1] * inv),
+                                                  pack_bf16x2(acc[2] * inv, acc[3] * inv));
+    else
+      *reinterpret_cast<uint32_t*>(dst) = pack_bf16x2(acc[0] * inv, acc[1] * inv);
   }
   if (lse && lane == 0) lse[row] = wsum > 0.f ? m + __logf(wsum) : -INFINITY;
 }
