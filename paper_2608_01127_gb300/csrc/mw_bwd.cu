@@ -468,14 +468,15 @@ __global__ void __launch_bounds__(BwdLayout<D>::THREADS, 1)
         }
         store_pt();
       }
-      // the step's D row (d = 64: read before dP^T is ready)
+      if (!(ok = warp_wait(dp_full, j & 1, ctl))) break;
+      tc_fence_after();
+      // the step's D row came with dO, which dP^T_j has read; d = 64: all of
+      // it is requested before the TMEM loads, so the two latencies overlap
       float4 dvv[L::PREFETCH ? CW / 4 : 1];
       if constexpr (L::PREFETCH) {
 #pragma unroll
         for (int c = 0; c < CW / 4; ++c) dvv[c] = reinterpret_cast<const float4*>(delta)[c];
       }
-      if (!(ok = warp_wait(dp_full, j & 1, ctl))) break;
-      tc_fence_after();
 #pragma unroll
       for (int h = 0; h < CW / 32; ++h) {
         uint32_t r[32];
