@@ -529,7 +529,29 @@ def run_extras(mw, dev, peaks):
     extra["rolling_cache"] = bench_rolling(mw, dev, peaks)
     extra["pipelined"] = bench_pipelined(mw, dev, peaks, flush)
     extra["sink_anchor"] = bench_sink(mw, dev, peaks, flush)
+    extra["qkv_rope_split"] = bench_qkv_split(mw, dev, peaks, flush)
     return extra
+
+
+def bench_qkv_split(mw, dev, peaks, flush):
+    """The QKV split with the temporal RoPE of Q and K at the d=64 training
+    layout (B2 H12, 16 x 880 tokens, 32 rotated channels, 440 tokens per
+    frame): HBM-bound, every element read and written once."""
+    cfg = TRAIN_CONFIGS["train_b12_d64"]
+    N = cfg.n_chunks * cfg.T
+    g = torch.Generator(device=dev).manual_seed(21)
+    qkv = torch.randn(cfg.B, N, 3, cfg.H, cfg.d, generator=g, device=dev).to(torch.bfloat16)
+    out = tuple(torch.empty(cfg.B, cfg.H, N, cfg.d, dtype=torch.bfloat16, device=dev)
+                for _ in range(3))
+    ts = time_repeated(lambda: mw.mw_qkv_rope_split(qkv, 32, 10000.0, 440, 0, out=out), 20,
+                       flush=flush)
+    med = statistics.median(ts) * 1e3
+    nbytes = 2 * qkv.numel() * qkv.element_size()
+    gbs = nbytes / (med / 1e6) / 1e9
+    return {"us_median": round(med, 2), "l2": "flushed between runs",
+            "bytes_algorithmic": nbytes, "gbs_algorithmic": round(gbs, 1),
+            "frac_hbm": round(gbs / peaks["hbm_gbs"], 4), "rope_dims": 32,
+            "tokens_per_frame": 440}
 
 
 def _cache_roofline(cfg, us, peaks):

@@ -176,7 +176,8 @@ mw_status mw_bca_cache_fwd_sink(const void* q, const void* k_new, const void* v_
  *                      mw_bca_cache_fwd_sink)
  *   rope_base        : > 1
  *   tokens_per_frame : >= 1
- *   first_frame      : 0 <= first_frame <= 2^24
+ *   first_frame      : >= 0, and first_frame + (cache_len - 1) / tokens_per_frame
+ *                      <= 2^24 (the angle reduction is exact up to there)
  * Every other argument is as for mw_bca_cache_fwd_sink.
  */
 mw_status mw_bca_cache_fwd_rope(const void* q, const void* k_new, const void* v_new,
@@ -200,6 +201,37 @@ mw_status mw_bca_cache_fwd_rope(const void* q, const void* k_new, const void* v_
 mw_status mw_bca_cache_commit(void* k_cache, void* v_cache, int cache_cap, int slot_start,
                               const void* k_src, const void* v_src, int rows, int B, int H, int d,
                               void* stream);
+
+/*
+ * QKV split with temporal RoPE (the input side of the attention: Sec. 3.2
+ * runs block-causal attention over the latent tokens; Sec. 3.5 gives keys
+ * temporal positions that the rolling cache re-shifts).  The fused QKV
+ * projection leaves each token's heads interleaved; this writes them
+ * head-major for the attention calls and rotates Q and K on the way:
+ *   qkv     : [B, N, 3, H, d] bf16 (index 0 = Q, 1 = K, 2 = V), read only
+ *   q, k, v : [B, H, N, d] bf16 outputs, written whole; must not overlap qkv
+ * Token t sits at frame first_frame + t / tokens_per_frame; channel pair
+ * (2i, 2i+1), 0 <= i < rope_dims / 2, of its query and key turns by
+ *     frame * rope_base^(-2i / rope_dims):  (x, y) -> (x cos - y sin, x sin + y cos)
+ * computed in fp32 and rounded to bf16 (V and the other channels are copied
+ * bit for bit).  mw_bca_cache_fwd_rope turns ring keys on read with the same
+ * arithmetic, so a key turned here to frame f equals an un-rotated ring key
+ * turned there to frame f.  rope_dims = 0 is a plain split (rope_base,
+ * tokens_per_frame and first_frame are then ignored).
+ *   d                : a multiple of 8 from 64 to 128
+ *   1 <= N <= 2^24, B * H * N <= 2^31
+ *   rope_dims        : even, 0 <= rope_dims <= d
+ *   rope_base        : > 1 (the frequencies base^(-2i/rope_dims) of this float
+ *                      value are formed in fp64, and the angles reduced so
+ *                      that they stay exact to ~1e-6 rad at every frame)
+ *   tokens_per_frame : >= 1
+ *   first_frame      : >= 0, and first_frame + (N - 1) / tokens_per_frame <= 2^24
+ * Errors: MW_ERR_INVALID_ARG (NULL or misaligned pointer, bad sizes),
+ * MW_ERR_UNSUPPORTED (d), MW_ERR_CUDA (launch).  Asynchronous on `stream`.
+ */
+mw_status mw_qkv_rope_split(const void* qkv, void* q, void* k, void* v, int B, int N, int H,
+                            int d, int rope_dims, float rope_base, int tokens_per_frame,
+                            int first_frame, void* stream);
 
 /* Size of the library's static scratch array used by
  * mw_bca_cache_fwd_noalloc (64 MiB on every device that loads the library). */

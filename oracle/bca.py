@@ -267,6 +267,24 @@ def rope_rotate(x: torch.Tensor, frames: torch.Tensor, rope_dims: int,
     return x
 
 
+def qkv_split_rope(qkv: torch.Tensor, rope_dims: int = 0, base: float = 10000.0,
+                   tokens_per_frame: int = 1, first_frame: int = 0
+                   ) -> Tuple[torch.Tensor, torch.Tensor, torch.Tensor]:
+    """Head-major Q, K, V [B, H, N, d] (fp64) from a fused QKV projection
+    ``qkv`` [B, N, 3, H, d] (index 0 = Q, 1 = K, 2 = V along dim 2).
+
+    Token t sits at frame first_frame + t // tokens_per_frame; Q and K are
+    turned by ``rope_rotate`` at those frames (the temporal positions of
+    Sec. 3.5), V is moved unchanged.
+    """
+    x = qkv.to(F64).permute(2, 0, 3, 1, 4)  # [3, B, H, N, d]
+    N = qkv.shape[1]
+    frames = first_frame + torch.arange(N) // tokens_per_frame
+    q = rope_rotate(x[0], frames, rope_dims, base)
+    k = rope_rotate(x[1], frames, rope_dims, base)
+    return q, k, x[2].clone()
+
+
 def cache_fwd(q: torch.Tensor, k_new: torch.Tensor, v_new: torch.Tensor,
               k_ring: torch.Tensor, v_ring: torch.Tensor, cap: int, head: int,
               length: int, T: int, scale: float, k_sink: torch.Tensor = None,

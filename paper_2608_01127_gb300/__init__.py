@@ -30,7 +30,8 @@ __all__ = [
     "MWError", "library", "lib_path", "mw_bca_fwd", "mw_bca_bwd", "mw_bca_cache_fwd",
     "mw_bca_cache_fwd_sink", "mw_bca_cache_fwd_rope",
     "mw_bca_cache_commit", "mw_bca_bwd_workspace_size", "mw_bca_cache_workspace_size",
-    "mw_device_status", "mw_set_option", "BlockCausalAttention", "EXPORTED_SYMBOLS",
+    "mw_device_status", "mw_set_option", "mw_qkv_rope_split", "BlockCausalAttention",
+    "EXPORTED_SYMBOLS",
     "RingState",
 ]
 
@@ -42,7 +43,7 @@ EXPORTED_SYMBOLS = (
     "mw_bca_cache_workspace_size",
     "mw_bca_cache_fwd", "mw_bca_cache_commit", "mw_status_string", "mw_last_error",
     "mw_device_status", "mw_set_option", "mw_bca_cache_fwd_noalloc", "mw_bca_cache_fwd_sink",
-    "mw_bca_cache_fwd_rope",
+    "mw_bca_cache_fwd_rope", "mw_qkv_rope_split",
 )
 
 STATUS = {0: "MW_OK", 1: "MW_ERR_INVALID_ARG", 2: "MW_ERR_UNSUPPORTED", 3: "MW_ERR_CUDA",
@@ -90,6 +91,7 @@ def library() -> ctypes.CDLL:
         "mw_bca_cache_fwd_rope": (_I, [_P, _P, _P, _P, _P, _I, _P, _P, _I, _I, _I, _I, _F, _I, _I,
                                        _P, _P, _P, _Z, _I, _I, _I, _I, _I, _F, _P]),
         "mw_bca_cache_commit": (_I, [_P, _P, _I, _I, _P, _P, _I, _I, _I, _I, _P]),
+        "mw_qkv_rope_split": (_I, [_P, _P, _P, _P, _I, _I, _I, _I, _I, _F, _I, _I, _P]),
         "mw_bca_cache_fwd_noalloc": (_I, [_P, _P, _P, _P, _P, _I, _I, _I, _P, _P,
                                           _I, _I, _I, _I, _I, _F, _P]),
         "mw_status_string": (ctypes.c_char_p, [_I]),
@@ -281,6 +283,34 @@ def mw_bca_cache_commit(k_cache, v_cache, slot_start: int, k_src, v_src) -> None
         raise ValueError("k_src / v_src must be [B, H, rows, d] matching the cache")
     _check(library().mw_bca_cache_commit(_ptr(k_cache), _ptr(v_cache), cap, slot_start,
                                          _ptr(k_src), _ptr(v_src), rows, B, H, d, _stream()))
+
+
+def mw_qkv_rope_split(qkv: torch.Tensor, rope_dims: int = 0, rope_base: float = 10000.0,
+                      tokens_per_frame: int = 1, first_frame: int = 0,
+                      out: Optional[Tuple[torch.Tensor, torch.Tensor, torch.Tensor]] = None
+                      ) -> Tuple[torch.Tensor, torch.Tensor, torch.Tensor]:
+    """Split a fused QKV projection [B, N, 3, H, d] into head-major Q, K, V
+    [B, H, N, d], turning the first ``rope_dims`` channels of Q and K by their
+    frame's temporal rotary angle (token t at frame first_frame + t //
+    tokens_per_frame; Sec. 3.2 inputs, Sec. 3.5 positions)."""
+    if qkv.dtype != torch.bfloat16:
+        raise TypeError(f"qkv must be bfloat16, got {qkv.dtype}")
+    if not qkv.is_cuda:
+        raise ValueError("qkv must be a CUDA tensor (there is no CPU path)")
+    if qkv.dim() != 5 or qkv.shape[2] != 3 or not qkv.is_contiguous():
+        raise ValueError("qkv must be a contiguous [B, N, 3, H, d] tensor")
+    B, N, _, H, d = qkv.shape
+    if out is None:
+        out = tuple(torch.empty(B, H, N, d, dtype=torch.bfloat16, device=qkv.device)
+                    for _ in range(3))
+    for t, name in zip(out, ("q", "k", "v")):
+        if tuple(_bhnd(t, name)) != (B, H, N, d):
+            raise ValueError(f"{name} must be [B, H, N, d] = {(B, H, N, d)}")
+    q, k, v = out
+    _check(library().mw_qkv_rope_split(_ptr(qkv), _ptr(q), _ptr(k), _ptr(v), B, N, H, d,
+                                       int(rope_dims), float(rope_base), int(tokens_per_frame),
+                                       int(first_frame), _stream()))
+    return q, k, v
 
 
 def mw_device_status(clear: bool = True) -> int:

@@ -23,7 +23,7 @@ BUILD_DIR = os.path.join(PKG, "_build")
 LIB_DIR = os.path.join(PKG, "_lib")
 LIB_PATH = os.path.join(LIB_DIR, "libmw_bca.so")
 
-SOURCES = ["mw_abi.cu", "mw_fwd.cu", "mw_bwd.cu", "mw_commit.cu"]
+SOURCES = ["mw_abi.cu", "mw_fwd.cu", "mw_bwd.cu", "mw_commit.cu", "mw_qkv.cu"]
 HEADERS = ["mw_ptx.cuh", "mw_internal.h"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 CFLAGS = ["-O3", "-std=c++17", "-lineinfo", "-Xcompiler", "-fPIC", "-Xcompiler", "-Wall",

@@ -274,10 +274,21 @@ mw_status launch_status(cudaError_t e, const char* what) {
 
 struct RopeArgs {
   int dims = 0;          // 0: off
-  float log2_base = 0.f;
+  mw::RopeFreq omega{};
   int per_frame = 1;
   int first_frame = 0;
 };
+
+// omega_i = base^(-2i / dims) in fp64, split into float hi + lo
+mw::RopeFreq rope_freq(int dims, float base) {
+  mw::RopeFreq f{};
+  for (int i = 0; i < dims / 2 && i < mw::kMaxRopePairs; ++i) {
+    const double w = std::pow(static_cast<double>(base), -2.0 * i / dims);
+    f.hi[i] = static_cast<float>(w);
+    f.lo[i] = static_cast<float>(w - static_cast<double>(f.hi[i]));
+  }
+  return f;
+}
 
 mw_status fwd_common(const void* q, const void* k, const void* v, const void* kr, const void* vr,
                      int cap, int head, int len, const void* ks, const void* vs, int sink_len,
@@ -317,7 +328,6 @@ mw_status fwd_common(const void* q, const void* k, const void* v, const void* kr
   p.ring_len = len;
   p.sink_len = sink_len;
   p.rope_dims = len > 0 ? rope.dims : 0;
-  p.rope_log2_base = rope.log2_base;
   p.rope_per_frame = rope.per_frame;
   p.rope_first_frame = rope.first_frame;
   p.num_splits = splits;
@@ -336,7 +346,8 @@ mw_status fwd_common(const void* q, const void* k, const void* v, const void* kr
     p.lse_part = reinterpret_cast<float*>(
         base + align256(static_cast<size_t>(p.num_splits) * BH * rows_q * D * sizeof(float)));
   }
-  MW_TRY(launch_status(mw::launch_fwd(D, tq, tk, tv, tkr, tvr, tks, tvs, p, stream), "forward kernel launch"));
+  MW_TRY(launch_status(mw::launch_fwd(D, tq, tk, tv, tkr, tvr, tks, tvs, p, rope.omega, stream),
+                       "forward kernel launch"));
   if (p.num_splits > 1)
     MW_TRY(launch_status(mw::launch_combine(D, d, p.o_part, p.lse_part, p.o, lse, p.num_splits, BH,
                                             rows_q, stream),
@@ -557,10 +568,13 @@ mw_status mw_bca_cache_fwd_rope(const void* q, const void* k_new, const void* v_
       return fail(MW_ERR_INVALID_ARG, "rope_base must be > 1 and finite");
     if (tokens_per_frame < 1)
       return fail(MW_ERR_INVALID_ARG, "tokens_per_frame=%d must be >= 1", tokens_per_frame);
-    if (first_frame < 0 || first_frame > (1 << 24))
-      return fail(MW_ERR_INVALID_ARG, "first_frame=%d out of range [0, 2^24]", first_frame);
+    if (first_frame < 0 ||
+        static_cast<long long>(first_frame) + (cache_len > 0 ? (cache_len - 1) / tokens_per_frame : 0) >
+            (1 << 24))
+      return fail(MW_ERR_INVALID_ARG,
+                  "first_frame=%d: ring frame positions must stay in [0, 2^24]", first_frame);
     rope.dims = rope_dims;
-    rope.log2_base = std::log2(rope_base);
+    rope.omega = rope_freq(rope_dims, rope_base);
     rope.per_frame = tokens_per_frame;
     rope.first_frame = first_frame;
   }
@@ -616,6 +630,40 @@ mw_status mw_bca_cache_commit(void* k_cache, void* v_cache, int cache_cap, int s
                         static_cast<const __nv_bfloat16*>(v_src), cache_cap, slot_start, rows,
                         B * H, static_cast<cudaStream_t>(stream)),
       "commit kernel launch");
+}
+
+mw_status mw_qkv_rope_split(const void* qkv, void* q, void* k, void* v, int B, int N, int H,
+                            int d, int rope_dims, float rope_base, int tokens_per_frame,
+                            int first_frame, void* stream) {
+  MW_TRY(check_dims(B, H, d));
+  MW_TRY(check_rows(N, "N"));
+  MW_TRY(check_tokens(static_cast<long long>(B) * H, N));
+  mw::RopeFreq omega{};
+  if (rope_dims != 0) {
+    if (rope_dims < 0 || rope_dims > d || (rope_dims & 1))
+      return fail(MW_ERR_INVALID_ARG, "rope_dims=%d must be even and in [0, d=%d]", rope_dims, d);
+    if (!(rope_base > 1.f) || !(rope_base < 1e30f))
+      return fail(MW_ERR_INVALID_ARG, "rope_base must be > 1 and finite");
+    if (tokens_per_frame < 1)
+      return fail(MW_ERR_INVALID_ARG, "tokens_per_frame=%d must be >= 1", tokens_per_frame);
+    if (first_frame < 0 ||
+        static_cast<long long>(first_frame) + (N - 1) / tokens_per_frame > (1 << 24))
+      return fail(MW_ERR_INVALID_ARG,
+                  "first_frame=%d: frame positions must stay in [0, 2^24]", first_frame);
+    omega = rope_freq(rope_dims, rope_base);
+  }
+  MW_TRY(check_ptr(qkv, "qkv"));
+  MW_TRY(check_ptr(q, "q"));
+  MW_TRY(check_ptr(k, "k"));
+  MW_TRY(check_ptr(v, "v"));
+  DeviceScope scope(static_cast<cudaStream_t>(stream));
+  MW_TRY(scope.status());
+  return launch_status(
+      mw::launch_qkv_rope(static_cast<const __nv_bfloat16*>(qkv), static_cast<__nv_bfloat16*>(q),
+                          static_cast<__nv_bfloat16*>(k), static_cast<__nv_bfloat16*>(v), B, N, H,
+                          d, rope_dims, omega, rope_dims != 0 ? tokens_per_frame : 1,
+                          rope_dims != 0 ? first_frame : 0, static_cast<cudaStream_t>(stream)),
+      "qkv split kernel launch");
 }
 
 mw_status mw_device_status(void* stream, int clear) {

@@ -44,7 +44,7 @@ struct FwdLayout {
   // (one copy per rotating warp)
   static constexpr int ROPE_FRAMES = 4;
   static constexpr int OFF_ROPE = OFF_ONES + ONES_BYTES;
-  static constexpr int ROPE_WARP_BYTES = D / 2 * 4 + ROPE_FRAMES * (D / 2) * 8;
+  static constexpr int ROPE_WARP_BYTES = 2 * (D / 2) * 4 + ROPE_FRAMES * (D / 2) * 8;
   static constexpr int ROPE_BYTES = 2 * ROPE_WARP_BYTES;
   static constexpr int OFF_BAR = OFF_ROPE + ROPE_BYTES;
   static constexpr int NBAR = 1 + 5 * STAGES + 3 * QT + 1;
@@ -116,7 +116,8 @@ __global__ void __launch_bounds__(FwdLayout<D>::THREADS, 1)
     bca_fwd_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_k,
                    const __grid_constant__ CUtensorMap tm_v, const __grid_constant__ CUtensorMap tm_kr,
                    const __grid_constant__ CUtensorMap tm_vr, const __grid_constant__ CUtensorMap tm_ks,
-                   const __grid_constant__ CUtensorMap tm_vs, const FwdParams p) {
+                   const __grid_constant__ CUtensorMap tm_vs, const FwdParams p,
+                   const __grid_constant__ RopeFreq rope_om) {
   using L = FwdLayout<D>;
   constexpr int QT = L::QT;
   constexpr int NS = L::STAGES;
@@ -346,10 +347,13 @@ __global__ void __launch_bounds__(FwdLayout<D>::THREADS, 1)
     // [64 h, 64 h + 64)), so they never wait for each other.
     const int half = warp - 10;
     float* omega = reinterpret_cast<float*>(smem + L::OFF_ROPE + half * L::ROPE_WARP_BYTES);
-    float2* table = reinterpret_cast<float2*>(omega + D / 2);  // [ROPE_FRAMES][4 n_ch]
+    float* omega_lo = omega + D / 2;
+    float2* table = reinterpret_cast<float2*>(omega + D);  // [ROPE_FRAMES][4 n_ch]
     const int pairs = p.rope_dims / 2;
-    for (int i = lane; i < pairs; i += 32)
-      omega[i] = exp2f(-(2.f * i / p.rope_dims) * p.rope_log2_base);
+    for (int i = lane; i < pairs; i += 32) {
+      omega[i] = rope_om.hi[i];
+      omega_lo[i] = rope_om.lo[i];
+    }
     __syncwarp();
     // lane -> (row within a pass, 16-byte chunk of 8 channels = 4 pairs)
     const int n_ch = (pairs + 3) / 4;
@@ -360,22 +364,8 @@ __global__ void __launch_bounds__(FwdLayout<D>::THREADS, 1)
     const int np = min(4, pairs - 4 * my_ch);        // pairs of the chunk that turn
     const int region_off = (c0 >> 6) * L::REGION_BYTES;
     const int cidx = (c0 & 63) >> 3;                 // chunk index within the 128-byte row
-    const float inv_2pi = 0.15915494309189535f;
-    const float two_pi = 6.283185307179586f;
-    auto angle_cs = [&](int f, int pi) {  // (cos, sin) of f * omega_pi
-      float th = static_cast<float>(f) * omega[pi];
-      th = fmaf(-two_pi, rintf(th * inv_2pi), th);
-      float sn, cs;
-      __sincosf(th, &sn, &cs);
-      return make_float2(cs, sn);
-    };
-    auto turn = [](uint32_t w, float2 csn) {  // bf16 pair (x0, x1) -> rotated pair
-      const float x0 = __uint_as_float(w << 16), x1 = __uint_as_float(w & 0xffff0000u);
-      // (x0 c - x1 s, x0 s + x1 c) as two packed operations
-      const float2 y = fma2(make_float2(-x1, x1), make_float2(csn.y, csn.x),
-                            mul2(make_float2(x0, x0), csn));
-      return pack_bf16x2(y.x, y.y);
-    };
+    auto angle_cs = [&](int f, int pi) { return rope_cos_sin(f, omega[pi], omega_lo[pi]); };
+    auto turn = [](uint32_t w, float2 csn) { return rope_turn(w, csn); };
     for (int i = 0; i < n_local; ++i) {
       const int st = i % NS;
       if (!warp_wait(&k_full[st], (i / NS) & 1, ctl)) break;
@@ -670,7 +660,8 @@ __global__ void __launch_bounds__(256) combine_kernel(const float* __restrict__ 
 template <int D, bool ROPE>
 cudaError_t launch_fwd_t(const CUtensorMap& tq, const CUtensorMap& tk, const CUtensorMap& tv,
                          const CUtensorMap& tkr, const CUtensorMap& tvr, const CUtensorMap& tks,
-                         const CUtensorMap& tvs, const FwdParams& p, cudaStream_t s) {
+                         const CUtensorMap& tvs, const FwdParams& p, const RopeFreq& om,
+                         cudaStream_t s) {
   using L = FwdLayout<D>;
   static bool attr_set = false;  // per process; the attribute is per function
   if (!attr_set) {
@@ -686,7 +677,8 @@ cudaError_t launch_fwd_t(const CUtensorMap& tq, const CUtensorMap& tk, const CUt
     attr_set = true;
   }
   const unsigned grid = static_cast<unsigned>(p.BH) * p.n_qblocks * p.num_splits;
-  bca_fwd_kernel<D, ROPE><<<grid, L::THREADS, L::BYTES, s>>>(tq, tk, tv, tkr, tvr, tks, tvs, p);
+  bca_fwd_kernel<D, ROPE><<<grid, L::THREADS, L::BYTES, s>>>(tq, tk, tv, tkr, tvr, tks, tvs, p,
+                                                              om);
   return cudaGetLastError();
 }
 
@@ -694,13 +686,14 @@ cudaError_t launch_fwd_t(const CUtensorMap& tq, const CUtensorMap& tk, const CUt
 
 cudaError_t launch_fwd(int d, const CUtensorMap& tq, const CUtensorMap& tk, const CUtensorMap& tv,
                        const CUtensorMap& tkr, const CUtensorMap& tvr, const CUtensorMap& tks,
-                       const CUtensorMap& tvs, const FwdParams& p, cudaStream_t s) {
+                       const CUtensorMap& tvs, const FwdParams& p, const RopeFreq& om,
+                       cudaStream_t s) {
   if (p.rope_dims > 0) {
-    if (d == 64) return launch_fwd_t<64, true>(tq, tk, tv, tkr, tvr, tks, tvs, p, s);
-    return launch_fwd_t<128, true>(tq, tk, tv, tkr, tvr, tks, tvs, p, s);
+    if (d == 64) return launch_fwd_t<64, true>(tq, tk, tv, tkr, tvr, tks, tvs, p, om, s);
+    return launch_fwd_t<128, true>(tq, tk, tv, tkr, tvr, tks, tvs, p, om, s);
   }
-  if (d == 64) return launch_fwd_t<64, false>(tq, tk, tv, tkr, tvr, tks, tvs, p, s);
-  return launch_fwd_t<128, false>(tq, tk, tv, tkr, tvr, tks, tvs, p, s);
+  if (d == 64) return launch_fwd_t<64, false>(tq, tk, tv, tkr, tvr, tks, tvs, p, om, s);
+  return launch_fwd_t<128, false>(tq, tk, tv, tkr, tvr, tks, tvs, p, om, s);
 }
 
 cudaError_t launch_combine(int d, int d_io, const float* o_part, const float* lse_part,

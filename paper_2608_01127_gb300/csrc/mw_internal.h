@@ -23,6 +23,15 @@ __host__ __device__ constexpr int bwd_q_rows(int) { return 128; }
 //   B: ring rows [0, lenB)                  (the part after the wrap)
 //   C: the queries' own rows [0, rows_q)    (chunk-causal: key < (chunk(i)+1) T)
 // Training uses C only (ring_len = 0).
+// RoPE frequencies omega_i = base^(-2i / rope_dims), i < rope_dims / 2,
+// computed in fp64 on the host and handed over as two floats (hi + lo), so
+// that frame * omega keeps its low bits for frames up to 2^24.
+constexpr int kMaxRopePairs = 64;  // head dims up to 128
+struct RopeFreq {
+  float hi[kMaxRopePairs];
+  float lo[kMaxRopePairs];
+};
+
 struct FwdParams {
   int BH;
   int rows_q;       // query rows (= rows of segment C) per (b,h)
@@ -35,9 +44,9 @@ struct FwdParams {
   int ring_len;
   int sink_len;     // tokens of the sink anchor, visited before the ring
   // RoPE re-shift of ring keys on read (0 rope_dims: off): ring token t turns
-  // to frame rope_first_frame + t / rope_per_frame
+  // to frame rope_first_frame + t / rope_per_frame (the frequencies are a
+  // kernel parameter of their own)
   int rope_dims;
-  float rope_log2_base;
   int rope_per_frame;
   int rope_first_frame;
   int num_splits;   // 1: write bf16 O + LSE; >1: fp32 partials for the combine
@@ -73,7 +82,8 @@ struct BwdParams {
 // the segment is empty)
 cudaError_t launch_fwd(int d, const CUtensorMap& tq, const CUtensorMap& tk, const CUtensorMap& tv,
                        const CUtensorMap& tkr, const CUtensorMap& tvr, const CUtensorMap& tks,
-                       const CUtensorMap& tvs, const FwdParams& p, cudaStream_t s);
+                       const CUtensorMap& tvs, const FwdParams& p, const RopeFreq& rope_om,
+                       cudaStream_t s);
 // d: the kernels' head dim (64 or 128); d_io: the caller's (a multiple of 8, <= d)
 cudaError_t launch_combine(int d, int d_io, const float* o_part, const float* lse_part,
                            __nv_bfloat16* o, float* lse, int splits, int BH, int rows,
@@ -92,5 +102,11 @@ cudaError_t launch_bwd_post(int d, int d_io, const float* dq_acc, __nv_bfloat16*
 cudaError_t launch_commit(int d, __nv_bfloat16* kc, __nv_bfloat16* vc, const __nv_bfloat16* ks,
                           const __nv_bfloat16* vs, int cap, int slot, int rows, int BH,
                           cudaStream_t s);
+// QKV split + temporal RoPE: qkv [B, N, 3, H, d] -> q, k, v [B, H, N, d]
+// (d a multiple of 8; rope_dims = 0 is a plain split)
+cudaError_t launch_qkv_rope(const __nv_bfloat16* qkv, __nv_bfloat16* q, __nv_bfloat16* k,
+                            __nv_bfloat16* v, int B, int N, int H, int d, int rope_dims,
+                            const RopeFreq& omega, int per_frame, int first_frame,
+                            cudaStream_t s);
 
 }  // namespace mw

@@ -387,4 +387,35 @@ __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
   return *reinterpret_cast<uint32_t*>(&v);
 }
 
+// Temporal RoPE (a channel pair turned by an angle): the (cos, sin) of
+// f * omega for an integer frame 0 <= f <= 2^24 and omega = om_hi + om_lo.
+// The angle is reduced to about [-pi, pi] before the fast sine and cosine:
+// the FMA yields the exact rounding error of f * om_hi (Dekker's product),
+// and 2 pi is subtracted in two parts (Cody and Waite), the first of which
+// cancels exactly, so the reduced angle stays within ~1e-6 rad however
+// large f * omega is.
+__device__ __forceinline__ float2 rope_cos_sin(int f, float om_hi, float om_lo) {
+  const float two_pi_hi = 6.28318548202514648f;    // 2 pi rounded to float
+  const float two_pi_lo = -1.74845553146951e-07f;  // 2 pi - two_pi_hi
+  const float ff = static_cast<float>(f);           // exact up to 2^24
+  const float th = ff * om_hi;
+  const float err = fmaf(ff, om_hi, -th);           // f * om_hi - th, exactly
+  const float k = rintf(th * 0.15915494309189535f);
+  float r = fmaf(-k, two_pi_hi, th);
+  r = fmaf(-k, two_pi_lo, r);
+  r += fmaf(ff, om_lo, err);
+  float sn, cs;
+  __sincosf(r, &sn, &cs);
+  return make_float2(cs, sn);
+}
+
+// The bf16 pair (x0, x1) in one 32-bit word (x0 in the low half) turned by
+// the angle whose (cos, sin) is csn: (x0 c - x1 s, x0 s + x1 c), rounded to
+// bf16 (two packed operations).
+__device__ __forceinline__ uint32_t rope_turn(uint32_t w, float2 csn) {
+  const float x0 = __uint_as_float(w << 16), x1 = __uint_as_float(w & 0xffff0000u);
+  const float2 y = fma2(make_float2(-x1, x1), make_float2(csn.y, csn.x), mul2(make_float2(x0, x0), csn));
+  return pack_bf16x2(y.x, y.y);
+}
+
 }  // namespace mw

@@ -146,6 +146,7 @@ def test_rope_entry_rejects_bad_rope(mw):
     assert call(base=float("nan")) == INVALID
     assert call(per_frame=0) == INVALID
     assert call(first=-1) == INVALID
+    assert call(first=(1 << 24) - 1, per_frame=440) == INVALID  # ring frames past 2^24
 
 
 def test_commit_rejects_bad_slots(mw):
@@ -160,6 +161,29 @@ def test_commit_rejects_bad_slots(mw):
     assert call(rows=101) == INVALID
     assert call(src=None) == INVALID
     assert call(src=MISALIGNED) == INVALID
+
+
+def test_qkv_split_rejects_bad_arguments(mw):
+    lib = mw.library()
+
+    def call(qkv=FAKE, q=FAKE, B=2, N=100, H=3, d=64, dims=32, base=1e4, per_frame=7, first=0):
+        return lib.mw_qkv_rope_split(qkv, q, FAKE, FAKE, B, N, H, d, dims, base, per_frame,
+                                     first, None)
+
+    assert call(qkv=None) == INVALID
+    assert call(qkv=MISALIGNED) == INVALID
+    assert call(q=MISALIGNED) == INVALID
+    assert call(N=0) == INVALID
+    assert call(B=0) == INVALID
+    assert call(N=1 << 24, B=200) == INVALID        # more than 2^31 tokens
+    assert call(d=100) == UNSUPPORTED
+    assert call(d=136) == UNSUPPORTED
+    assert call(dims=33) == INVALID                 # odd
+    assert call(dims=66) == INVALID                 # more than d
+    assert call(base=0.5) == INVALID
+    assert call(per_frame=0) == INVALID
+    assert call(first=-1) == INVALID
+    assert call(first=(1 << 24) - 10, per_frame=1) == INVALID  # frame positions past 2^24
 
 
 def test_options(mw):

@@ -277,6 +277,76 @@ def test_commit_is_bit_exact(mw, d):
         assert torch.equal(kg.cpu(), k_ref) and torch.equal(vg.cpu(), v_ref)
 
 
+def _check_qkv(qkv, rope_dims, base, per_frame, first, got):
+    """Rotated channels of Q and K within one bf16 ulp of the fp64 oracle (the
+    kernel turns them in fp32 and rounds once, so near a rounding tie it may
+    land on the other neighbour) plus 2^-16 absolute (the fast sine and cosine
+    are good to about 2^-21 on the reduced angle, which matters where x cos
+    and y sin nearly cancel), and nearly all of them rounded exactly like the
+    oracle; everything else, and all of V, bit for bit."""
+    ref = oracle.qkv_split_rope(qkv, rope_dims, base, per_frame, first)
+    for name, g, r in zip("QKV", got, ref):
+        g = g.cpu()
+        rot = rope_dims if name != "V" else 0
+        assert torch.equal(g[..., rot:].double(), r[..., rot:]), f"{name} unrotated channels"
+        if rot:
+            gr, rr = g[..., :rot].double(), r[..., :rot]
+            err = (gr - rr).abs()
+            assert bool((err <= rr.abs() * 2.0 ** -7 + 2.0 ** -16).all()), \
+                f"{name} max err {float(err.max()):.3e}"
+            same = float((g[..., :rot] == rr.to(torch.bfloat16)).double().mean())
+            assert same >= 0.99, f"{name}: only {same:.4f} of rotated values round like the oracle"
+
+
+@pytest.mark.parametrize("B,N,H,d,rope_dims,base,per_frame,first", [
+    (2, 100, 3, 64, 32, 1e4, 7, 3),          # ragged token block, several frames per block
+    (1, 77, 2, 72, 20, 500.0, 1, 0),         # d = 72; rope_dims ends inside a 16-byte piece
+    (1, 64, 4, 128, 128, 1e4, 440, 1000),    # every channel turns
+    (1, 50, 2, 64, 0, 1e4, 1, 0),            # plain split
+    (1, 40, 1, 64, 64, 1e4, 1, (1 << 24) - 39),  # the largest positions
+])
+def test_qkv_split_rope(mw, B, N, H, d, rope_dims, base, per_frame, first):
+    g = torch.Generator().manual_seed(17)
+    qkv = torch.randn(B, N, 3, H, d, generator=g).to(torch.bfloat16)
+    got = mw.mw_qkv_rope_split(qkv.cuda(), rope_dims, base, per_frame, first)
+    torch.cuda.synchronize()
+    _check_qkv(qkv, rope_dims, base, per_frame, first, got)
+    assert mw.mw_device_status() == 0
+
+
+def test_qkv_split_rope_training_shape(mw):
+    """The d=64 training layout (B2 H12, 16 chunks of 880 tokens, 440 tokens
+    per latent frame, 32 rotated channels): V everywhere, Q and K on two token
+    ranges that start on frame boundaries (the oracle restarts there)."""
+    B, N, H, d, P = 2, 16 * 880, 12, 64, 440
+    g = torch.Generator().manual_seed(18)
+    qkv = torch.randn(B, N, 3, H, d, generator=g).to(torch.bfloat16)
+    q, k, v = mw.mw_qkv_rope_split(qkv.cuda(), 32, 1e4, P, 0)
+    torch.cuda.synchronize()
+    assert torch.equal(v.cpu(), qkv[:, :, 2].permute(0, 2, 1, 3))
+    for t0, n in ((0, 1000), (N - 2 * P, 2 * P)):
+        sl = slice(t0, t0 + n)
+        part = tuple(x[:, :, sl] for x in (q, k, v))
+        _check_qkv(qkv[:, sl].contiguous(), 32, 1e4, P, t0 // P, part)
+
+
+def test_qkv_split_rope_matches_the_fused_ring_rotation(mw):
+    """Keys turned by the split kernel and stored rotated give bit for bit the
+    same attention as un-rotated ring keys turned on read (both round the same
+    fp32 rotation to bf16; head 0 keeps the key tiles identical)."""
+    B, H, T, cap, d, P, first = 1, 2, 128, 1280, 64, 200, 5
+    g = torch.Generator().manual_seed(19)
+    q, kn, vn = (torch.randn(B, H, T, d, generator=g).to(torch.bfloat16).cuda() for _ in range(3))
+    kr, vr = (torch.randn(B, H, cap, d, generator=g).to(torch.bfloat16).cuda() for _ in range(2))
+    o1, l1 = mw.mw_bca_cache_fwd_rope(q, kn, vn, None, None, kr, vr, 0, cap, T, 32, 1e4, P, first)
+    qkv = torch.zeros(B, cap, 3, H, d, dtype=torch.bfloat16, device="cuda")
+    qkv[:, :, 1] = kr.permute(0, 2, 1, 3)
+    _, k_rot, _ = mw.mw_qkv_rope_split(qkv, 32, 1e4, P, first)
+    o2, l2 = mw.mw_bca_cache_fwd(q, kn, vn, k_rot, vr, 0, cap, T)
+    torch.cuda.synchronize()
+    assert torch.equal(o1, o2) and torch.equal(l1, l2)
+
+
 def test_rolling_cache_config_steps(mw):
     """The streaming workload: one 880-token chunk against an 8-chunk ring
     whose head wraps mid-buffer; each step commits the chunk (FIFO eviction)."""
@@ -377,6 +447,7 @@ ROPE_SMALL = [
     (1, 1, 1, 880, 1760, 1760, 1759, 440, 128, 16, 440, 1, 3),  # one-frame sink, frames of 440
     (2, 1, 2, 64, 640, 640, 0, 0, 64, 2, 1, 5, 0),           # one token per frame
     (1, 2, 1, 64, 512, 512, 200, 16, 72, 24, 64, 1, 2),     # padded head dim, sink, splits
+    (1, 2, 1, 64, 512, 512, 300, 0, 64, 64, 2, (1 << 24) - 255, 0),  # the largest frames
 ]
 
 

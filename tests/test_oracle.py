@@ -475,3 +475,53 @@ def test_product_ring_bookkeeping_matches_oracle():
             slot, h, n = oracle.ring_advance(cap, h, n, rows)
             assert ring.commit(rows) == slot
             assert (ring.head, ring.length) == (h, n)
+
+
+def test_qkv_split_moves_every_element_to_its_head():
+    """Without rotation the split is a pure relabelling: written out element by
+    element, Q[b,h,t,c] = qkv[b,t,0,h,c], K takes index 1 and V index 2."""
+    B, N, H, d = 2, 3, 2, 8
+    qkv = torch.arange(B * N * 3 * H * d, dtype=F64).reshape(B, N, 3, H, d)
+    q, k, v = oracle.qkv_split_rope(qkv)
+    for b in range(B):
+        for t in range(N):
+            for h in range(H):
+                for c in range(d):
+                    flat = (((b * N + t) * 3) * H + h) * d + c
+                    assert q[b, h, t, c] == flat
+                    assert k[b, h, t, c] == flat + H * d
+                    assert v[b, h, t, c] == flat + 2 * H * d
+
+
+def test_qkv_split_rope_hand_values():
+    """Token 5 with two tokens per frame, first frame 1, sits at frame 3: its
+    query and key pair i turn by 3 * base^(-2i/rope_dims); V never turns, and
+    channels past rope_dims never move."""
+    B, N, H, d = 1, 6, 1, 8
+    qkv = torch.zeros(B, N, 3, H, d, dtype=F64)
+    qkv[0, 5, 0, 0, :] = torch.tensor([1.0, 0.0, 0.0, 2.0, 1.0, 1.0, 5.0, 6.0])
+    qkv[0, 5, 1, 0, :] = torch.tensor([0.0, 1.0, 3.0, 0.0, 2.0, 0.0, 7.0, 8.0])
+    qkv[0, 5, 2, 0, :] = torch.tensor([1.0, 2.0, 3.0, 4.0, 5.0, 6.0, 7.0, 8.0])
+    q, k, v = oracle.qkv_split_rope(qkv, rope_dims=6, base=64.0, tokens_per_frame=2,
+                                    first_frame=1)
+    a0, a1, a2 = 3.0, 3.0 * 64.0 ** (-2.0 / 6), 3.0 * 64.0 ** (-4.0 / 6)  # 3, 0.75, 0.1875
+    c, s = math.cos, math.sin
+    want_q = [c(a0), s(a0), -2 * s(a1), 2 * c(a1), c(a2) - s(a2), s(a2) + c(a2), 5.0, 6.0]
+    want_k = [-s(a0), c(a0), 3 * c(a1), 3 * s(a1), 2 * c(a2), 2 * s(a2), 7.0, 8.0]
+    assert torch.allclose(q[0, 0, 5], torch.tensor(want_q, dtype=F64), atol=1e-15, rtol=0)
+    assert torch.allclose(k[0, 0, 5], torch.tensor(want_k, dtype=F64), atol=1e-15, rtol=0)
+    assert torch.equal(v[0, 0, 5], qkv[0, 5, 2, 0])
+    assert torch.equal(q[0, 0, :5], torch.zeros(5, d, dtype=F64))
+
+
+def test_qkv_split_rope_scores_depend_on_frame_differences():
+    """With every channel rotated, Q K^T is unchanged when all positions move
+    by the same number of frames, and changes when the spacing changes."""
+    B, N, H, d = 1, 12, 2, 8
+    qkv = _rand(B, N, 3 * H, d, seed=98).to(F64).reshape(B, N, 3, H, d)
+    q1, k1, _ = oracle.qkv_split_rope(qkv, d, 100.0, 3, 0)
+    q2, k2, _ = oracle.qkv_split_rope(qkv, d, 100.0, 3, 11)
+    q3, k3, _ = oracle.qkv_split_rope(qkv, d, 100.0, 2, 0)
+    s1, s2, s3 = q1 @ k1.transpose(-1, -2), q2 @ k2.transpose(-1, -2), q3 @ k3.transpose(-1, -2)
+    assert torch.allclose(s1, s2, atol=1e-12, rtol=0)
+    assert (s3 - s1).abs().max() > 1e-3
