@@ -54,11 +54,13 @@ struct FwdLayout {
   static constexpr uint32_t O_COL(int t) { return 256u + OW * t; }
   static constexpr int THREADS = 384;
   // registers per thread after the re-split: softmax warpgroups 0-1 get
-  // more, warpgroup 2 (TMA, MMA, two idle warps) less; 2*128*224 + 128*56
-  // equals the launch's 384 threads x 168 registers
+  // more, warpgroup 2 (TMA, MMA, RoPE or idle warps) less; 2*128*S + 128*C
+  // equals the launch's 384 threads x 168 registers.  d = 128: the MMA
+  // warp's unrolled issue loop needs more than 56 (measured: 208/88 runs
+  // the d=128 forward 4% faster, 224/56 the d=64 one 1% faster)
   static constexpr int REGS_LAUNCH = 168;
-  static constexpr int REGS_SOFTMAX = 224;
-  static constexpr int REGS_CONTROL = 56;
+  static constexpr int REGS_SOFTMAX = (D == 64) ? 224 : 208;
+  static constexpr int REGS_CONTROL = (D == 64) ? 56 : 88;
   static_assert(2 * 128 * REGS_SOFTMAX + 128 * REGS_CONTROL == THREADS * REGS_LAUNCH,
                 "register re-split must hand out exactly the launch's registers");
 };
@@ -300,7 +302,12 @@ __global__ void __launch_bounds__(FwdLayout<D>::THREADS, 1)
         const uint32_t php = ((i - 1) / NS) & 1;
         if (!(ok = warp_wait(ROPE ? &k_rdy[st] : &k_full[st], ph, ctl))) break;
         tc_fence_after();
-        for (int t = 0; t < qt_n; ++t) {
+        // unrolled over the compile-time tile count, so every descriptor
+        // offset stays a constant (a runtime trip count here slows the whole
+        // forward by ~8%: the issuing code must never pause)
+#pragma unroll
+        for (int t = 0; t < QT; ++t) {
+          if (t >= qt_n) break;
           if (i > 0) {
             // PV of the first 64 keys while the softmax warps store the rest of P
             if (!(ok = warp_wait(&p_half[t], (i - 1) & 1, ctl))) break;
@@ -321,7 +328,9 @@ __global__ void __launch_bounds__(FwdLayout<D>::THREADS, 1)
       if (ok) {
         const int il = n_local - 1;
         const int stl = il % NS;
-        for (int t = 0; ok && t < qt_n; ++t) {
+#pragma unroll
+        for (int t = 0; t < QT; ++t) {
+          if (!ok || t >= qt_n) break;
           if (!(ok = warp_wait(&p_half[t], il & 1, ctl))) break;
           if (t == 0 && !(ok = warp_wait(&v_full[stl], (il / NS) & 1, ctl))) break;
           tc_fence_after();
