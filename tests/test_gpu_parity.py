@@ -237,7 +237,7 @@ def test_cache_split_count_does_not_change_the_result(mw):
     q, kn, vn, kr, vr = (t.cuda() for t in cpu)
     o_ref, lse_ref = oracle.cache_fwd(*cpu, 2400, 1700, 2400, 200, 0.09)
     outs = []
-    for s in (1, 2, 7):
+    for s in (1, 2, 7, 8, 12):
         mw.mw_set_option("cache_splits", s)
         try:
             outs.append(mw.mw_bca_cache_fwd(q, kn, vn, kr, vr, 1700, 2400, 200, 0.09))
