@@ -56,10 +56,15 @@ mw_status check_ptr(const void* p, const char* name) {
 }
 
 // Head dims: the kernels are built for 64 and 128; a head dim in between (a
-// multiple of 8, e.g. 72) runs on the 128 kernels, whose TMA maps read the
-// caller's d columns and fill the rest of each 128-column tile with zeros.
+// multiple of 8, e.g. 72) runs on the 128-wide tiles, whose TMA maps read
+// the caller's d columns and fill the rest of each 128-column tile with
+// zeros; up to 80 the MMAs themselves cover only 80 columns.
 bool d_supported(int d) { return d >= 64 && d <= 128 && d % 8 == 0; }
 int kernel_d(int d) { return d == 64 ? 64 : 128; }
+// The columns the MMAs cover: head dims up to 80 on the 128-wide tiles run
+// 80-wide MMAs (QK^T over 80 columns, 80 output columns), the rest use the
+// tile width.
+int mma_d(int d) { return d == 64 ? 64 : (d <= 80 ? 80 : 128); }
 
 mw_status check_dims(int B, int H, int d) {
   if (B < 1 || H < 1) return fail(MW_ERR_INVALID_ARG, "B and H must be >= 1 (B=%d H=%d)", B, H);
@@ -346,7 +351,7 @@ mw_status fwd_common(const void* q, const void* k, const void* v, const void* kr
     p.lse_part = reinterpret_cast<float*>(
         base + align256(static_cast<size_t>(p.num_splits) * BH * rows_q * D * sizeof(float)));
   }
-  MW_TRY(launch_status(mw::launch_fwd(D, tq, tk, tv, tkr, tvr, tks, tvs, p, rope.omega, stream),
+  MW_TRY(launch_status(mw::launch_fwd(D, mma_d(d), tq, tk, tv, tkr, tvr, tks, tvs, p, rope.omega, stream),
                        "forward kernel launch"));
   if (p.num_splits > 1)
     MW_TRY(launch_status(mw::launch_combine(D, d, p.o_part, p.lse_part, p.o, lse, p.num_splits, BH,
@@ -490,7 +495,8 @@ mw_status mw_bca_bwd_stage(int stage, const void* q, const void* k, const void* 
     p.dv = static_cast<__nv_bfloat16*>(dv);
     p.status = status;
     p.budget_ns = budget_ns();
-    MW_TRY(launch_status(mw::launch_bwd_main(D, tq, tk, tv, tdo, tdq, p, s), "backward kernel launch"));
+    MW_TRY(launch_status(mw::launch_bwd_main(D, mma_d(d), tq, tk, tv, tdo, tdq, p, s),
+                         "backward kernel launch"));
   }
   if (post)
     MW_TRY(launch_status(mw::launch_bwd_post(kernel_d(d), d, dq_acc, static_cast<__nv_bfloat16*>(dq), scale, BH,

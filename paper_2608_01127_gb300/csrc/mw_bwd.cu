@@ -38,8 +38,12 @@
 namespace mw {
 namespace {
 
-template <int D>
+// D: the head-dim width of the shared-memory tiles (64 or 128); DM <= D:
+// the columns the MMAs cover (S^T and dP^T reduce over DM, dK and dV have DM
+// columns), 80 for head dims up to 80 on the 128-wide tiles
+template <int D, int DM = D>
 struct BwdLayout {
+  static_assert(DM % 16 == 0 && DM <= D, "MMA width");
   static constexpr int QN = bwd_q_rows(D);           // query rows per step
   static constexpr bool DQT = (D == 128);            // dQ produced transposed
   static constexpr int CW = QN / 2;                  // query columns per P/dS warpgroup
@@ -104,12 +108,12 @@ __device__ __forceinline__ void red_add(float* addr, float a) {
   asm volatile("red.global.add.f32 [%0], %1;" ::"l"(addr), "f"(a) : "memory");
 }
 
-template <int D>
-__global__ void __launch_bounds__(BwdLayout<D>::THREADS, 1)
+template <int D, int DM>
+__global__ void __launch_bounds__(BwdLayout<D, DM>::THREADS, 1)
     bca_bwd_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_k,
                    const __grid_constant__ CUtensorMap tm_v, const __grid_constant__ CUtensorMap tm_do,
                    const __grid_constant__ CUtensorMap tm_dq, const BwdParams p) {
-  using L = BwdLayout<D>;
+  using L = BwdLayout<D, DM>;
   constexpr int NS = L::STAGES;
   constexpr int QN = L::QN;
   constexpr int CW = L::CW;
@@ -245,7 +249,7 @@ __global__ void __launch_bounds__(BwdLayout<D>::THREADS, 1)
       const bool role_a = !L::TWO_ISSUERS || warp == 13;  // S^T, dV, dP^T
       const bool role_b = !L::TWO_ISSUERS || warp == 14;  // dK, dQ
       constexpr uint32_t idesc_s = idesc_bf16_f32(128, QN, false, false);    // S^T, dP^T
-      constexpr uint32_t idesc_tn = idesc_bf16_f32(128, D, false, true);     // dV, dK
+      constexpr uint32_t idesc_tn = idesc_bf16_f32(128, DM, false, true);    // dV, dK
       // d = 64: dQ = dS K (M = query rows); d = 128: dQ^T = K^T dS^T (M = head dim)
       constexpr uint32_t idesc_dq = L::DQT ? idesc_bf16_f32(128, QN, true, true)
                                            : idesc_bf16_f32(128, D, true, true);
@@ -262,7 +266,7 @@ __global__ void __launch_bounds__(BwdLayout<D>::THREADS, 1)
       // X = A B^T, both K-major over d (S^T = K Q^T, dP^T = V dO^T)
       auto issue_kmajor = [&](uint32_t d_col, uint64_t a, uint64_t b) {
 #pragma unroll
-        for (int kk = 0; kk < D / 16; ++kk) {
+        for (int kk = 0; kk < DM / 16; ++kk) {
           const uint32_t ka = (kk >> 2) * L::KREGION + (kk & 3) * 32;
           const uint32_t kq = (kk >> 2) * L::QREGION + (kk & 3) * 32;
           umma_ss(tmem + d_col, sdesc_add(a, ka), sdesc_add(b, kq), idesc_s, kk > 0 ? 1u : 0u);
@@ -544,7 +548,7 @@ __global__ void __launch_bounds__(BwdLayout<D>::THREADS, 1)
       const int d_io = (D == 64) ? D : p.d_io;
       const size_t row_off = (static_cast<size_t>(bh) * p.N + krow) * d_io;
 #pragma unroll
-      for (int c = 0; c < D / 32; ++c) {
+      for (int c = 0; c < (DM + 31) / 32; ++c) {  // the chunks holding the DM columns
         uint32_t r[32];
         tmem_ld32(lane_base + col0 + 32 * c, r);
         tmem_wait_ld();
@@ -573,6 +577,8 @@ __global__ void __launch_bounds__(BwdLayout<D>::THREADS, 1)
         // lanes = head-dim columns, TMEM columns = the QN query rows; one warp
         // instruction reduces 32 consecutive head-dim columns of one row
         float* dst = p.dq_acc + (static_cast<size_t>(bh) * p.N_pad + q0) * D + wq * 32 + lane;
+        // head-dim columns past the caller's hold zeros: no reductions for them
+        const bool col_ok = wq * 32 + lane < p.d_io;
 #pragma unroll
         for (int half = 0; half < QN / 64; ++half) {
           uint32_t r0[32], r1[32];
@@ -584,10 +590,12 @@ __global__ void __launch_bounds__(BwdLayout<D>::THREADS, 1)
             __syncwarp();
             if (lane == 0) mbar_arrive(dq_free);
           }
+          if (col_ok) {
 #pragma unroll
-          for (int c = 0; c < 32; ++c) {
-            red_add(dst + static_cast<size_t>(64 * half + c) * D, __uint_as_float(r0[c]));
-            red_add(dst + static_cast<size_t>(64 * half + c + 32) * D, __uint_as_float(r1[c]));
+            for (int c = 0; c < 32; ++c) {
+              red_add(dst + static_cast<size_t>(64 * half + c) * D, __uint_as_float(r0[c]));
+              red_add(dst + static_cast<size_t>(64 * half + c + 32) * D, __uint_as_float(r1[c]));
+            }
           }
         }
       } else {
@@ -704,26 +712,26 @@ __global__ void __launch_bounds__(256) bwd_post_kernel(const float* __restrict__
   *reinterpret_cast<uint2*>(dq + e) = out;
 }
 
-template <int D>
+template <int D, int DM>
 cudaError_t launch_bwd_main_t(const CUtensorMap& tq, const CUtensorMap& tk, const CUtensorMap& tv,
                               const CUtensorMap& tdo, const CUtensorMap& tdq, const BwdParams& p,
                               cudaStream_t s) {
-  using L = BwdLayout<D>;
+  using L = BwdLayout<D, DM>;
   static bool attr_set = false;
   if (!attr_set) {
     // The in-kernel register re-split assumes the launch register count; with
     // any other count its setmaxnreg.inc could never be satisfied, so refuse.
     cudaFuncAttributes fa;
-    cudaError_t e0 = cudaFuncGetAttributes(&fa, bca_bwd_kernel<D>);
+    cudaError_t e0 = cudaFuncGetAttributes(&fa, bca_bwd_kernel<D, DM>);
     if (e0 != cudaSuccess) return e0;
     if (fa.numRegs != L::REGS_LAUNCH) return cudaErrorInvalidKernelImage;
-    cudaError_t e = cudaFuncSetAttribute(bca_bwd_kernel<D>,
+    cudaError_t e = cudaFuncSetAttribute(bca_bwd_kernel<D, DM>,
                                          cudaFuncAttributeMaxDynamicSharedMemorySize, L::BYTES);
     if (e != cudaSuccess) return e;
     attr_set = true;
   }
   const unsigned grid = static_cast<unsigned>(p.BH) * (p.N_pad / kTileRows);
-  bca_bwd_kernel<D><<<grid, L::THREADS, L::BYTES, s>>>(tq, tk, tv, tdo, tdq, p);
+  bca_bwd_kernel<D, DM><<<grid, L::THREADS, L::BYTES, s>>>(tq, tk, tv, tdo, tdq, p);
   return cudaGetLastError();
 }
 
@@ -741,11 +749,12 @@ cudaError_t launch_bwd_pre(int d, int d_io, const __nv_bfloat16* o, const __nv_b
   return cudaGetLastError();
 }
 
-cudaError_t launch_bwd_main(int d, const CUtensorMap& tq, const CUtensorMap& tk,
+cudaError_t launch_bwd_main(int d, int dm, const CUtensorMap& tq, const CUtensorMap& tk,
                             const CUtensorMap& tv, const CUtensorMap& tdo, const CUtensorMap& tdq,
                             const BwdParams& p, cudaStream_t s) {
-  if (d == 64) return launch_bwd_main_t<64>(tq, tk, tv, tdo, tdq, p, s);
-  return launch_bwd_main_t<128>(tq, tk, tv, tdo, tdq, p, s);
+  if (d == 64) return launch_bwd_main_t<64, 64>(tq, tk, tv, tdo, tdq, p, s);
+  if (dm == 80) return launch_bwd_main_t<128, 80>(tq, tk, tv, tdo, tdq, p, s);
+  return launch_bwd_main_t<128, 128>(tq, tk, tv, tdo, tdq, p, s);
 }
 
 cudaError_t launch_bwd_post(int d, int d_io, const float* dq_acc, __nv_bfloat16* dq, float scale,

@@ -22,8 +22,13 @@
 namespace mw {
 namespace {
 
-template <int D>
+// D: the head-dim width of the shared-memory tiles (64, or 128 with the
+// columns past the caller's zero-filled by TMA); DM <= D: the columns the
+// MMAs cover (QK^T reduces over DM, O has DM columns), 80 for head dims up
+// to 80 on the 128-wide tiles
+template <int D, int DM = D, bool ROPE = false>
 struct FwdLayout {
+  static_assert(DM % 16 == 0 && DM <= D, "MMA width");
   static constexpr int QT = kFwdQTiles;
   static constexpr int REG = D / 64;                  // 64-column swizzle regions per row
   static constexpr int REGION_BYTES = kTileRows * 128;
@@ -32,13 +37,19 @@ struct FwdLayout {
   static constexpr int OFF_Q = 0;
   static constexpr int OFF_K = OFF_Q + QT * TILE_BYTES;
   static constexpr int OFF_V = OFF_K + STAGES * TILE_BYTES;
-  // d = 64: the row sum of P comes out of the PV MMA itself: V is extended
-  // by a region of bf16 ones (reached through each stage descriptor's
-  // leading-byte offset), so O gets 16 extra columns that all hold sum_j P_ij
-  static constexpr bool SUM_MMA = (D == 64);
-  static constexpr int OW = SUM_MMA ? D + 16 : D;     // O columns in TMEM
+  // The row sum of P comes out of the PV MMA itself: V gets 16 extra columns
+  // of bf16 ones, so O gets 16 extra columns that all hold sum_j P_ij.
+  // d = 64: the ones are a region of their own, reached through each stage
+  // descriptor's leading-byte offset.  80-wide MMAs on the 128-wide tiles:
+  // the ones go into columns 80..95 of each V tile (which TMA fills with
+  // zeros), written by warps 10-11 after every load; with the RoPE re-shift
+  // those warps are busy and the softmax sums P itself.
+  static constexpr bool ONES_IN_V = (D == 128 && DM == 80 && !ROPE);
+  static constexpr bool SUM_MMA = (D == 64) || ONES_IN_V;
+  static constexpr int OW = SUM_MMA ? DM + 16 : DM;   // O columns in TMEM
+  static constexpr int SUM_COL = DM;                  // first row-sum column of O
   static constexpr int OFF_ONES = OFF_V + STAGES * TILE_BYTES;
-  static constexpr int ONES_BYTES = SUM_MMA ? REGION_BYTES : 0;
+  static constexpr int ONES_BYTES = (D == 64) ? REGION_BYTES : 0;
   // RoPE re-shift: per-pair frequencies, then (cos, sin) per (frame, pair) for
   // up to ROPE_FRAMES frames of the tile being rotated
   // (one copy per rotating warp)
@@ -47,7 +58,7 @@ struct FwdLayout {
   static constexpr int ROPE_WARP_BYTES = 2 * (D / 2) * 4 + ROPE_FRAMES * (D / 2) * 8;
   static constexpr int ROPE_BYTES = 2 * ROPE_WARP_BYTES;
   static constexpr int OFF_BAR = OFF_ROPE + ROPE_BYTES;
-  static constexpr int NBAR = 1 + 5 * STAGES + 3 * QT + 1;
+  static constexpr int NBAR = 1 + 6 * STAGES + 3 * QT + 1;
   static constexpr int OFF_MISC = OFF_BAR + NBAR * 8;
   static constexpr int BYTES = OFF_MISC + 16;
   static constexpr uint32_t S_COL(int t) { return 128u * t; }
@@ -113,14 +124,14 @@ __device__ __forceinline__ TileSrc tile_src(const Segs& g, int j) {
 // ROPE: the cache form with the ring's RoPE re-shift (warps 10-11 rotate ring
 // key tiles before the MMAs read them); the training and plain cache forms
 // are compiled without it.
-template <int D, bool ROPE>
-__global__ void __launch_bounds__(FwdLayout<D>::THREADS, 1)
+template <int D, int DM, bool ROPE>
+__global__ void __launch_bounds__(FwdLayout<D, DM>::THREADS, 1)
     bca_fwd_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_k,
                    const __grid_constant__ CUtensorMap tm_v, const __grid_constant__ CUtensorMap tm_kr,
                    const __grid_constant__ CUtensorMap tm_vr, const __grid_constant__ CUtensorMap tm_ks,
                    const __grid_constant__ CUtensorMap tm_vs, const FwdParams p,
                    const __grid_constant__ RopeFreq rope_om) {
-  using L = FwdLayout<D>;
+  using L = FwdLayout<D, DM, ROPE>;
   constexpr int QT = L::QT;
   constexpr int NS = L::STAGES;
   extern __shared__ __align__(1024) uint8_t smem[];
@@ -135,7 +146,8 @@ __global__ void __launch_bounds__(FwdLayout<D>::THREADS, 1)
   uint64_t* v_full = k_empty + NS;
   uint64_t* v_empty = v_full + NS;
   uint64_t* k_rdy = v_empty + NS;  // K tile in shared memory, RoPE re-shift applied
-  uint64_t* s_full = k_rdy + NS;
+  uint64_t* v_rdy = k_rdy + NS;    // V tile in shared memory with its ones columns
+  uint64_t* s_full = v_rdy + NS;
   uint64_t* p_full = s_full + QT;
   uint64_t* p_half = p_full + QT;  // first 64 keys of P in TMEM
   uint64_t* o_full = p_half + QT;
@@ -183,6 +195,7 @@ __global__ void __launch_bounds__(FwdLayout<D>::THREADS, 1)
       mbar_init(&v_full[s], 1);
       mbar_init(&v_empty[s], 1);
       mbar_init(&k_rdy[s], 2);
+      mbar_init(&v_rdy[s], 2);
     }
     for (int t = 0; t < QT; ++t) {
       mbar_init(&s_full[t], 1);
@@ -197,7 +210,7 @@ __global__ void __launch_bounds__(FwdLayout<D>::THREADS, 1)
     tmem_alloc(tmem_slot, 512);
     tmem_relinquish();
   }
-  if constexpr (L::SUM_MMA) {
+  if constexpr (L::ONES_BYTES > 0) {
     uint32_t* ones = reinterpret_cast<uint32_t*>(smem + L::OFF_ONES);
     for (int k = threadIdx.x; k < L::ONES_BYTES / 4; k += L::THREADS) ones[k] = 0x3F803F80u;  // bf16 1.0
     fence_proxy_async_smem();  // read by the tensor core (async proxy)
@@ -274,7 +287,7 @@ __global__ void __launch_bounds__(FwdLayout<D>::THREADS, 1)
         const uint64_t qa = sdesc_add(q_desc, t * L::TILE_BYTES);
         const uint64_t kb = sdesc_add(k_desc, st * L::TILE_BYTES);
 #pragma unroll
-        for (int kk = 0; kk < D / 16; ++kk) {
+        for (int kk = 0; kk < DM / 16; ++kk) {
           const uint32_t off = (kk >> 2) * L::REGION_BYTES + (kk & 3) * 32;
           umma_ss(tmem + L::S_COL(t), sdesc_add(qa, off), sdesc_add(kb, off), idesc_qk,
                   kk > 0 ? 1u : 0u);
@@ -284,7 +297,7 @@ __global__ void __launch_bounds__(FwdLayout<D>::THREADS, 1)
       auto issue_pv = [&](int t, int st, bool acc, int half) {
         // V stage st; for d = 64 the next 64 "columns" are the ones region
         const uint32_t vs = v_addr + st * L::TILE_BYTES;
-        const uint64_t vb = sdesc_sw128(vs, L::SUM_MMA ? ones_addr - vs : L::REGION_BYTES, 1024);
+        const uint64_t vb = sdesc_sw128(vs, L::ONES_BYTES > 0 ? ones_addr - vs : L::REGION_BYTES, 1024);
 #pragma unroll
         for (int k4 = 0; k4 < 4; ++k4) {
           const int kk = 4 * half + k4;
@@ -311,7 +324,7 @@ __global__ void __launch_bounds__(FwdLayout<D>::THREADS, 1)
           if (i > 0) {
             // PV of the first 64 keys while the softmax warps store the rest of P
             if (!(ok = warp_wait(&p_half[t], (i - 1) & 1, ctl))) break;
-            if (t == 0 && !(ok = warp_wait(&v_full[stp], php, ctl))) break;
+            if (t == 0 && !(ok = warp_wait(L::ONES_IN_V ? &v_rdy[stp] : &v_full[stp], php, ctl))) break;
             tc_fence_after();
             issue_pv(t, stp, i - 1 > 0, 0);
             if (!(ok = warp_wait(&p_full[t], (i - 1) & 1, ctl))) break;
@@ -332,7 +345,8 @@ __global__ void __launch_bounds__(FwdLayout<D>::THREADS, 1)
         for (int t = 0; t < QT; ++t) {
           if (!ok || t >= qt_n) break;
           if (!(ok = warp_wait(&p_half[t], il & 1, ctl))) break;
-          if (t == 0 && !(ok = warp_wait(&v_full[stl], (il / NS) & 1, ctl))) break;
+          if (t == 0 && !(ok = warp_wait(L::ONES_IN_V ? &v_rdy[stl] : &v_full[stl], (il / NS) & 1, ctl)))
+            break;
           tc_fence_after();
           issue_pv(t, stl, il > 0, 0);
           if (!(ok = warp_wait(&p_full[t], il & 1, ctl))) break;
@@ -437,6 +451,29 @@ __global__ void __launch_bounds__(FwdLayout<D>::THREADS, 1)
       __syncwarp();
       if (lane == 0) mbar_arrive(&k_rdy[st]);
     }
+  } else if (L::ONES_IN_V && (warp == 10 || warp == 11) && n_local > 0) {
+    // ------------------------------------------------------------ ones columns of V
+    // columns DM..DM+15 of each V tile hold bf16 ones (the row-sum columns of
+    // the PV MMA); TMA zero-fills them on every load, so they are written
+    // again after each one: 16-byte chunks (DM-64)/8 and (DM-64)/8 + 1 of
+    // region 1's 128-byte rows, at their 128-byte-swizzle positions
+    const int half = warp - 10;
+    const int c0 = (DM - 64) / 8;
+    const uint4 ones = make_uint4(0x3F803F80u, 0x3F803F80u, 0x3F803F80u, 0x3F803F80u);
+    for (int i = 0; i < n_local; ++i) {
+      const int st = i % NS;
+      if (!warp_wait(&v_full[st], (i / NS) & 1, ctl)) break;
+      uint8_t* reg1 = sV + st * L::TILE_BYTES + L::REGION_BYTES;
+#pragma unroll
+      for (int k = 0; k < 2; ++k) {
+        const int r = 64 * half + 32 * k + lane;
+        *reinterpret_cast<uint4*>(reg1 + r * 128 + ((c0 ^ (r & 7)) << 4)) = ones;
+        *reinterpret_cast<uint4*>(reg1 + r * 128 + (((c0 + 1) ^ (r & 7)) << 4)) = ones;
+      }
+      fence_proxy_async_smem();  // the tensor core reads the tile next
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&v_rdy[st]);
+    }
   }
   } else {
     regs_inc<L::REGS_SOFTMAX>();
@@ -499,8 +536,9 @@ __global__ void __launch_bounds__(FwdLayout<D>::THREADS, 1)
         }
         l *= alpha;
         if (i > 0) {
+          // exactly the tile's O columns (the next tile's O follows them)
 #pragma unroll
-          for (int c = 0; c < D / 32; ++c) {
+          for (int c = 0; c < DM / 32; ++c) {
             uint32_t r[32];
             tmem_ld32(o_addr + 32 * c, r);
             tmem_wait_ld();
@@ -508,13 +546,21 @@ __global__ void __launch_bounds__(FwdLayout<D>::THREADS, 1)
             for (int k = 0; k < 32; ++k) r[k] = __float_as_uint(__uint_as_float(r[k]) * alpha);
             tmem_st32(o_addr + 32 * c, r);
           }
-          if constexpr (L::SUM_MMA) {  // the row-sum columns scale with O
+          if constexpr (DM % 32 != 0) {
             uint32_t r[16];
-            tmem_ld16(o_addr + D, r);
+            tmem_ld16(o_addr + DM - 16, r);
             tmem_wait_ld();
 #pragma unroll
             for (int k = 0; k < 16; ++k) r[k] = __float_as_uint(__uint_as_float(r[k]) * alpha);
-            tmem_st16(o_addr + D, r);
+            tmem_st16(o_addr + DM - 16, r);
+          }
+          if constexpr (L::SUM_MMA) {  // the row-sum columns scale with O
+            uint32_t r[16];
+            tmem_ld16(o_addr + L::SUM_COL, r);
+            tmem_wait_ld();
+#pragma unroll
+            for (int k = 0; k < 16; ++k) r[k] = __float_as_uint(__uint_as_float(r[k]) * alpha);
+            tmem_st16(o_addr + L::SUM_COL, r);
           }
           tmem_wait_st();
         }
@@ -559,7 +605,7 @@ __global__ void __launch_bounds__(FwdLayout<D>::THREADS, 1)
     if constexpr (L::SUM_MMA) {
       if (have) {
         uint32_t r[16];
-        tmem_ld16(o_addr + D, r);
+        tmem_ld16(o_addr + L::SUM_COL, r);
         tmem_wait_ld();
         l = __uint_as_float(r[0]);
       }
@@ -569,8 +615,9 @@ __global__ void __launch_bounds__(FwdLayout<D>::THREADS, 1)
     const float m_eff = (m_used == -INFINITY) ? 0.f : m_used;
     const float lse = nonzero ? (m_eff + __log2f(l)) * 0.69314718055994530942f : -INFINITY;
     const size_t row_off = static_cast<size_t>(bh) * p.rows_q + row;
+    // the chunks that hold the DM columns of O (the caller's d_io <= DM)
 #pragma unroll
-    for (int c = 0; c < D / 32; ++c) {
+    for (int c = 0; c < (DM + 31) / 32; ++c) {
       uint32_t r[32];
       if (have) {
         tmem_ld32(o_addr + 32 * c, r);
@@ -666,43 +713,45 @@ __global__ void __launch_bounds__(256) combine_kernel(const float* __restrict__ 
   if (lse && lane == 0) lse[row] = wsum > 0.f ? m + __logf(wsum) : -INFINITY;
 }
 
-template <int D, bool ROPE>
+template <int D, int DM, bool ROPE>
 cudaError_t launch_fwd_t(const CUtensorMap& tq, const CUtensorMap& tk, const CUtensorMap& tv,
                          const CUtensorMap& tkr, const CUtensorMap& tvr, const CUtensorMap& tks,
                          const CUtensorMap& tvs, const FwdParams& p, const RopeFreq& om,
                          cudaStream_t s) {
-  using L = FwdLayout<D>;
+  using L = FwdLayout<D, DM, ROPE>;
   static bool attr_set = false;  // per process; the attribute is per function
   if (!attr_set) {
     // The in-kernel register re-split assumes the launch register count; with
     // any other count its setmaxnreg.inc could never be satisfied, so refuse.
     cudaFuncAttributes fa;
-    cudaError_t e = cudaFuncGetAttributes(&fa, bca_fwd_kernel<D, ROPE>);
+    cudaError_t e = cudaFuncGetAttributes(&fa, bca_fwd_kernel<D, DM, ROPE>);
     if (e != cudaSuccess) return e;
     if (fa.numRegs != L::REGS_LAUNCH) return cudaErrorInvalidKernelImage;
-    e = cudaFuncSetAttribute(bca_fwd_kernel<D, ROPE>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+    e = cudaFuncSetAttribute(bca_fwd_kernel<D, DM, ROPE>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                              L::BYTES);
     if (e != cudaSuccess) return e;
     attr_set = true;
   }
   const unsigned grid = static_cast<unsigned>(p.BH) * p.n_qblocks * p.num_splits;
-  bca_fwd_kernel<D, ROPE><<<grid, L::THREADS, L::BYTES, s>>>(tq, tk, tv, tkr, tvr, tks, tvs, p,
+  bca_fwd_kernel<D, DM, ROPE><<<grid, L::THREADS, L::BYTES, s>>>(tq, tk, tv, tkr, tvr, tks, tvs, p,
                                                               om);
   return cudaGetLastError();
 }
 
 }  // namespace
 
-cudaError_t launch_fwd(int d, const CUtensorMap& tq, const CUtensorMap& tk, const CUtensorMap& tv,
+cudaError_t launch_fwd(int d, int dm, const CUtensorMap& tq, const CUtensorMap& tk, const CUtensorMap& tv,
                        const CUtensorMap& tkr, const CUtensorMap& tvr, const CUtensorMap& tks,
                        const CUtensorMap& tvs, const FwdParams& p, const RopeFreq& om,
                        cudaStream_t s) {
   if (p.rope_dims > 0) {
-    if (d == 64) return launch_fwd_t<64, true>(tq, tk, tv, tkr, tvr, tks, tvs, p, om, s);
-    return launch_fwd_t<128, true>(tq, tk, tv, tkr, tvr, tks, tvs, p, om, s);
+    if (d == 64) return launch_fwd_t<64, 64, true>(tq, tk, tv, tkr, tvr, tks, tvs, p, om, s);
+    if (dm == 80) return launch_fwd_t<128, 80, true>(tq, tk, tv, tkr, tvr, tks, tvs, p, om, s);
+    return launch_fwd_t<128, 128, true>(tq, tk, tv, tkr, tvr, tks, tvs, p, om, s);
   }
-  if (d == 64) return launch_fwd_t<64, false>(tq, tk, tv, tkr, tvr, tks, tvs, p, om, s);
-  return launch_fwd_t<128, false>(tq, tk, tv, tkr, tvr, tks, tvs, p, om, s);
+  if (d == 64) return launch_fwd_t<64, 64, false>(tq, tk, tv, tkr, tvr, tks, tvs, p, om, s);
+  if (dm == 80) return launch_fwd_t<128, 80, false>(tq, tk, tv, tkr, tvr, tks, tvs, p, om, s);
+  return launch_fwd_t<128, 128, false>(tq, tk, tv, tkr, tvr, tks, tvs, p, om, s);
 }
 
 cudaError_t launch_combine(int d, int d_io, const float* o_part, const float* lse_part,

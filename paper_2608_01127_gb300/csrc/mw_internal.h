@@ -80,8 +80,10 @@ struct BwdParams {
 // Launchers (return cudaGetLastError() of the launch).
 // tkr/tvr: ring buffer maps; tks/tvs: sink anchor maps (any valid map when
 // the segment is empty)
-cudaError_t launch_fwd(int d, const CUtensorMap& tq, const CUtensorMap& tk, const CUtensorMap& tv,
-                       const CUtensorMap& tkr, const CUtensorMap& tvr, const CUtensorMap& tks,
+// d: tile width (64 or 128); dm: MMA width (d, or 80 on the 128-wide tiles
+// for head dims up to 80)
+cudaError_t launch_fwd(int d, int dm, const CUtensorMap& tq, const CUtensorMap& tk,
+                       const CUtensorMap& tv, const CUtensorMap& tkr, const CUtensorMap& tvr, const CUtensorMap& tks,
                        const CUtensorMap& tvs, const FwdParams& p, const RopeFreq& rope_om,
                        cudaStream_t s);
 // d: the kernels' head dim (64 or 128); d_io: the caller's (a multiple of 8, <= d)
@@ -93,7 +95,8 @@ cudaError_t launch_bwd_pre(int d, int d_io, const __nv_bfloat16* o, const __nv_b
                            int N, int N_pad, cudaStream_t s);
 // tdq: f32 map over dQacc [BH, N_pad, d] with 32 x 32 boxes (128-byte
 // swizzle), the target of the d = 64 kernel's TMA reduce-adds
-cudaError_t launch_bwd_main(int d, const CUtensorMap& tq, const CUtensorMap& tk,
+// dm: MMA width as for launch_fwd
+cudaError_t launch_bwd_main(int d, int dm, const CUtensorMap& tq, const CUtensorMap& tk,
                             const CUtensorMap& tv, const CUtensorMap& tdo, const CUtensorMap& tdq,
                             const BwdParams& p, cudaStream_t s);
 cudaError_t launch_bwd_post(int d, int d_io, const float* dq_acc, __nv_bfloat16* dq, float scale,
