@@ -366,11 +366,11 @@ def run_ours(args):
                    "flops_per_step": step_flops, "unmasked_pairs": pairs,
                    "l2": "256 MiB buffer written between timed steps (outside the events)"},
         "frac_of_bf16_peak": round(value / world / peaks["bf16_tflops"], 4),
-        "roofline": {"kernel": f"bca_bwd_kernel<{cfg.d}> (backward key-tile kernel)", "bound": "tensor",
+        "roofline": {"kernel": f"bca_bwd_kernel<{cfg.d}, {cfg.d}> (backward key-tile kernel)", "bound": "tensor",
                      "achieved": round(achieved, 2), "peak": peaks["bf16_tflops"],
                      "peak_source": peaks["source"] + " bf16 burst", "unit": "TFLOP/s",
                      "frac": round(achieved / peaks["bf16_tflops"], 4),
-                     "traffic": profiled_traffic(f"bca_bwd_kernel<{cfg.d}>", workload),
+                     "traffic": profiled_traffic(f"bca_bwd_kernel<{cfg.d},{cfg.d}>", workload),
                      "algorithmic_bytes": bwd_main_bytes(cfg),
                      "ms_per_launch": round(main_ms, 4)},
         "fwd": {"ms": round(fwd_ms, 4),
