@@ -85,7 +85,8 @@ TRAIN_CONFIGS: Dict[str, TrainConfig] = {
     # 4 chunks x 64 tokens, forward only
     "tiny_fwd": TrainConfig("tiny_fwd", B=1, H=2, d=64, n_chunks=4, T=64, seed=0,
                             backward=False),
-    # MiniWorld-B-like width 768 / 12 heads, 16 chunks of one 22x40 latent frame
+    # MiniWorld-B-like width 768 / 12 heads, 16 chunks of 880 tokens (two
+    # latent frames of 440 tokens each)
     "train_b12_d64": TrainConfig("train_b12_d64", B=2, H=12, d=64, n_chunks=16,
                                  T=880, seed=1),
     # width 2048 / 16 heads, 21 chunks, peaky logits from per-head gains
