@@ -331,6 +331,19 @@ __global__ void __launch_bounds__(BwdLayout<D, DM>::THREADS, 1)
         if (role_b) {
           if (!(ok = warp_wait(p_ready, j & 1, ctl))) break;
           tc_fence_after();
+          if constexpr (!L::SHARED_X) {
+            // d = 64: dQ_j first, so the drain starts while dK_j runs
+            if (j > 0) {
+              if (!(ok = warp_wait(dq_free, (j - 1) & 1, ctl))) break;
+              tc_fence_after();
+            }
+            const uint64_t ds_mn = sdesc_add(ds_mn0, (j % L::DS_BUFS) * L::DS_BYTES);
+#pragma unroll
+            for (int kk = 0; kk < kTileRows / 16; ++kk)
+              umma_ss(tmem + L::DQ_COL, sdesc_add(ds_mn, kk * 2048), sdesc_add(k_mn, kk * 2048),
+                      idesc_dq, kk > 0 ? 1u : 0u);
+            umma_commit(dq_full);
+          }
           // dK += dS^T Q_j (d = 64: dS^T read from shared memory, K-major)
           const uint64_t ds_kmaj = sdesc_add(ds_kmaj0, (j % L::DS_BUFS) * L::DS_BYTES);
 #pragma unroll
@@ -343,6 +356,7 @@ __global__ void __launch_bounds__(BwdLayout<D, DM>::THREADS, 1)
                       sdesc_add(q_mn, kk * 2048), idesc_tn, (j > 0 || kk > 0) ? 1u : 0u);
           }
           umma_commit(&q_empty[st]);
+          if constexpr (!L::SHARED_X) umma_commit(&ds_free[j % L::DS_BUFS]);
         }
         if (L::SHARED_X && more) {
           // X is free once dV/dK have read P^T/dS^T (issue order): S^T of the
@@ -357,7 +371,7 @@ __global__ void __launch_bounds__(BwdLayout<D, DM>::THREADS, 1)
           issue_kmajor(L::DP_COL, v_kmaj, sdesc_add(do_kmaj0, st1 * L::QTILE));
           umma_commit(dp_full);
         }
-        if (role_b) {
+        if (L::SHARED_X && role_b) {
           // dQ of this step, once the drain has read the previous one
           if (j > 0) {
             if (!(ok = warp_wait(dq_free, (j - 1) & 1, ctl))) break;
