@@ -85,7 +85,9 @@ SMALL = [
     (1, 3, 5, 200, 64, 1.0),
     (2, 2, 1, 600, 128, 1.0),    # a single chunk: full bidirectional attention
     (1, 20, 3, 96, 128, 1.0),    # the 3B head layout (20 heads of 128)
-    (1, 2, 3, 100, 72, 1.0),     # the 0.5B head dim (72: zero-padded to 128 in the kernels)
+    (1, 2, 3, 100, 72, 1.0),     # the 0.5B head dim (72: 80-wide MMAs on 128-wide tiles)
+    (1, 2, 3, 100, 80, 2.0),     # the widest head dim on 80-wide MMAs (ones from column 80)
+    (1, 1, 2, 150, 88, 1.0),     # the narrowest on 128-wide MMAs
     (2, 1, 2, 130, 96, 2.0),     # another padded head dim
 ]
 
@@ -209,6 +211,7 @@ CACHE_SMALL = [
     (1, 2, 2, 130, 780, 780, 390, 128, 1),     # forced single pass
     (1, 1, 1, 16, 48, 40, 30, 64, 3),          # tiny ring, more splits than needed
     (1, 2, 2, 64, 640, 640, 320, 72, 3),       # padded head dim with split-KV
+    (1, 2, 2, 200, 1200, 1000, 900, 80, 2),    # 80-wide MMAs, wrapped ring, split-KV
 ]
 
 
