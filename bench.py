@@ -568,7 +568,9 @@ def _cache_roofline(cfg, us, peaks):
 
 def bench_rolling(mw, dev, peaks):
     """64 streaming steps: cache forward of one 880-token chunk against the
-    8-chunk ring, then commit of that chunk (FIFO eviction); per-step latency."""
+    8-chunk ring, then commit of that chunk (FIFO eviction), through the
+    one-call streaming step; per-step latency.  The same steps as separate
+    forward and commit calls are timed beside it."""
     cfg = CACHE_CONFIGS["rolling_cache"]
     x = gen_cache(cfg)
     kr, vr = x["k_ring"].to(dev), x["v_ring"].to(dev)
@@ -583,6 +585,11 @@ def bench_rolling(mw, dev, peaks):
         plan.append((head, length, ring.commit(cfg.T)))
 
     def step(s):
+        h, ln, slot = plan[s]
+        mw.mw_bca_cache_step(qs[s], ks[s], vs[s], kr, vr, h, ln, slot, cfg.T, cfg.T, cfg.scale,
+                             need_lse=False, workspace=ws, out=o)
+
+    def step_separate(s):
         h, ln, slot = plan[s]
         mw.mw_bca_cache_fwd(qs[s], ks[s], vs[s], kr, vr, h, ln, cfg.T, cfg.scale, need_lse=False,
                             workspace=ws, out=o)
@@ -603,31 +610,37 @@ def bench_rolling(mw, dev, peaks):
     med = statistics.median(us)
     # the same 64 steps captured once as a CUDA graph and replayed: device
     # time per step without host launch overhead
-    graph = torch.cuda.CUDAGraph()
-    side = torch.cuda.Stream()
-    side.wait_stream(torch.cuda.current_stream())
-    with torch.cuda.stream(side):
-        with torch.cuda.graph(graph, stream=side, capture_error_mode="relaxed"):
-            for s in range(cfg.steps):
-                step(s)
-    torch.cuda.current_stream().wait_stream(side)
-    graph.replay()
-    torch.cuda.synchronize()
-    reps = []
-    for _ in range(5):
-        e = Events()
-        e.start()
+    def graph_us(fn):
+        graph = torch.cuda.CUDAGraph()
+        side = torch.cuda.Stream()
+        side.wait_stream(torch.cuda.current_stream())
+        with torch.cuda.stream(side):
+            with torch.cuda.graph(graph, stream=side, capture_error_mode="relaxed"):
+                for s in range(cfg.steps):
+                    fn(s)
+        torch.cuda.current_stream().wait_stream(side)
         graph.replay()
-        e.stop()
         torch.cuda.synchronize()
-        reps.append(e.ms() * 1e3 / cfg.steps)
-    g_us = statistics.median(reps)
+        reps = []
+        for _ in range(5):
+            e = Events()
+            e.start()
+            graph.replay()
+            e.stop()
+            torch.cuda.synchronize()
+            reps.append(e.ms() * 1e3 / cfg.steps)
+        return statistics.median(reps)
+    g_us = graph_us(step)
+    g_sep_us = graph_us(step_separate)
     res = {"steps": cfg.steps, "us_per_step_median": round(med, 2),
            "us_per_step_p90": round(us[int(0.9 * (len(us) - 1))], 2),
            "us_per_step_graph": round(g_us, 2),
-           "gpu_launches_per_step": 3 if ws_bytes > 0 else 2,
-           "note": "eager: per-step events with host launch in the loop; graph: the 64 steps "
-                   "replayed as one CUDA graph. The ring (57.7 MB) stays L2-resident across "
+           "us_per_step_graph_separate_calls": round(g_sep_us, 2),
+           "gpu_launches_per_step": 2,
+           "note": "mw_bca_cache_step (forward, then the split combine and the ring commit in "
+                   "one launch); eager: per-step events with host launch in the loop; graph: "
+                   "the 64 steps replayed as one CUDA graph; separate_calls: forward and "
+                   "commit as two API calls. The ring (57.7 MB) stays L2-resident across "
                    "steps, as in streaming"}
     res.update(_cache_roofline(cfg, g_us, peaks))
     # the same stream with the ring's RoPE re-shift fused into its read (32

@@ -203,6 +203,29 @@ mw_status mw_bca_cache_commit(void* k_cache, void* v_cache, int cache_cap, int s
                               void* stream);
 
 /*
+ * One streaming step (Sec. 3.5): the in-flight chunks attend to the ring as
+ * in mw_bca_cache_fwd, then the oldest commit_rows rows of k_new / v_new
+ * (the chunk that reached the data endpoint) are committed to ring rows
+ * (commit_slot + r) mod cache_cap, exactly as mw_bca_cache_commit would.
+ * The commit runs after the forward has read the ring (stream order), so
+ * commit_slot may be the slot of the tokens it evicts; when the forward
+ * splits its key range, the commit shares one launch with the split
+ * combine.  The result equals mw_bca_cache_fwd followed by
+ * mw_bca_cache_commit, bit for bit.
+ *   k_cache, v_cache : written ([B,H,cache_cap,d])
+ *   commit_rows      : 0 <= commit_rows <= min(cache_cap, n_q_chunks*T_chunk)
+ *                      (0: no commit, i.e. mw_bca_cache_fwd)
+ *   commit_slot      : 0 <= commit_slot < cache_cap
+ * Every other argument, the workspace and the errors are as for
+ * mw_bca_cache_fwd.
+ */
+mw_status mw_bca_cache_step(const void* q, const void* k_new, const void* v_new, void* k_cache,
+                            void* v_cache, int cache_cap, int cache_head, int cache_len,
+                            int commit_slot, int commit_rows, void* o, float* lse,
+                            void* workspace, size_t ws_bytes, int B, int H, int n_q_chunks,
+                            int T_chunk, int d, float scale, void* stream);
+
+/*
  * QKV split with temporal RoPE (the input side of the attention: Sec. 3.2
  * runs block-causal attention over the latent tokens; Sec. 3.5 gives keys
  * temporal positions that the rolling cache re-shifts).  The fused QKV

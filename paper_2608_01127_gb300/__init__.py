@@ -28,7 +28,7 @@ import torch
 
 __all__ = [
     "MWError", "library", "lib_path", "mw_bca_fwd", "mw_bca_bwd", "mw_bca_cache_fwd",
-    "mw_bca_cache_fwd_sink", "mw_bca_cache_fwd_rope",
+    "mw_bca_cache_fwd_sink", "mw_bca_cache_fwd_rope", "mw_bca_cache_step",
     "mw_bca_cache_commit", "mw_bca_bwd_workspace_size", "mw_bca_cache_workspace_size",
     "mw_device_status", "mw_set_option", "mw_qkv_rope_split", "BlockCausalAttention",
     "EXPORTED_SYMBOLS",
@@ -43,7 +43,7 @@ EXPORTED_SYMBOLS = (
     "mw_bca_cache_workspace_size",
     "mw_bca_cache_fwd", "mw_bca_cache_commit", "mw_status_string", "mw_last_error",
     "mw_device_status", "mw_set_option", "mw_bca_cache_fwd_noalloc", "mw_bca_cache_fwd_sink",
-    "mw_bca_cache_fwd_rope", "mw_qkv_rope_split",
+    "mw_bca_cache_fwd_rope", "mw_qkv_rope_split", "mw_bca_cache_step",
 )
 
 STATUS = {0: "MW_OK", 1: "MW_ERR_INVALID_ARG", 2: "MW_ERR_UNSUPPORTED", 3: "MW_ERR_CUDA",
@@ -92,6 +92,8 @@ def library() -> ctypes.CDLL:
                                        _P, _P, _P, _Z, _I, _I, _I, _I, _I, _F, _P]),
         "mw_bca_cache_commit": (_I, [_P, _P, _I, _I, _P, _P, _I, _I, _I, _I, _P]),
         "mw_qkv_rope_split": (_I, [_P, _P, _P, _P, _I, _I, _I, _I, _I, _F, _I, _I, _P]),
+        "mw_bca_cache_step": (_I, [_P, _P, _P, _P, _P, _I, _I, _I, _I, _I, _P, _P, _P, _Z,
+                                   _I, _I, _I, _I, _I, _F, _P]),
         "mw_bca_cache_fwd_noalloc": (_I, [_P, _P, _P, _P, _P, _I, _I, _I, _P, _P,
                                           _I, _I, _I, _I, _I, _F, _P]),
         "mw_status_string": (ctypes.c_char_p, [_I]),
@@ -229,7 +231,7 @@ def mw_bca_cache_fwd_rope(q, k_new, v_new, k_sink, v_sink, k_cache, v_cache, cac
 
 
 def _cache_fwd(q, k_new, v_new, k_sink, v_sink, k_cache, v_cache, cache_head, cache_len,
-               T_chunk, scale, need_lse, workspace, out, rope=None):
+               T_chunk, scale, need_lse, workspace, out, rope=None, commit=None):
     B, H, M, d = _bhnd(q, "q")
     for t, n in ((k_new, "k_new"), (v_new, "v_new")):
         if _bhnd(t, n) != (B, H, M, d):
@@ -252,7 +254,13 @@ def _cache_fwd(q, k_new, v_new, k_sink, v_sink, k_cache, v_cache, cache_head, ca
         workspace = torch.empty(ws_bytes, dtype=torch.uint8, device=q.device)
     o = torch.empty_like(q) if out is None else out
     lse = torch.empty((B, H, M), dtype=torch.float32, device=q.device) if need_lse else None
-    if rope is not None:
+    if commit is not None:
+        _check(library().mw_bca_cache_step(
+            _ptr(q), _ptr(k_new), _ptr(v_new), _ptr(k_cache), _ptr(v_cache), cap, cache_head,
+            cache_len, int(commit[0]), int(commit[1]), _ptr(o), _ptr(lse),
+            _ptr(workspace) if ws_bytes else None, ws_bytes, B, H, W, T_chunk, d,
+            _scale(scale, d), _stream()))
+    elif rope is not None:
         _check(library().mw_bca_cache_fwd_rope(
             _ptr(q), _ptr(k_new), _ptr(v_new), _ptr(k_sink), _ptr(v_sink), sink_len,
             _ptr(k_cache), _ptr(v_cache), cap, cache_head, cache_len, int(rope[0]),
@@ -271,6 +279,18 @@ def _cache_fwd(q, k_new, v_new, k_sink, v_sink, k_cache, v_cache, cache_head, ca
             _ptr(workspace) if ws_bytes else None, ws_bytes, B, H, W, T_chunk, d,
             _scale(scale, d), _stream()))
     return o, lse
+
+
+def mw_bca_cache_step(q, k_new, v_new, k_cache, v_cache, cache_head: int, cache_len: int,
+                      commit_slot: int, commit_rows: int, T_chunk: int,
+                      scale: Optional[float] = None, need_lse: bool = True,
+                      workspace: Optional[torch.Tensor] = None, out: Optional[torch.Tensor] = None):
+    """One streaming step (Sec. 3.5): mw_bca_cache_fwd, then the first
+    ``commit_rows`` rows of k_new / v_new go to ring rows (commit_slot + r) mod
+    cap (FIFO eviction); returns (O, LSE or None)."""
+    return _cache_fwd(q, k_new, v_new, None, None, k_cache, v_cache, cache_head, cache_len,
+                      T_chunk, scale, need_lse, workspace, out,
+                      commit=(commit_slot, commit_rows))
 
 
 def mw_bca_cache_commit(k_cache, v_cache, slot_start: int, k_src, v_src) -> None:

@@ -298,7 +298,8 @@ mw::RopeFreq rope_freq(int dims, float base) {
 mw_status fwd_common(const void* q, const void* k, const void* v, const void* kr, const void* vr,
                      int cap, int head, int len, const void* ks, const void* vs, int sink_len,
                      const RopeArgs& rope, void* o, float* lse, void* ws, size_t ws_bytes, int BH,
-                     int rows_q, int T, int d, float scale, int splits, cudaStream_t stream) {
+                     int rows_q, int T, int d, float scale, int splits,
+                     const mw::CommitJob& commit, cudaStream_t stream) {
   DeviceScope scope(stream);
   MW_TRY(scope.status());
   unsigned* status = nullptr;
@@ -355,8 +356,10 @@ mw_status fwd_common(const void* q, const void* k, const void* v, const void* kr
                        "forward kernel launch"));
   if (p.num_splits > 1)
     MW_TRY(launch_status(mw::launch_combine(D, d, p.o_part, p.lse_part, p.o, lse, p.num_splits, BH,
-                                            rows_q, stream),
+                                            rows_q, commit, stream),
                          "combine kernel launch"));
+  else if (commit.rows > 0)
+    MW_TRY(launch_status(mw::launch_commit(commit, stream), "commit kernel launch"));
   return ok();
 }
 
@@ -410,8 +413,9 @@ mw_status mw_bca_fwd(const void* q, const void* k, const void* v, void* o, float
   MW_TRY(check_ptr(o, "o"));
   if (lse && (reinterpret_cast<uintptr_t>(lse) & 3u))
     return fail(MW_ERR_INVALID_ARG, "lse is not 4-byte aligned");
-  return fwd_common(q, k, v, nullptr, nullptr, 1, 0, 0, nullptr, nullptr, 0, RopeArgs{}, o, lse, nullptr, 0, B * H,
-                    static_cast<int>(N), T_chunk, d, scale, 1, static_cast<cudaStream_t>(stream));
+  return fwd_common(q, k, v, nullptr, nullptr, 1, 0, 0, nullptr, nullptr, 0, RopeArgs{}, o, lse,
+                    nullptr, 0, B * H, static_cast<int>(N), T_chunk, d, scale, 1, mw::CommitJob{},
+                    static_cast<cudaStream_t>(stream));
 }
 
 size_t mw_bca_bwd_workspace_size(int B, int H, int n_chunks, int T_chunk, int d) {
@@ -544,13 +548,16 @@ mw_status mw_bca_cache_fwd_sink(const void* q, const void* k_new, const void* v_
                                ws_bytes, B, H, n_q_chunks, T_chunk, d, scale, stream);
 }
 
-mw_status mw_bca_cache_fwd_rope(const void* q, const void* k_new, const void* v_new,
+// The cache forward in all its forms; `commit` (rows > 0) is a ring commit
+// that runs once the forward has read the ring.
+static mw_status cache_fwd_impl(const void* q, const void* k_new, const void* v_new,
                                 const void* k_sink, const void* v_sink, int sink_len,
                                 const void* k_cache, const void* v_cache, int cache_cap,
                                 int cache_head, int cache_len, int rope_dims, float rope_base,
                                 int tokens_per_frame, int first_frame, void* o, float* lse,
                                 void* workspace, size_t ws_bytes, int B, int H, int n_q_chunks,
-                                int T_chunk, int d, float scale, void* stream) {
+                                int T_chunk, int d, float scale, const mw::CommitJob& commit,
+                                void* stream) {
   MW_TRY(check_dims(B, H, d));
   if (n_q_chunks < 1 || T_chunk < 1)
     return fail(MW_ERR_INVALID_ARG, "n_q_chunks=%d and T_chunk=%d must be >= 1", n_q_chunks, T_chunk);
@@ -610,8 +617,53 @@ mw_status mw_bca_cache_fwd_rope(const void* q, const void* k_new, const void* v_
   }
   return fwd_common(q, k_new, v_new, k_cache, v_cache, cache_cap, cache_head, cache_len, k_sink,
                     v_sink, sink_len, rope, o, lse, need > 0 ? workspace : nullptr, ws_bytes, BH,
-                    static_cast<int>(rows), T_chunk, d, scale, splits,
+                    static_cast<int>(rows), T_chunk, d, scale, splits, commit,
                     static_cast<cudaStream_t>(stream));
+}
+
+mw_status mw_bca_cache_fwd_rope(const void* q, const void* k_new, const void* v_new,
+                                const void* k_sink, const void* v_sink, int sink_len,
+                                const void* k_cache, const void* v_cache, int cache_cap,
+                                int cache_head, int cache_len, int rope_dims, float rope_base,
+                                int tokens_per_frame, int first_frame, void* o, float* lse,
+                                void* workspace, size_t ws_bytes, int B, int H, int n_q_chunks,
+                                int T_chunk, int d, float scale, void* stream) {
+  return cache_fwd_impl(q, k_new, v_new, k_sink, v_sink, sink_len, k_cache, v_cache, cache_cap,
+                        cache_head, cache_len, rope_dims, rope_base, tokens_per_frame, first_frame,
+                        o, lse, workspace, ws_bytes, B, H, n_q_chunks, T_chunk, d, scale,
+                        mw::CommitJob{}, stream);
+}
+
+mw_status mw_bca_cache_step(const void* q, const void* k_new, const void* v_new, void* k_cache,
+                            void* v_cache, int cache_cap, int cache_head, int cache_len,
+                            int commit_slot, int commit_rows, void* o, float* lse,
+                            void* workspace, size_t ws_bytes, int B, int H, int n_q_chunks,
+                            int T_chunk, int d, float scale, void* stream) {
+  mw::CommitJob job;
+  if (commit_rows != 0) {
+    const long long rows = static_cast<long long>(n_q_chunks) * T_chunk;
+    if (commit_rows < 0 || commit_rows > cache_cap || commit_rows > rows)
+      return fail(MW_ERR_INVALID_ARG, "commit_rows=%d not in [0, min(cache_cap, n_q_chunks*T_chunk)]",
+                  commit_rows);
+    if (commit_slot < 0 || commit_slot >= cache_cap)
+      return fail(MW_ERR_INVALID_ARG, "commit_slot=%d not in [0, cache_cap=%d)", commit_slot,
+                  cache_cap);
+    MW_TRY(check_ptr(k_cache, "k_cache"));
+    MW_TRY(check_ptr(v_cache, "v_cache"));
+    job.kc = static_cast<__nv_bfloat16*>(k_cache);
+    job.vc = static_cast<__nv_bfloat16*>(v_cache);
+    job.ks = static_cast<const __nv_bfloat16*>(k_new);
+    job.vs = static_cast<const __nv_bfloat16*>(v_new);
+    job.cap = cache_cap;
+    job.slot = commit_slot;
+    job.rows = commit_rows;
+    job.src_rows = static_cast<int>(rows);
+    job.d = d;
+    job.BH = B * H;
+  }
+  return cache_fwd_impl(q, k_new, v_new, nullptr, nullptr, 0, k_cache, v_cache, cache_cap,
+                        cache_head, cache_len, 0, 0.f, 1, 0, o, lse, workspace, ws_bytes, B, H,
+                        n_q_chunks, T_chunk, d, scale, job, stream);
 }
 
 mw_status mw_bca_cache_commit(void* k_cache, void* v_cache, int cache_cap, int slot_start,
@@ -630,12 +682,19 @@ mw_status mw_bca_cache_commit(void* k_cache, void* v_cache, int cache_cap, int s
   MW_TRY(check_ptr(v_src, "v_src"));
   DeviceScope scope(static_cast<cudaStream_t>(stream));
   MW_TRY(scope.status());
-  return launch_status(
-      mw::launch_commit(d, static_cast<__nv_bfloat16*>(k_cache), static_cast<__nv_bfloat16*>(v_cache),
-                        static_cast<const __nv_bfloat16*>(k_src),
-                        static_cast<const __nv_bfloat16*>(v_src), cache_cap, slot_start, rows,
-                        B * H, static_cast<cudaStream_t>(stream)),
-      "commit kernel launch");
+  mw::CommitJob job;
+  job.kc = static_cast<__nv_bfloat16*>(k_cache);
+  job.vc = static_cast<__nv_bfloat16*>(v_cache);
+  job.ks = static_cast<const __nv_bfloat16*>(k_src);
+  job.vs = static_cast<const __nv_bfloat16*>(v_src);
+  job.cap = cache_cap;
+  job.slot = slot_start;
+  job.rows = rows;
+  job.src_rows = rows;
+  job.d = d;
+  job.BH = B * H;
+  return launch_status(mw::launch_commit(job, static_cast<cudaStream_t>(stream)),
+                       "commit kernel launch");
 }
 
 mw_status mw_qkv_rope_split(const void* qkv, void* q, void* k, void* v, int B, int N, int H,

@@ -665,13 +665,25 @@ __global__ void __launch_bounds__(FwdLayout<D, DM>::THREADS, 1)
 }
 
 // Merge of split-KV partials (per row): LSE = ln sum_s exp(LSE_s),
-// O = sum_s exp(LSE_s - LSE) O_s.  One warp per row.
+// O = sum_s exp(LSE_s - LSE) O_s.  One warp per row, 8 rows per block; the
+// blocks after those carry the ring commit cj (one thread per 16-byte piece
+// of a committed row of one head), when there is one.
 template <int D>
 __global__ void __launch_bounds__(256) combine_kernel(const float* __restrict__ o_part,
                                                       const float* __restrict__ lse_part,
                                                       __nv_bfloat16* __restrict__ o,
                                                       float* __restrict__ lse, int splits,
-                                                      int n_rows, int d_io_arg) {
+                                                      int n_rows, int d_io_arg,
+                                                      const CommitJob cj) {
+  const int combine_blocks = (n_rows + 7) / 8;
+  if (static_cast<int>(blockIdx.x) >= combine_blocks) {
+    const long long idx =
+        static_cast<long long>(blockIdx.x - combine_blocks) * blockDim.x + threadIdx.x;
+    const int per_head = cj.rows * (cj.d / 8);
+    if (idx < static_cast<long long>(per_head) * cj.BH)
+      commit_piece(cj, static_cast<int>(idx / per_head), static_cast<int>(idx % per_head));
+    return;
+  }
   const int d_io = (D == 64) ? D : d_io_arg;  // padded head dims use the 128-wide kernels
   const int row = blockIdx.x * 8 + (threadIdx.x >> 5);
   const int lane = threadIdx.x & 31;
@@ -756,13 +768,15 @@ cudaError_t launch_fwd(int d, int dm, const CUtensorMap& tq, const CUtensorMap& 
 
 cudaError_t launch_combine(int d, int d_io, const float* o_part, const float* lse_part,
                            __nv_bfloat16* o, float* lse, int splits, int BH, int rows,
-                           cudaStream_t s) {
+                           const CommitJob& cj, cudaStream_t s) {
   const int n_rows = BH * rows;
-  const unsigned grid = static_cast<unsigned>((n_rows + 7) / 8);
+  const long long commit_pieces = static_cast<long long>(cj.rows) * (cj.d / 8) * cj.BH;
+  const long long blocks = (n_rows + 7) / 8 + (commit_pieces + 255) / 256;
+  const unsigned grid = static_cast<unsigned>(blocks);
   if (d == 64)
-    combine_kernel<64><<<grid, 256, 0, s>>>(o_part, lse_part, o, lse, splits, n_rows, d_io);
+    combine_kernel<64><<<grid, 256, 0, s>>>(o_part, lse_part, o, lse, splits, n_rows, d_io, cj);
   else
-    combine_kernel<128><<<grid, 256, 0, s>>>(o_part, lse_part, o, lse, splits, n_rows, d_io);
+    combine_kernel<128><<<grid, 256, 0, s>>>(o_part, lse_part, o, lse, splits, n_rows, d_io, cj);
   return cudaGetLastError();
 }
 

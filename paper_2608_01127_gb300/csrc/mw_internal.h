@@ -77,6 +77,31 @@ struct BwdParams {
   unsigned long long budget_ns;
 };
 
+// A ring commit (Sec. 3.5): rows [0, rows) of each head of k_src / v_src
+// ([B,H,src_rows,d], src_rows >= rows) go to ring rows (slot + r) mod cap of
+// k_cache / v_cache ([B,H,cap,d]).  rows == 0: nothing to do.
+struct CommitJob {
+  __nv_bfloat16* kc = nullptr;
+  __nv_bfloat16* vc = nullptr;
+  const __nv_bfloat16* ks = nullptr;
+  const __nv_bfloat16* vs = nullptr;
+  int cap = 1, slot = 0, rows = 0, src_rows = 0, d = 0, BH = 0;
+};
+
+// One 16-byte piece of a commit: piece `idx` of head bh (row idx / (d/8),
+// 16-byte column chunk idx % (d/8)) of K and of V.
+__device__ __forceinline__ void commit_piece(const CommitJob& j, int bh, int idx) {
+  const int pieces = j.d / 8;
+  const int piece = idx % pieces;
+  const int r = idx / pieces;
+  int dst = j.slot + r;
+  if (dst >= j.cap) dst -= j.cap;  // slot < cap and rows <= cap
+  const size_t so = (static_cast<size_t>(bh) * j.src_rows + r) * j.d + piece * 8;
+  const size_t dso = (static_cast<size_t>(bh) * j.cap + dst) * j.d + piece * 8;
+  *reinterpret_cast<uint4*>(j.kc + dso) = *reinterpret_cast<const uint4*>(j.ks + so);
+  *reinterpret_cast<uint4*>(j.vc + dso) = *reinterpret_cast<const uint4*>(j.vs + so);
+}
+
 // Launchers (return cudaGetLastError() of the launch).
 // tkr/tvr: ring buffer maps; tks/tvs: sink anchor maps (any valid map when
 // the segment is empty)
@@ -87,9 +112,12 @@ cudaError_t launch_fwd(int d, int dm, const CUtensorMap& tq, const CUtensorMap& 
                        const CUtensorMap& tvs, const FwdParams& p, const RopeFreq& rope_om,
                        cudaStream_t s);
 // d: the kernels' head dim (64 or 128); d_io: the caller's (a multiple of 8, <= d)
+// The combine's launch also carries the ring commit `cj` (if cj.rows > 0)
+// in blocks of its own: both only run once the forward has finished, and
+// they touch disjoint memory.
 cudaError_t launch_combine(int d, int d_io, const float* o_part, const float* lse_part,
                            __nv_bfloat16* o, float* lse, int splits, int BH, int rows,
-                           cudaStream_t s);
+                           const CommitJob& cj, cudaStream_t s);
 cudaError_t launch_bwd_pre(int d, int d_io, const __nv_bfloat16* o, const __nv_bfloat16* dout,
                            const float* lse, float* lse2, float* delta, float* dq_acc, int BH,
                            int N, int N_pad, cudaStream_t s);
@@ -102,9 +130,7 @@ cudaError_t launch_bwd_main(int d, int dm, const CUtensorMap& tq, const CUtensor
 cudaError_t launch_bwd_post(int d, int d_io, const float* dq_acc, __nv_bfloat16* dq, float scale,
                             int BH, int N, int N_pad, cudaStream_t s);
 // d: any multiple of 8 (rows are copied in 16-byte pieces)
-cudaError_t launch_commit(int d, __nv_bfloat16* kc, __nv_bfloat16* vc, const __nv_bfloat16* ks,
-                          const __nv_bfloat16* vs, int cap, int slot, int rows, int BH,
-                          cudaStream_t s);
+cudaError_t launch_commit(const CommitJob& j, cudaStream_t s);
 // QKV split + temporal RoPE: qkv [B, N, 3, H, d] -> q, k, v [B, H, N, d]
 // (d a multiple of 8; rope_dims = 0 is a plain split)
 cudaError_t launch_qkv_rope(const __nv_bfloat16* qkv, __nv_bfloat16* q, __nv_bfloat16* k,

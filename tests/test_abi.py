@@ -149,6 +149,22 @@ def test_rope_entry_rejects_bad_rope(mw):
     assert call(first=(1 << 24) - 1, per_frame=440) == INVALID  # ring frames past 2^24
 
 
+def test_step_rejects_bad_commit(mw):
+    lib = mw.library()
+
+    def call(slot=100, rows=880, kc=FAKE):
+        # one 880-token chunk against a full 7040-token ring
+        return lib.mw_bca_cache_step(FAKE, FAKE, FAKE, kc, FAKE, 7040, 0, 7040, slot, rows, FAKE,
+                                     None, None, 0, 1, 2, 1, 880, 64, 0.125, None)
+
+    assert call(rows=-1) == INVALID
+    assert call(rows=881) == INVALID        # more rows than the in-flight chunks hold
+    assert call(slot=7040) == INVALID
+    assert call(slot=-1) == INVALID
+    assert call(kc=MISALIGNED) == INVALID
+    assert call(kc=None) == INVALID
+
+
 def test_commit_rejects_bad_slots(mw):
     lib = mw.library()
 

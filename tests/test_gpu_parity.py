@@ -350,6 +350,31 @@ def test_qkv_split_rope_matches_the_fused_ring_rotation(mw):
     assert torch.equal(o1, o2) and torch.equal(l1, l2)
 
 
+@pytest.mark.parametrize("W,T,cap,length,head,d,splits", [
+    (2, 100, 1000, 1000, 700, 64, 3),    # split-KV: the commit shares the combine's launch
+    (2, 100, 1000, 1000, 700, 64, 1),    # single pass: the commit runs on its own
+    (1, 128, 640, 512, 88, 128, 2),      # ring not yet full; the commit wraps past its end
+])
+def test_cache_step_equals_forward_then_commit(mw, W, T, cap, length, head, d, splits):
+    """mw_bca_cache_step gives bit for bit what mw_bca_cache_fwd followed by
+    mw_bca_cache_commit of the oldest in-flight chunk gives (Sec. 3.5)."""
+    q, kn, vn, kr, vr = (t.cuda() for t in _ring_case(1, 2, W, T, cap, d, seed=cap + d))
+    slot = (head + length) % cap  # append position (evicts nothing until the ring is full)
+    mw.mw_set_option("cache_splits", splits)
+    try:
+        k1, v1 = kr.clone(), vr.clone()
+        o1, l1 = mw.mw_bca_cache_fwd(q, kn, vn, k1, v1, head, length, T)
+        mw.mw_bca_cache_commit(k1, v1, slot, kn[:, :, :T].contiguous(), vn[:, :, :T].contiguous())
+        k2, v2 = kr.clone(), vr.clone()
+        o2, l2 = mw.mw_bca_cache_step(q, kn, vn, k2, v2, head, length, slot, T, T)
+        torch.cuda.synchronize()
+    finally:
+        mw.mw_set_option("cache_splits", 0)
+    assert torch.equal(o1, o2) and torch.equal(l1, l2)
+    assert torch.equal(k1, k2) and torch.equal(v1, v2)
+    assert mw.mw_device_status() == 0
+
+
 def test_rolling_cache_config_steps(mw):
     """The streaming workload: one 880-token chunk against an 8-chunk ring
     whose head wraps mid-buffer; each step commits the chunk (FIFO eviction)."""
