@@ -278,6 +278,20 @@ def time_repeated(fn, reps: int, warmup: int = 3, flush=None):
 
 # ------------------------------------------------------------------ our arm
 
+def run_extras_only(args):
+    """Named secondary workloads alone, on one GPU (for profiling their kernels)."""
+    import paper_2608_01127_gb300 as mw
+
+    names = [n.strip() for n in args.extras_only.split(",") if n.strip()]
+    unknown = [n for n in names if n not in EXTRA_NAMES]
+    if unknown:
+        raise SystemExit(f"unknown secondary workloads: {unknown}")
+    torch.cuda.set_device(0)
+    dev = torch.device("cuda", 0)
+    extra = run_extras(mw, dev, load_peaks(), only=names)
+    print(json.dumps({"extras_only": names, "extra": extra}), flush=True)
+
+
 def run_ours(args):
     import paper_2608_01127_gb300 as mw
 
@@ -366,10 +380,14 @@ def run_ours(args):
                    "flops_per_step": step_flops, "unmasked_pairs": pairs,
                    "l2": "256 MiB buffer written between timed steps (outside the events)"},
         "frac_of_bf16_peak": round(value / world / peaks["bf16_tflops"], 4),
+        "frac_of_bf16_sustained": round(value / world / peaks["bf16_tflops_sustained"], 4),
+        "ms_per_step_median": round(statistics.median(step_ms), 4),
+        "ms_per_step_min": round(min(step_ms), 4),
         "roofline": {"kernel": f"bca_bwd_kernel<{cfg.d}, {cfg.d}> (backward key-tile kernel)", "bound": "tensor",
                      "achieved": round(achieved, 2), "peak": peaks["bf16_tflops"],
                      "peak_source": peaks["source"] + " bf16 burst", "unit": "TFLOP/s",
                      "frac": round(achieved / peaks["bf16_tflops"], 4),
+                     "frac_of_sustained": round(achieved / peaks["bf16_tflops_sustained"], 4),
                      "traffic": profiled_traffic(f"bca_bwd_kernel<{cfg.d},{cfg.d}>", workload),
                      "algorithmic_bytes": bwd_main_bytes(cfg),
                      "ms_per_launch": round(main_ms, 4)},
@@ -499,15 +517,23 @@ def run_e2e(mw, cfg, dev, args, world, step_flops):
                        "during step i's compute (double-buffered device sets)"}
 
 
-def run_extras(mw, dev, peaks):
+EXTRA_NAMES = ("train_h16_d128_peaky", "train_1b_32x600", "train_05b_d72", "rolling_cache",
+               "pipelined", "sink_anchor", "qkv_rope_split")
+
+
+def run_extras(mw, dev, peaks, only=None):
+    """The secondary workloads (all, or the names in `only`)."""
     flush_buf = torch.empty(L2_FLUSH_BYTES, dtype=torch.uint8, device=dev)
     flush = flush_buf.zero_
     extra = {}
+    want = set(EXTRA_NAMES if only is None else only)
     # forward / backward of the other training workloads: d=128 with peaky
     # logits, the paper's 32-chunk window of 600-token chunks at the
     # MiniWorld-1B head layout (12 heads of 128), and the 0.5B head dim (72,
     # run on the 128-wide kernels with zero-filled columns)
     for name in ("train_h16_d128_peaky", "train_1b_32x600", "train_05b_d72"):
+        if name not in want:
+            continue
         cfg = TRAIN_CONFIGS[name]
         x = gen_train(cfg)
         q, k, v, do = (x[n].to(dev) for n in ("q", "k", "v", "do"))
@@ -526,10 +552,14 @@ def run_extras(mw, dev, peaks):
             "fwd_bwd_tflops": round((fwd_flops(pairs, cfg.d) + bwd_flops(pairs, cfg.d))
                                     / (fm + bm) / 1e9, 2)}
         del q, k, v, do, o, lse, ws, grads
-    extra["rolling_cache"] = bench_rolling(mw, dev, peaks)
-    extra["pipelined"] = bench_pipelined(mw, dev, peaks, flush)
-    extra["sink_anchor"] = bench_sink(mw, dev, peaks, flush)
-    extra["qkv_rope_split"] = bench_qkv_split(mw, dev, peaks, flush)
+    if "rolling_cache" in want:
+        extra["rolling_cache"] = bench_rolling(mw, dev, peaks)
+    if "pipelined" in want:
+        extra["pipelined"] = bench_pipelined(mw, dev, peaks, flush)
+    if "sink_anchor" in want:
+        extra["sink_anchor"] = bench_sink(mw, dev, peaks, flush)
+    if "qkv_rope_split" in want:
+        extra["qkv_rope_split"] = bench_qkv_split(mw, dev, peaks, flush)
     return extra
 
 
@@ -781,6 +811,10 @@ def main(argv=None):
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", choices=("ours", "reference"), default="ours")
     ap.add_argument("--no-extras", action="store_true", help="skip the secondary workloads")
+    ap.add_argument("--extras-only", default=None,
+                    help="comma-separated secondary workloads to run alone, without the "
+                         "headline step (profiling; prints their results only): "
+                         + ", ".join(EXTRA_NAMES))
     ap.add_argument("--workload", choices=sorted(n for n, c in TRAIN_CONFIGS.items() if c.backward),
                     default=WORKLOAD,
                     help="training workload of the timed step (default: the headline one)")
@@ -796,6 +830,8 @@ def main(argv=None):
         ap.error(f"--gpus {args.gpus} but WORLD_SIZE={world}")
     if args.impl == "reference":
         run_reference(args)
+    elif args.extras_only:
+        run_extras_only(args)
     else:
         run_ours(args)
 
