@@ -392,6 +392,8 @@ mw_status mw_set_option(const char* name, long long value) {
     g_opt_budget_ms = value;
   } else if (std::strcmp(name, "debug_skip_q_load") == 0) {
     g_opt_skip_q = value;
+  } else if (std::strcmp(name, "pdl") == 0) {
+    mw::g_pdl_enabled = value != 0;
   } else {
     return fail(MW_ERR_INVALID_ARG, "unknown option '%s'", name);
   }

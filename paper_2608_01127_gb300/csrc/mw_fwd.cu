@@ -220,6 +220,9 @@ __global__ void __launch_bounds__(FwdLayout<D, DM>::THREADS, 1)
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
   const WaitCtl ctl{abort_flag, p.status, p.budget_ns};
+  // launched early (programmatic dependent launch): the setup above has run
+  // while the previous kernel finished; global memory only from here on
+  pdl_wait();
 
   uint8_t* sQ = smem + L::OFF_Q;
   uint8_t* sK = smem + L::OFF_K;
@@ -600,6 +603,7 @@ __global__ void __launch_bounds__(FwdLayout<D, DM>::THREADS, 1)
     }
 
     // ---- epilogue
+    pdl_trigger();  // the next kernel (the split combine) may be scheduled now
     const bool have = __all_sync(0xffffffffu, ok) && n_steps > 0 && warp_wait(o_full, 0, ctl);
     tc_fence_after();
     if constexpr (L::SUM_MMA) {
@@ -675,6 +679,8 @@ __global__ void __launch_bounds__(256) combine_kernel(const float* __restrict__ 
                                                       float* __restrict__ lse, int splits,
                                                       int n_rows, int d_io_arg,
                                                       const CommitJob cj) {
+  pdl_wait();     // the forward's partials (and its reads of the ring) are complete
+  pdl_trigger();  // the next step's forward may start its setup meanwhile
   const int combine_blocks = (n_rows + 7) / 8;
   if (static_cast<int>(blockIdx.x) >= combine_blocks) {
     const long long idx =
@@ -745,9 +751,10 @@ cudaError_t launch_fwd_t(const CUtensorMap& tq, const CUtensorMap& tk, const CUt
     attr_set = true;
   }
   const unsigned grid = static_cast<unsigned>(p.BH) * p.n_qblocks * p.num_splits;
-  bca_fwd_kernel<D, DM, ROPE><<<grid, L::THREADS, L::BYTES, s>>>(tq, tk, tv, tkr, tvr, tks, tvs, p,
-                                                              om);
-  return cudaGetLastError();
+  cudaLaunchConfig_t cfg;
+  cudaLaunchAttribute attr;
+  pdl_config(cfg, attr, dim3(grid), dim3(L::THREADS), L::BYTES, s);
+  return cudaLaunchKernelEx(&cfg, bca_fwd_kernel<D, DM, ROPE>, tq, tk, tv, tkr, tvr, tks, tvs, p, om);
 }
 
 }  // namespace
@@ -772,12 +779,14 @@ cudaError_t launch_combine(int d, int d_io, const float* o_part, const float* ls
   const int n_rows = BH * rows;
   const long long commit_pieces = static_cast<long long>(cj.rows) * (cj.d / 8) * cj.BH;
   const long long blocks = (n_rows + 7) / 8 + (commit_pieces + 255) / 256;
-  const unsigned grid = static_cast<unsigned>(blocks);
+  cudaLaunchConfig_t cfg;
+  cudaLaunchAttribute attr;
+  pdl_config(cfg, attr, dim3(static_cast<unsigned>(blocks)), dim3(256), 0, s);
   if (d == 64)
-    combine_kernel<64><<<grid, 256, 0, s>>>(o_part, lse_part, o, lse, splits, n_rows, d_io, cj);
-  else
-    combine_kernel<128><<<grid, 256, 0, s>>>(o_part, lse_part, o, lse, splits, n_rows, d_io, cj);
-  return cudaGetLastError();
+    return cudaLaunchKernelEx(&cfg, combine_kernel<64>, o_part, lse_part, o, lse, splits, n_rows,
+                              d_io, cj);
+  return cudaLaunchKernelEx(&cfg, combine_kernel<128>, o_part, lse_part, o, lse, splits, n_rows,
+                            d_io, cj);
 }
 
 }  // namespace mw

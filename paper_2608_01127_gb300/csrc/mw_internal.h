@@ -102,6 +102,24 @@ __device__ __forceinline__ void commit_piece(const CommitJob& j, int bh, int idx
   *reinterpret_cast<uint4*>(j.vc + dso) = *reinterpret_cast<const uint4*>(j.vs + so);
 }
 
+// Programmatic dependent launch of the forward, the split combine and the
+// commit (option "pdl", on by default): each may start while the previous
+// kernel in the stream finishes and waits in-kernel before touching global
+// memory.  pdl_config fills `cfg` (and its one attribute `attr`).
+extern int g_pdl_enabled;
+inline void pdl_config(cudaLaunchConfig_t& cfg, cudaLaunchAttribute& attr, dim3 grid, dim3 block,
+                       size_t smem, cudaStream_t s) {
+  cfg = cudaLaunchConfig_t{};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = s;
+  attr.id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr.val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = &attr;
+  cfg.numAttrs = g_pdl_enabled ? 1 : 0;
+}
+
 // Launchers (return cudaGetLastError() of the launch).
 // tkr/tvr: ring buffer maps; tks/tvs: sink anchor maps (any valid map when
 // the segment is empty)

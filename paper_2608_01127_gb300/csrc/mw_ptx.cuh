@@ -356,6 +356,16 @@ __device__ __forceinline__ float ex2_approx(float x) {
   return y;
 }
 
+// Programmatic dependent launch: a kernel launched with programmatic
+// stream serialization may start while the previous kernel in the stream
+// finishes; pdl_wait blocks until that kernel has completed and its memory
+// is visible (a no-op for a kernel launched without the attribute), and
+// pdl_trigger lets the next such kernel be scheduled early.
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+__device__ __forceinline__ void pdl_trigger() {
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+
 // Packed fp32 pair arithmetic (one instruction for two lanes of work).
 __device__ __forceinline__ float2 fma2(float2 a, float2 b, float2 c) {
   uint64_t d;
