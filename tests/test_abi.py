@@ -209,6 +209,8 @@ def test_options(mw):
     assert lib.mw_set_option(b"cache_splits", 99) == INVALID
     assert lib.mw_set_option(b"wait_budget_ms", 0) == INVALID
     assert lib.mw_set_option(b"cache_splits", 0) == OK
+    assert lib.mw_set_option(b"pdl", 0) == OK
+    assert lib.mw_set_option(b"pdl", 1) == OK
 
 
 def test_workspace_follows_split_override(mw):

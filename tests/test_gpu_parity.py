@@ -375,6 +375,38 @@ def test_cache_step_equals_forward_then_commit(mw, W, T, cap, length, head, d, s
     assert mw.mw_device_status() == 0
 
 
+def test_programmatic_launch_changes_nothing(mw):
+    """Forward, streaming step and backward give the same bits with the
+    programmatic dependent launch on and off (only the launch overlaps)."""
+    q, kn, vn, kr, vr = (t.cuda() for t in _ring_case(1, 2, 2, 100, 1000, 64, seed=23))
+    g = torch.Generator().manual_seed(24)
+    do = torch.randn(1, 2, 200, 64, generator=g).to(torch.bfloat16).cuda()
+    runs = []
+    try:
+        for pdl in (1, 0):
+            mw.mw_set_option("pdl", pdl)
+            mw.mw_set_option("cache_splits", 3)
+            k1, v1 = kr.clone(), vr.clone()
+            o_c, l_c = mw.mw_bca_cache_step(q, kn, vn, k1, v1, 700, 1000, 700, 100, 100)
+            o, lse = mw.mw_bca_fwd(q, kn, vn, 100)
+            grads = mw.mw_bca_bwd(q, kn, vn, o, lse, do, 100)
+            torch.cuda.synchronize()
+            runs.append((o_c, l_c, k1, v1, o, lse))
+            runs[-1] += tuple(grads)
+    finally:
+        mw.mw_set_option("pdl", 1)
+        mw.mw_set_option("cache_splits", 0)
+    # dQ accumulates with floating-point atomics in no fixed order: compare it
+    # to within rounding, everything else bit for bit
+    for a, b in zip(runs[0][:-3], runs[1][:-3]):
+        assert torch.equal(a, b)
+    dq0, dq1 = runs[0][-3].double(), runs[1][-3].double()
+    assert float((dq0 - dq1).norm() / dq0.norm()) < 1e-3
+    for a, b in zip(runs[0][-2:], runs[1][-2:]):
+        assert torch.equal(a, b)
+    assert mw.mw_device_status() == 0
+
+
 def test_rolling_cache_config_steps(mw):
     """The streaming workload: one 880-token chunk against an 8-chunk ring
     whose head wraps mid-buffer; each step commits the chunk (FIFO eviction)."""
