@@ -6,14 +6,19 @@ training path) over the workload B=2, H=12, d=64, 16 chunks x 880 tokens
 (N = 14080), bf16, synthetic N(0,1) inputs.  `value` is TFLOP/s counted over
 unmasked (query, key) pairs only: fwd 4*d*pairs + bwd 10*d*pairs.
 
-Also reported in the same JSON line: the roofline of the dominant kernel
-(backward key-tile kernel, timed with CUDA events around it), an end-to-end
-number through the C ABI with pinned host buffers, the fp64 oracle on the
-host cores (cpu_baseline), and secondary workloads (forward only, the
-d=128 peaky config, the rolling-KV-cache streaming step and the pipelined
-4-chunk window).
+Also reported in the same JSON line: the fractions of the measured bf16
+peak (burst and sustained), the median and minimum step time, the roofline
+of the dominant kernel (backward key-tile kernel, timed with CUDA events
+around it, with its ncu DRAM traffic while the sources match the profiled
+build), an end-to-end number through the C ABI with pinned host buffers,
+SM clocks sampled during the timed region, the fp64 oracle on the host
+cores (cpu_baseline), and secondary workloads (the d=128 peaky config, the
+paper's 32 x 600 window, the d=72 layout, the rolling-KV-cache streaming
+step, the pipelined 4-chunk window, the sink anchor with and without the
+RoPE re-shift, and the QKV-RoPE split).
 
     python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+    python bench.py --extras-only rolling_cache[,pipelined,...]   # profiling
 
 Under torchrun (N > 1) every rank runs its own batch of the same workload
 (independent problems: weak scaling, no collective on the data path); the
