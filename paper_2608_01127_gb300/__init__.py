@@ -124,13 +124,78 @@ def _ptr(t: Optional[torch.Tensor]) -> Optional[int]:
 
 
 def _bhnd(t: torch.Tensor, name: str) -> Tuple[int, int, int, int]:
+    """Shape of a contiguous bf16 [B, H, rows, d] tensor (its device is
+    checked by _on_device, once every shape is known to be right)."""
+    if not isinstance(t, torch.Tensor):
+        raise TypeError(f"{name} must be a torch.Tensor, got {type(t).__name__}")
     if t.dtype != torch.bfloat16:
         raise TypeError(f"{name} must be bfloat16, got {t.dtype}")
-    if not t.is_cuda:
-        raise ValueError(f"{name} must be a CUDA tensor (there is no CPU path)")
     if t.dim() != 4 or not t.is_contiguous():
         raise ValueError(f"{name} must be a contiguous [B, H, rows, d] tensor")
     return tuple(t.shape)  # type: ignore[return-value]
+
+
+def _expect(t, name: str, shape, dtype=torch.bfloat16) -> None:
+    """A caller-supplied output buffer: exactly this shape and dtype,
+    contiguous.  The library cannot see buffer sizes, so a short buffer
+    would be written past its end."""
+    if not isinstance(t, torch.Tensor) or t.dtype != dtype or not t.is_contiguous() \
+            or tuple(t.shape) != tuple(shape):
+        got = (f"{t.dtype} {tuple(t.shape)}" + ("" if t.is_contiguous() else " non-contiguous")
+               if isinstance(t, torch.Tensor) else type(t).__name__)
+        raise ValueError(f"{name} must be a contiguous {dtype} tensor of shape {tuple(shape)}, "
+                         f"got {got}")
+
+
+def _chunks(rows: int, T_chunk: int, what: str) -> int:
+    if int(T_chunk) < 1:
+        raise ValueError(f"T_chunk must be >= 1, got {T_chunk}")
+    if rows % T_chunk != 0:
+        raise ValueError(f"{what} {rows} is not a multiple of T_chunk={T_chunk}")
+    return rows // T_chunk
+
+
+def _on_device(ref: torch.Tensor, named) -> None:
+    """Every tensor on ref's CUDA device, and that device current (the
+    library launches on the current device and stream)."""
+    if not ref.is_cuda:
+        raise ValueError("the tensors must be CUDA tensors (there is no CPU path)")
+    for name, t in named:
+        if t is not None and t.device != ref.device:
+            raise ValueError(f"{name} is on {t.device}, the other tensors on {ref.device}")
+    if ref.device.index != torch.cuda.current_device():
+        raise ValueError(f"the tensors are on {ref.device} but the current device is "
+                         f"cuda:{torch.cuda.current_device()}: call under torch.cuda.device")
+
+
+def _no_alias(outputs, inputs) -> None:
+    """No output buffer shares bytes with an input or with another output
+    (the kernels read inputs while they write outputs)."""
+    spans = []
+    for kind, group in (("output", outputs), ("input", inputs)):
+        for name, t in group:
+            if t is not None and t.numel() > 0:
+                p = t.data_ptr()
+                spans.append((f"{kind} {name}", p, p + t.numel() * t.element_size()))
+    n_out = sum(1 for _, t in outputs if t is not None and t.numel() > 0)
+    for a in range(n_out):
+        for b in range(a + 1, len(spans)):
+            if spans[a][1] < spans[b][2] and spans[b][1] < spans[a][2]:
+                raise ValueError(f"{spans[a][0]} overlaps {spans[b][0]}")
+
+
+def _workspace(ws: Optional[torch.Tensor], nbytes: int,
+               device: torch.device) -> Optional[torch.Tensor]:
+    """At least nbytes of device scratch (None when none is needed): the
+    caller's buffer when it is large enough, else a new one."""
+    if nbytes == 0:
+        return None
+    if ws is not None:
+        if not ws.is_contiguous():
+            raise ValueError("workspace must be contiguous")
+        if ws.numel() * ws.element_size() >= nbytes:
+            return ws
+    return torch.empty(nbytes, dtype=torch.uint8, device=device)
 
 
 def _scale(scale: Optional[float], d: int) -> float:
@@ -148,16 +213,20 @@ def mw_bca_fwd(q: torch.Tensor, k: torch.Tensor, v: torch.Tensor, T_chunk: int,
     for t, n in ((k, "k"), (v, "v")):
         if _bhnd(t, n) != (B, H, N, d):
             raise ValueError(f"{n} shape {tuple(t.shape)} != q shape {(B, H, N, d)}")
-    if N % T_chunk != 0:
-        raise ValueError(f"sequence length {N} is not a multiple of T_chunk={T_chunk}")
+    n_chunks = _chunks(N, T_chunk, "sequence length")
+    o, lse = out if out is not None else (None, None)
     if out is not None:
-        o, lse = out
-        _bhnd(o, "o")
-    else:
+        _expect(o, "o", (B, H, N, d))
+        if lse is not None:
+            _expect(lse, "lse", (B, H, N), torch.float32)
+    _on_device(q, (("k", k), ("v", v), ("o", o), ("lse", lse)))
+    if out is None:
         o = torch.empty_like(q)
         lse = torch.empty((B, H, N), dtype=torch.float32, device=q.device) if need_lse else None
+    else:
+        _no_alias((("o", o), ("lse", lse)), (("q", q), ("k", k), ("v", v)))
     _check(library().mw_bca_fwd(_ptr(q), _ptr(k), _ptr(v), _ptr(o), _ptr(lse), B, H,
-                                N // T_chunk, T_chunk, d, _scale(scale, d), _stream()))
+                                n_chunks, T_chunk, d, _scale(scale, d), _stream()))
     return o, lse
 
 
@@ -175,19 +244,20 @@ def mw_bca_bwd(q, k, v, o, lse, dout, T_chunk: int, scale: Optional[float] = Non
     for t, n in ((k, "k"), (v, "v"), (o, "o"), (dout, "dout")):
         if _bhnd(t, n) != (B, H, N, d):
             raise ValueError(f"{n} shape {tuple(t.shape)} != q shape {(B, H, N, d)}")
-    if lse is None or lse.dtype != torch.float32 or tuple(lse.shape) != (B, H, N) \
-            or not lse.is_contiguous():
-        raise ValueError("lse must be a contiguous fp32 [B, H, N] tensor")
-    if N % T_chunk != 0:
-        raise ValueError(f"sequence length {N} is not a multiple of T_chunk={T_chunk}")
-    n = N // T_chunk
+    _expect(lse, "lse", (B, H, N), torch.float32)
+    n = _chunks(N, T_chunk, "sequence length")
+    dq, dk, dv = out if out is not None else (None, None, None)
+    if out is not None:
+        for t, name in ((dq, "dq"), (dk, "dk"), (dv, "dv")):
+            _expect(t, name, (B, H, N, d))
+    _on_device(q, (("k", k), ("v", v), ("o", o), ("lse", lse), ("dout", dout), ("dq", dq),
+                   ("dk", dk), ("dv", dv), ("workspace", workspace)))
     ws_bytes = mw_bca_bwd_workspace_size(B, H, n, T_chunk, d)
-    if workspace is None or workspace.numel() < ws_bytes:
-        workspace = torch.empty(ws_bytes, dtype=torch.uint8, device=q.device)
+    workspace = _workspace(workspace, ws_bytes, q.device)
     if out is None:
         dq, dk, dv = torch.empty_like(q), torch.empty_like(k), torch.empty_like(v)
-    else:
-        dq, dk, dv = out
+    _no_alias((("dq", dq), ("dk", dk), ("dv", dv), ("workspace", workspace)),
+              (("q", q), ("k", k), ("v", v), ("o", o), ("lse", lse), ("dout", dout)))
     _check(library().mw_bca_bwd_stage(stage, _ptr(q), _ptr(k), _ptr(v), _ptr(o), _ptr(lse),
                                       _ptr(dout), _ptr(dq), _ptr(dk), _ptr(dv), _ptr(workspace),
                                       ws_bytes, B, H, n, T_chunk, d, _scale(scale, d), _stream()))
@@ -240,43 +310,51 @@ def _cache_fwd(q, k_new, v_new, k_sink, v_sink, k_cache, v_cache, cache_head, ca
     if (Bc, Hc, dc) != (B, H, d) or tuple(v_cache.shape) != tuple(k_cache.shape):
         raise ValueError("k_cache / v_cache must be [B, H, cap, d] matching q")
     _bhnd(v_cache, "v_cache")
-    if M % T_chunk != 0:
-        raise ValueError(f"{M} query rows is not a multiple of T_chunk={T_chunk}")
-    W = M // T_chunk
+    W = _chunks(M, T_chunk, "query rows")
     sink_len = 0
     if k_sink is not None:
         Bs, Hs, sink_len, ds = _bhnd(k_sink, "k_sink")
         _bhnd(v_sink, "v_sink")
         if (Bs, Hs, ds) != (B, H, d) or tuple(v_sink.shape) != tuple(k_sink.shape):
             raise ValueError("k_sink / v_sink must be [B, H, S, d] matching q")
+    if out is not None:
+        _expect(out, "out", (B, H, M, d))
+    _on_device(q, (("k_new", k_new), ("v_new", v_new), ("k_cache", k_cache),
+                   ("v_cache", v_cache), ("k_sink", k_sink), ("v_sink", v_sink), ("out", out),
+                   ("workspace", workspace)))
     ws_bytes = mw_bca_cache_workspace_size(B, H, W, T_chunk, d, sink_len + cache_len)
-    if ws_bytes and (workspace is None or workspace.numel() < ws_bytes):
-        workspace = torch.empty(ws_bytes, dtype=torch.uint8, device=q.device)
+    workspace = _workspace(workspace, ws_bytes, q.device)
     o = torch.empty_like(q) if out is None else out
     lse = torch.empty((B, H, M), dtype=torch.float32, device=q.device) if need_lse else None
+    # the streaming step also writes the ring (its commit)
+    ring = (("k_cache", k_cache), ("v_cache", v_cache))
+    _no_alias((("out", o), ("lse", lse), ("workspace", workspace))
+              + (ring if commit is not None else ()),
+              (("q", q), ("k_new", k_new), ("v_new", v_new), ("k_sink", k_sink),
+               ("v_sink", v_sink)) + (ring if commit is None else ()))
     if commit is not None:
         _check(library().mw_bca_cache_step(
             _ptr(q), _ptr(k_new), _ptr(v_new), _ptr(k_cache), _ptr(v_cache), cap, cache_head,
             cache_len, int(commit[0]), int(commit[1]), _ptr(o), _ptr(lse),
-            _ptr(workspace) if ws_bytes else None, ws_bytes, B, H, W, T_chunk, d,
+            _ptr(workspace), ws_bytes, B, H, W, T_chunk, d,
             _scale(scale, d), _stream()))
     elif rope is not None:
         _check(library().mw_bca_cache_fwd_rope(
             _ptr(q), _ptr(k_new), _ptr(v_new), _ptr(k_sink), _ptr(v_sink), sink_len,
             _ptr(k_cache), _ptr(v_cache), cap, cache_head, cache_len, int(rope[0]),
             float(rope[1]), int(rope[2]), int(rope[3]), _ptr(o), _ptr(lse),
-            _ptr(workspace) if ws_bytes else None, ws_bytes, B, H, W, T_chunk, d,
+            _ptr(workspace), ws_bytes, B, H, W, T_chunk, d,
             _scale(scale, d), _stream()))
     elif k_sink is None:
         _check(library().mw_bca_cache_fwd(
             _ptr(q), _ptr(k_new), _ptr(v_new), _ptr(k_cache), _ptr(v_cache), cap, cache_head,
-            cache_len, _ptr(o), _ptr(lse), _ptr(workspace) if ws_bytes else None, ws_bytes,
+            cache_len, _ptr(o), _ptr(lse), _ptr(workspace), ws_bytes,
             B, H, W, T_chunk, d, _scale(scale, d), _stream()))
     else:
         _check(library().mw_bca_cache_fwd_sink(
             _ptr(q), _ptr(k_new), _ptr(v_new), _ptr(k_sink), _ptr(v_sink), sink_len,
             _ptr(k_cache), _ptr(v_cache), cap, cache_head, cache_len, _ptr(o), _ptr(lse),
-            _ptr(workspace) if ws_bytes else None, ws_bytes, B, H, W, T_chunk, d,
+            _ptr(workspace), ws_bytes, B, H, W, T_chunk, d,
             _scale(scale, d), _stream()))
     return o, lse
 
@@ -301,6 +379,10 @@ def mw_bca_cache_commit(k_cache, v_cache, slot_start: int, k_src, v_src) -> None
     _bhnd(v_src, "v_src")
     if (Bs, Hs, ds) != (B, H, d) or tuple(v_src.shape) != tuple(k_src.shape):
         raise ValueError("k_src / v_src must be [B, H, rows, d] matching the cache")
+    if tuple(v_cache.shape) != (B, H, cap, d):
+        raise ValueError("k_cache / v_cache must have the same shape")
+    _on_device(k_cache, (("v_cache", v_cache), ("k_src", k_src), ("v_src", v_src)))
+    _no_alias((("k_cache", k_cache), ("v_cache", v_cache)), (("k_src", k_src), ("v_src", v_src)))
     _check(library().mw_bca_cache_commit(_ptr(k_cache), _ptr(v_cache), cap, slot_start,
                                          _ptr(k_src), _ptr(v_src), rows, B, H, d, _stream()))
 
@@ -313,20 +395,22 @@ def mw_qkv_rope_split(qkv: torch.Tensor, rope_dims: int = 0, rope_base: float = 
     [B, H, N, d], turning the first ``rope_dims`` channels of Q and K by their
     frame's temporal rotary angle (token t at frame first_frame + t //
     tokens_per_frame; Sec. 3.2 inputs, Sec. 3.5 positions)."""
-    if qkv.dtype != torch.bfloat16:
-        raise TypeError(f"qkv must be bfloat16, got {qkv.dtype}")
-    if not qkv.is_cuda:
-        raise ValueError("qkv must be a CUDA tensor (there is no CPU path)")
+    if not isinstance(qkv, torch.Tensor) or qkv.dtype != torch.bfloat16:
+        raise TypeError("qkv must be a bfloat16 tensor")
     if qkv.dim() != 5 or qkv.shape[2] != 3 or not qkv.is_contiguous():
         raise ValueError("qkv must be a contiguous [B, N, 3, H, d] tensor")
     B, N, _, H, d = qkv.shape
+    if out is not None:
+        if len(out) != 3:
+            raise ValueError("out must be (q, k, v)")
+        for t, name in zip(out, ("q", "k", "v")):
+            _expect(t, name, (B, H, N, d))
+    _on_device(qkv, tuple(zip(("q", "k", "v"), out)) if out is not None else ())
     if out is None:
         out = tuple(torch.empty(B, H, N, d, dtype=torch.bfloat16, device=qkv.device)
                     for _ in range(3))
-    for t, name in zip(out, ("q", "k", "v")):
-        if tuple(_bhnd(t, name)) != (B, H, N, d):
-            raise ValueError(f"{name} must be [B, H, N, d] = {(B, H, N, d)}")
     q, k, v = out
+    _no_alias((("q", q), ("k", k), ("v", v)), (("qkv", qkv),))
     _check(library().mw_qkv_rope_split(_ptr(qkv), _ptr(q), _ptr(k), _ptr(v), B, N, H, d,
                                        int(rope_dims), float(rope_base), int(tokens_per_frame),
                                        int(first_frame), _stream()))

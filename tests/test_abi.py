@@ -229,3 +229,86 @@ def test_python_binding_has_no_cpu_path(mw):
     q = torch.zeros(1, 1, 64, 64, dtype=torch.bfloat16)
     with pytest.raises(ValueError):
         mw.mw_bca_fwd(q, q, q, 64)
+
+
+def _bf(*shape):
+    return torch.zeros(*shape, dtype=torch.bfloat16)
+
+
+def test_python_binding_checks_every_buffer_before_the_device(mw):
+    """The library cannot see buffer sizes, so the binding checks the shape,
+    dtype and layout of every argument, caller-supplied outputs included, and
+    the chunking, before anything is launched.  The device comes last: CPU
+    tensors that pass every other check still get no CPU path."""
+    q = _bf(1, 2, 128, 64)
+    lse = torch.zeros(1, 2, 128)
+    ring = _bf(1, 2, 512, 64)
+    qkv = _bf(1, 128, 3, 2, 64)
+    strided = _bf(1, 2, 64, 128).transpose(2, 3)   # [1, 2, 128, 64], not contiguous
+    cases = [
+        (lambda: mw.mw_bca_fwd(q, q, q, 0), "T_chunk must be >= 1"),
+        (lambda: mw.mw_bca_fwd(q, q, q, 48), "not a multiple of T_chunk"),
+        (lambda: mw.mw_bca_fwd(q, q, q, 64, out=(_bf(1, 2, 64, 64), None)), "o must be"),
+        (lambda: mw.mw_bca_fwd(q, q, q, 64, out=(strided, None)), "o must be"),
+        (lambda: mw.mw_bca_fwd(q, q, q, 64, out=(_bf(1, 2, 128, 64), lse.double())),
+         "lse must be"),
+        (lambda: mw.mw_bca_fwd(q, q, q, 64, out=(_bf(1, 2, 128, 64), lse[:, :, :64])),
+         "lse must be"),
+        (lambda: mw.mw_bca_bwd(q, q, q, q, lse.double(), q, 64), "lse must be"),
+        (lambda: mw.mw_bca_bwd(q, q, q, q, lse, q, -64), "T_chunk must be >= 1"),
+        (lambda: mw.mw_bca_bwd(q, q, q, q, lse, q, 64,
+                               out=(_bf(1, 2, 128, 64), _bf(1, 2, 128, 64), _bf(1, 2, 128, 32))),
+         "dv must be"),
+        (lambda: mw.mw_bca_bwd(q, q, q, q, lse, q, 64,
+                               out=(strided, _bf(1, 2, 128, 64), _bf(1, 2, 128, 64))),
+         "dq must be"),
+        (lambda: mw.mw_bca_cache_fwd(q, q, q, ring, ring, 0, 256, 64, out=_bf(1, 2, 64, 64)),
+         "out must be"),
+        (lambda: mw.mw_bca_cache_fwd(q, q, q, ring, ring, 0, 256, 0), "T_chunk must be >= 1"),
+        (lambda: mw.mw_bca_cache_step(q, q, q, ring, ring, 0, 256, 256, 64, 64,
+                                      out=torch.zeros(1, 2, 128, 64)), "out must be"),
+        (lambda: mw.mw_bca_cache_commit(ring, _bf(1, 2, 256, 64), 0, q, q), "same shape"),
+        (lambda: mw.mw_qkv_rope_split(qkv, out=(q, q)), "out must be"),
+        (lambda: mw.mw_qkv_rope_split(qkv, out=(q, q, _bf(2, 2, 128, 64))), "v must be"),
+        # everything right but the device
+        (lambda: mw.mw_bca_fwd(q, q, q, 64), "CUDA tensors"),
+        (lambda: mw.mw_bca_bwd(q, q, q, q, lse, q, 64), "CUDA tensors"),
+        (lambda: mw.mw_bca_cache_fwd(q, q, q, ring, ring, 0, 256, 64), "CUDA tensors"),
+        (lambda: mw.mw_bca_cache_commit(ring, ring, 0, q, q), "CUDA tensors"),
+        (lambda: mw.mw_qkv_rope_split(qkv), "CUDA tensors"),
+    ]
+    for fn, msg in cases:
+        with pytest.raises(ValueError, match=msg):
+            fn()
+    with pytest.raises(TypeError):
+        mw.mw_bca_fwd(q, q.float(), q, 64)
+    with pytest.raises(TypeError):
+        mw.mw_bca_cache_fwd_sink(q, q, q, _bf(1, 2, 64, 64), None, ring, ring, 0, 256, 64)
+
+
+def test_alias_check(mw):
+    """Outputs may share no byte with an input or with another output."""
+    from paper_2608_01127_gb300 import _no_alias
+    buf = torch.zeros(4, 100, dtype=torch.bfloat16)
+    a, b, c = buf[0], buf[1], buf[2]
+    _no_alias((("o", a), ("lse", b)), (("q", c), ("k", c), ("none", None)))  # inputs may share
+    with pytest.raises(ValueError, match="output o overlaps input q"):
+        _no_alias((("o", a),), (("q", buf[0, 50:]),))
+    with pytest.raises(ValueError, match="output dq overlaps output dk"):
+        _no_alias((("dq", buf[1:3].reshape(-1)), ("dk", buf[2])), (("q", a),))
+    # adjacent but disjoint byte ranges are fine
+    _no_alias((("o", buf[0, :50]),), (("q", buf[0, 50:]),))
+    _no_alias((("o", buf[0, :0]),), (("q", buf[0]),))                      # empty output
+
+
+def test_workspace_is_counted_in_bytes(mw):
+    from paper_2608_01127_gb300 import _workspace
+    cpu = torch.device("cpu")
+    assert _workspace(torch.zeros(4), 0, cpu) is None                      # none needed
+    ws = torch.zeros(4, dtype=torch.float32)                               # 16 bytes
+    assert _workspace(ws, 16, cpu) is ws
+    grown = _workspace(ws, 17, cpu)
+    assert grown is not ws and grown.dtype == torch.uint8 and grown.numel() == 17
+    assert _workspace(None, 8, cpu).numel() == 8
+    with pytest.raises(ValueError, match="contiguous"):
+        _workspace(torch.zeros(8, 2)[:, 0], 4, cpu)
