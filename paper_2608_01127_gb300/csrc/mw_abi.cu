@@ -228,16 +228,35 @@ size_t cache_ws_bytes(int splits, int BH, int rows_q, int d) {
 }
 
 struct BwdWs {
-  size_t dq_acc, lse2, delta, total;
+  size_t dq_acc, lse2, delta, bias, total;
 };
 
+// d = 64 adds the bias rows of the MMA-folded LSE and D terms: 8 floats
+// (32 bytes) per padded row
 BwdWs bwd_ws_layout(int BH, int N_pad, int d) {
   BwdWs w;
   w.dq_acc = 0;
   w.lse2 = align256(static_cast<size_t>(BH) * N_pad * d * sizeof(float));
   w.delta = w.lse2 + align256(static_cast<size_t>(BH) * N_pad * sizeof(float));
-  w.total = w.delta + align256(static_cast<size_t>(BH) * N_pad * sizeof(float));
+  w.bias = w.delta + align256(static_cast<size_t>(BH) * N_pad * sizeof(float));
+  w.total = w.bias + (d == 64 ? align256(static_cast<size_t>(BH) * N_pad * 8 * sizeof(float)) : 0);
   return w;
+}
+
+// 3-D map over the bias rows [BH, N_pad, 8] f32: 8 x box_rows boxes with the
+// 32-byte swizzle the tf32 MMA descriptors read
+mw_status encode_bias_map(CUtensorMap* m, const float* bias, int N_pad, int BH, int box_rows) {
+  auto fn = encode_fn();
+  if (!fn) return fail(MW_ERR_CUDA, "cuTensorMapEncodeTiled is unavailable (no CUDA driver?)");
+  cuuint64_t dims[3] = {8, static_cast<cuuint64_t>(N_pad), static_cast<cuuint64_t>(BH)};
+  cuuint64_t strides[2] = {32, static_cast<cuuint64_t>(N_pad) * 32};
+  cuuint32_t box[3] = {8, static_cast<cuuint32_t>(box_rows), 1};
+  cuuint32_t estr[3] = {1, 1, 1};
+  CUresult r = fn(m, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 3, const_cast<float*>(bias), dims, strides,
+                  box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_32B,
+                  CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  if (r != CUDA_SUCCESS) return fail(MW_ERR_CUDA, "cuTensorMapEncodeTiled(bias) failed: %d", (int)r);
+  return MW_OK;
 }
 
 // Makes the device of `stream` current on the calling thread for the scope
@@ -470,10 +489,12 @@ mw_status mw_bca_bwd_stage(int stage, const void* q, const void* k, const void* 
   float* dq_acc = reinterpret_cast<float*>(base + w.dq_acc);
   float* lse2 = reinterpret_cast<float*>(base + w.lse2);
   float* delta = reinterpret_cast<float*>(base + w.delta);
+  float* bias = kernel_d(d) == 64 ? reinterpret_cast<float*>(base + w.bias) : nullptr;
   if (pre)
     MW_TRY(launch_status(mw::launch_bwd_pre(kernel_d(d), d, static_cast<const __nv_bfloat16*>(o),
                                             static_cast<const __nv_bfloat16*>(dout), lse, lse2,
-                                            delta, dq_acc, BH, static_cast<int>(N), N_pad, s),
+                                            delta, dq_acc, bias, 1.f / scale, BH,
+                                            static_cast<int>(N), N_pad, s),
                          "backward pre kernel launch"));
   if (main) {
     unsigned* status = nullptr;
@@ -486,6 +507,8 @@ mw_status mw_bca_bwd_stage(int stage, const void* q, const void* k, const void* 
     MW_TRY(make_map(&tv, v, static_cast<int>(N), BH, d, "v"));
     MW_TRY(make_map(&tdo, dout, static_cast<int>(N), BH, d, "dout", qrows));
     MW_TRY(make_map(&tdq, dq_acc, N_pad, BH, D, "dq_acc", 32, true));
+    CUtensorMap tbias = tdq;  // d = 128: unused
+    if (bias != nullptr) MW_TRY(encode_bias_map(&tbias, bias, N_pad, BH, qrows));
     mw::BwdParams p{};
     p.BH = BH;
     p.N = static_cast<int>(N);
@@ -501,7 +524,7 @@ mw_status mw_bca_bwd_stage(int stage, const void* q, const void* k, const void* 
     p.dv = static_cast<__nv_bfloat16*>(dv);
     p.status = status;
     p.budget_ns = budget_ns();
-    MW_TRY(launch_status(mw::launch_bwd_main(D, mma_d(d), tq, tk, tv, tdo, tdq, p, s),
+    MW_TRY(launch_status(mw::launch_bwd_main(D, mma_d(d), tq, tk, tv, tdo, tdq, tbias, p, s),
                          "backward kernel launch"));
   }
   if (post)

@@ -59,16 +59,24 @@ struct BwdLayout {
   // d = 64: per drain warp, one 32 x 32 f32 box with the 128-byte swizzle (the
   // TMA reduce-add source); 1024-byte aligned
   static constexpr int STG_BYTES = DQT ? 0 : 4 * 32 * 32 * 4;
-  static constexpr int VEC_BYTES = QN * 4;
+  // d = 64: the per-query LSE and D terms enter S^T and dP^T through one
+  // tf32 MMA each (a QN x 32-byte bias tile in each Q stage, all-ones A
+  // rows), so the P/dS warps read no LSE or D rows from shared memory
+  static constexpr bool FOLD = (D == 64);
+  static constexpr int BIAS_BYTES = FOLD ? QN * 32 : 0;
+  static constexpr int QSTRIDE = QTILE + BIAS_BYTES;  // one Q stage
+  static constexpr int VEC_BYTES = FOLD ? 0 : QN * 4;
+  static constexpr int ONES_BYTES = FOLD ? 512 : 0;   // two 256-byte atoms of A rows
   static constexpr int OFF_K = 0;
   static constexpr int OFF_V = OFF_K + KTILE;
   static constexpr int OFF_Q = OFF_V + KTILE;
-  static constexpr int OFF_DO = OFF_Q + STAGES * QTILE;
+  static constexpr int OFF_DO = OFF_Q + STAGES * QSTRIDE;
   static constexpr int OFF_DS = OFF_DO + STAGES * QTILE;
   static constexpr int OFF_STG = OFF_DS + DS_BUFS * DS_BYTES;
   static constexpr int OFF_LSE = OFF_STG + STG_BYTES;
   static constexpr int OFF_DELTA = OFF_LSE + STAGES * VEC_BYTES;
-  static constexpr int OFF_BAR = OFF_DELTA + STAGES * VEC_BYTES;
+  static constexpr int OFF_ONES = OFF_DELTA + STAGES * VEC_BYTES;
+  static constexpr int OFF_BAR = OFF_ONES + ONES_BYTES;
   // kv_full, q_full[S], q_empty[S], do_full[S], do_empty[S], s_full, s_free,
   // dp_full, dp_free, pt_ready, pt_free, p_ready, dq_full, dq_free,
   // ds_free[DS_BUFS], dkv_full
@@ -112,7 +120,8 @@ template <int D, int DM>
 __global__ void __launch_bounds__(BwdLayout<D, DM>::THREADS, 1)
     bca_bwd_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_k,
                    const __grid_constant__ CUtensorMap tm_v, const __grid_constant__ CUtensorMap tm_do,
-                   const __grid_constant__ CUtensorMap tm_dq, const BwdParams p) {
+                   const __grid_constant__ CUtensorMap tm_dq,
+                   const __grid_constant__ CUtensorMap tm_bias, const BwdParams p) {
   using L = BwdLayout<D, DM>;
   constexpr int NS = L::STAGES;
   constexpr int QN = L::QN;
@@ -159,6 +168,17 @@ __global__ void __launch_bounds__(BwdLayout<D, DM>::THREADS, 1)
   // dQ tiles instead of contending for the same L2 lines
   const int q_rot = kt % n_q;
 
+  if constexpr (L::FOLD) {
+    // A rows of the bias MMAs: [1 1 0 0 | 1 1 0 0] picks the LSE pair of a
+    // bias row, [0 0 1 1 | 0 0 1 1] its D pair; both 16-byte halves alike, so
+    // the 32-byte swizzle leaves them unchanged (8 rows of each)
+    if (threadIdx.x < 128) {
+      const int a = threadIdx.x >> 6, c = threadIdx.x & 7;
+      reinterpret_cast<float*>(smem + L::OFF_ONES)[threadIdx.x] =
+          (((c & 3) < 2) == (a == 0)) ? 1.f : 0.f;
+      fence_proxy_async_smem();
+    }
+  }
   if (threadIdx.x == 0) {
     mbar_init(kv_full, 1);
     for (int s = 0; s < NS; ++s) {
@@ -219,16 +239,19 @@ __global__ void __launch_bounds__(BwdLayout<D, DM>::THREADS, 1)
         const int q0 = (m_begin + (j + q_rot) % n_q) * QN;
         const size_t voff = static_cast<size_t>(bh) * p.N_pad + q0;
         if (!mbar_wait(&q_empty[st], ph ^ 1, ctl)) break;
-        mbar_arrive_expect_tx(&q_full[st], L::QTILE + L::VEC_BYTES);
+        mbar_arrive_expect_tx(&q_full[st], L::QTILE + L::BIAS_BYTES + L::VEC_BYTES);
         for (int r = 0; r < L::REG; ++r)
-          tma_load_3d(sQ + st * L::QTILE + r * L::QREGION, &tm_q, &q_full[st], 64 * r, q0, bh);
-        bulk_load(sLSE + st * QN, p.lse2 + voff, L::VEC_BYTES, &q_full[st]);
+          tma_load_3d(sQ + st * L::QSTRIDE + r * L::QREGION, &tm_q, &q_full[st], 64 * r, q0, bh);
+        if constexpr (L::FOLD)
+          tma_load_3d(sQ + st * L::QSTRIDE + L::QTILE, &tm_bias, &q_full[st], 0, q0, bh);
+        else
+          bulk_load(sLSE + st * QN, p.lse2 + voff, L::VEC_BYTES, &q_full[st]);
         ++issued_q;
         if (!mbar_wait(&do_empty[st], ph ^ 1, ctl)) break;
         mbar_arrive_expect_tx(&do_full[st], L::QTILE + L::VEC_BYTES);
         for (int r = 0; r < L::REG; ++r)
           tma_load_3d(sDO + st * L::QTILE + r * L::QREGION, &tm_do, &do_full[st], 64 * r, q0, bh);
-        bulk_load(sDelta + st * QN, p.delta + voff, L::VEC_BYTES, &do_full[st]);
+        if constexpr (!L::FOLD) bulk_load(sDelta + st * QN, p.delta + voff, L::VEC_BYTES, &do_full[st]);
         ++issued_do;
       }
       if (*abort_flag) {
@@ -263,6 +286,16 @@ __global__ void __launch_bounds__(BwdLayout<D, DM>::THREADS, 1)
       const uint64_t do_mn0 = sdesc_sw128(smem_u32(sDO), L::QREGION, 1024);
       const uint64_t ds_mn0 = sdesc_sw128(smem_u32(sDS), L::KREGION, 1024);
       const uint64_t ds_kmaj0 = sdesc_sw128(smem_u32(sDS), 16, 1024);
+      // d = 64: S^T += ones x (-LSE/scale) and dP^T += ones x (-D), one tf32
+      // MMA each (K = 8); the 256-byte A atoms serve every 8-row group (SBO 0)
+      const uint64_t ones_l = sdesc_sw32(smem_u32(smem + L::OFF_ONES), 0);
+      const uint64_t ones_d = sdesc_sw32(smem_u32(smem + L::OFF_ONES + 256), 0);
+      const uint64_t bias0 = sdesc_sw32(smem_u32(sQ + L::QTILE), 256);
+      auto add_bias = [&](uint32_t d_col, uint64_t ones, int stage) {
+        if constexpr (L::FOLD)
+          umma_ss_tf32(tmem + d_col, ones, sdesc_add(bias0, stage * L::QSTRIDE),
+                       idesc_tf32_f32(128, QN), 1u);
+      };
       // X = A B^T, both K-major over d (S^T = K Q^T, dP^T = V dO^T)
       auto issue_kmajor = [&](uint32_t d_col, uint64_t a, uint64_t b) {
 #pragma unroll
@@ -285,6 +318,7 @@ __global__ void __launch_bounds__(BwdLayout<D, DM>::THREADS, 1)
       tc_fence_after();
       if (ok && role_a) {
         issue_kmajor(L::S_COL, k_kmaj, q_kmaj0);
+        add_bias(L::S_COL, ones_l, 0);
         umma_commit(s_full);
         if (L::SHARED_X) ok = warp_wait(s_free, 0, ctl);  // X holds S^T_0 until read
         if (ok) ok = warp_wait(&do_full[0], 0, ctl);
@@ -292,6 +326,7 @@ __global__ void __launch_bounds__(BwdLayout<D, DM>::THREADS, 1)
       }
       if (ok && role_a) {
         issue_kmajor(L::DP_COL, v_kmaj, do_kmaj0);
+        add_bias(L::DP_COL, ones_d, 0);
         umma_commit(dp_full);
       }
       for (int j = 0; ok && j < n_q; ++j) {
@@ -300,14 +335,15 @@ __global__ void __launch_bounds__(BwdLayout<D, DM>::THREADS, 1)
         const uint32_t ph1 = ((j + 1) / NS) & 1;
         const bool more = j + 1 < n_q;
         const uint64_t do_mn = sdesc_add(do_mn0, st * L::QTILE);
-        const uint64_t q_mn = sdesc_add(q_mn0, st * L::QTILE);
+        const uint64_t q_mn = sdesc_add(q_mn0, st * L::QSTRIDE);
         if (role_a) {
           if (!L::SHARED_X && more) {
             // S^T of the next step as soon as the P/dS warps hold S^T_j
             if (!(ok = warp_wait(s_free, j & 1, ctl))) break;
             if (!(ok = warp_wait(&q_full[st1], ph1, ctl))) break;
             tc_fence_after();
-            issue_kmajor(L::S_COL, k_kmaj, sdesc_add(q_kmaj0, st1 * L::QTILE));
+            issue_kmajor(L::S_COL, k_kmaj, sdesc_add(q_kmaj0, st1 * L::QSTRIDE));
+            add_bias(L::S_COL, ones_l, st1);
             umma_commit(s_full);
           }
           // dV += P^T dO_j as soon as P^T_j is in TMEM (while dS_j is computed)
@@ -325,6 +361,7 @@ __global__ void __launch_bounds__(BwdLayout<D, DM>::THREADS, 1)
             if (!(ok = warp_wait(&do_full[st1], ph1, ctl))) break;
             tc_fence_after();
             issue_kmajor(L::DP_COL, v_kmaj, sdesc_add(do_kmaj0, st1 * L::QTILE));
+            add_bias(L::DP_COL, ones_d, st1);
             umma_commit(dp_full);
           }
         }
@@ -363,12 +400,14 @@ __global__ void __launch_bounds__(BwdLayout<D, DM>::THREADS, 1)
           // next step, then its dP^T once the P/dS warps have read that S^T
           if (!(ok = warp_wait(&q_full[st1], ph1, ctl))) break;
           tc_fence_after();
-          issue_kmajor(L::S_COL, k_kmaj, sdesc_add(q_kmaj0, st1 * L::QTILE));
+          issue_kmajor(L::S_COL, k_kmaj, sdesc_add(q_kmaj0, st1 * L::QSTRIDE));
+            add_bias(L::S_COL, ones_l, st1);
           umma_commit(s_full);
           if (!(ok = warp_wait(s_free, (j + 1) & 1, ctl))) break;
           if (!(ok = warp_wait(&do_full[st1], ph1, ctl))) break;
           tc_fence_after();
           issue_kmajor(L::DP_COL, v_kmaj, sdesc_add(do_kmaj0, st1 * L::QTILE));
+            add_bias(L::DP_COL, ones_d, st1);
           umma_commit(dp_full);
         }
         if (L::SHARED_X && role_b) {
@@ -435,7 +474,7 @@ __global__ void __launch_bounds__(BwdLayout<D, DM>::THREADS, 1)
           nl[2 * c + 1] = make_float2(-v.z, -v.w);
         }
       };
-      if constexpr (L::PREFETCH) load_lse();
+      if constexpr (L::PREFETCH && !L::FOLD) load_lse();
       float pr[CW];
       {
         uint32_t r[CW / 32][32];
@@ -455,7 +494,9 @@ __global__ void __launch_bounds__(BwdLayout<D, DM>::THREADS, 1)
       const float2 sl2x2 = make_float2(sl2, sl2);
 #pragma unroll
       for (int c = 0; c < CW / 2; ++c) {
-        const float2 x = fma2(make_float2(pr[2 * c], pr[2 * c + 1]), sl2x2, nl[c]);
+        // d = 64: the MMA already subtracted LSE/scale
+        const float2 x = L::FOLD ? mul2(make_float2(pr[2 * c], pr[2 * c + 1]), sl2x2)
+                                 : fma2(make_float2(pr[2 * c], pr[2 * c + 1]), sl2x2, nl[c]);
         pr[2 * c] = ex2_approx(x.x);
         pr[2 * c + 1] = ex2_approx(x.y);
       }
@@ -491,7 +532,7 @@ __global__ void __launch_bounds__(BwdLayout<D, DM>::THREADS, 1)
       // the step's D row came with dO, which dP^T_j has read; d = 64: all of
       // it is requested before the TMEM loads, so the two latencies overlap
       float4 dvv[L::PREFETCH ? CW / 4 : 1];
-      if constexpr (L::PREFETCH) {
+      if constexpr (L::PREFETCH && !L::FOLD) {
 #pragma unroll
         for (int c = 0; c < CW / 4; ++c) dvv[c] = reinterpret_cast<const float4*>(delta)[c];
       }
@@ -508,14 +549,16 @@ __global__ void __launch_bounds__(BwdLayout<D, DM>::THREADS, 1)
         }
 #pragma unroll
         for (int k = 0; k < 8; ++k) {
-          const float4 dv = L::PREFETCH ? dvv[L::PREFETCH ? 8 * h + k : 0]
+          // d = 64: the MMA already subtracted D
+          const float4 dv = L::FOLD ? make_float4(0.f, 0.f, 0.f, 0.f)
+                          : L::PREFETCH ? dvv[L::PREFETCH ? 8 * h + k : 0]
                                         : reinterpret_cast<const float4*>(delta)[8 * h + k];
           const int c = 32 * h + 4 * k;
           // dS = P (dP - D), two columns per instruction
-          const float2 t0 = add2(make_float2(__uint_as_float(r[4 * k]), __uint_as_float(r[4 * k + 1])),
-                                 make_float2(-dv.x, -dv.y));
-          const float2 t1 = add2(make_float2(__uint_as_float(r[4 * k + 2]), __uint_as_float(r[4 * k + 3])),
-                                 make_float2(-dv.z, -dv.w));
+          const float2 dp0 = make_float2(__uint_as_float(r[4 * k]), __uint_as_float(r[4 * k + 1]));
+          const float2 dp1 = make_float2(__uint_as_float(r[4 * k + 2]), __uint_as_float(r[4 * k + 3]));
+          const float2 t0 = L::FOLD ? dp0 : add2(dp0, make_float2(-dv.x, -dv.y));
+          const float2 t1 = L::FOLD ? dp1 : add2(dp1, make_float2(-dv.z, -dv.w));
           const float2 s0 = mul2(make_float2(pr[c], pr[c + 1]), t0);
           const float2 s1 = mul2(make_float2(pr[c + 2], pr[c + 3]), t1);
           dk[16 * h + 2 * k] = pack_bf16x2(s0.x, s0.y);
@@ -670,8 +713,9 @@ __global__ void __launch_bounds__(256) bwd_pre_kernel(const __nv_bfloat16* __res
                                                       const float* __restrict__ lse,
                                                       float* __restrict__ lse2,
                                                       float* __restrict__ delta,
-                                                      float* __restrict__ dq_acc, int BH, int N,
-                                                      int N_pad, int d_io_arg) {
+                                                      float* __restrict__ dq_acc,
+                                                      float* __restrict__ bias, float inv_scale,
+                                                      int BH, int N, int N_pad, int d_io_arg) {
   const int d_io = (D == 64) ? D : d_io_arg;  // padded head dims use the 128-wide kernels
   constexpr int G = D / 8;                     // lanes per row (8 bf16 = 16 bytes each)
   const int lane = threadIdx.x & 31;
@@ -703,6 +747,16 @@ __global__ void __launch_bounds__(256) bwd_pre_kernel(const __nv_bfloat16* __res
   if (valid && sub == 0) {
     delta[gr] = sum;
     lse2[gr] = (i < N) ? lse[static_cast<size_t>(bh) * N + i] * 1.4426950408889634f : INFINITY;
+    if (bias != nullptr) {
+      // -LSE/scale and -D, each as a tf32 part (low 13 mantissa bits cleared)
+      // and the fp32 remainder; padding rows get -1e30, so their P is 0
+      const float lb = (i < N) ? -lse[static_cast<size_t>(bh) * N + i] * inv_scale : -1e30f;
+      const float lh = __uint_as_float(__float_as_uint(lb) & 0xffffe000u);
+      const float dh = __uint_as_float(__float_as_uint(-sum) & 0xffffe000u);
+      float4* row = reinterpret_cast<float4*>(bias + gr * 8);
+      row[0] = make_float4(lh, lb - lh, dh, -sum - dh);
+      row[1] = make_float4(0.f, 0.f, 0.f, 0.f);
+    }
   }
 }
 
@@ -728,8 +782,8 @@ __global__ void __launch_bounds__(256) bwd_post_kernel(const float* __restrict__
 
 template <int D, int DM>
 cudaError_t launch_bwd_main_t(const CUtensorMap& tq, const CUtensorMap& tk, const CUtensorMap& tv,
-                              const CUtensorMap& tdo, const CUtensorMap& tdq, const BwdParams& p,
-                              cudaStream_t s) {
+                              const CUtensorMap& tdo, const CUtensorMap& tdq,
+                              const CUtensorMap& tbias, const BwdParams& p, cudaStream_t s) {
   using L = BwdLayout<D, DM>;
   static bool attr_set = false;
   if (!attr_set) {
@@ -745,30 +799,30 @@ cudaError_t launch_bwd_main_t(const CUtensorMap& tq, const CUtensorMap& tk, cons
     attr_set = true;
   }
   const unsigned grid = static_cast<unsigned>(p.BH) * (p.N_pad / kTileRows);
-  bca_bwd_kernel<D, DM><<<grid, L::THREADS, L::BYTES, s>>>(tq, tk, tv, tdo, tdq, p);
+  bca_bwd_kernel<D, DM><<<grid, L::THREADS, L::BYTES, s>>>(tq, tk, tv, tdo, tdq, tbias, p);
   return cudaGetLastError();
 }
 
 }  // namespace
 
 cudaError_t launch_bwd_pre(int d, int d_io, const __nv_bfloat16* o, const __nv_bfloat16* dout,
-                           const float* lse, float* lse2, float* delta, float* dq_acc, int BH,
-                           int N, int N_pad, cudaStream_t s) {
+                           const float* lse, float* lse2, float* delta, float* dq_acc,
+                           float* bias, float inv_scale, int BH, int N, int N_pad, cudaStream_t s) {
   const size_t threads = static_cast<size_t>(BH) * N_pad * (d / 8);  // d / 8 lanes per row
   const unsigned grid = static_cast<unsigned>((threads + 255) / 256);
   if (d == 64)
-    bwd_pre_kernel<64><<<grid, 256, 0, s>>>(o, dout, lse, lse2, delta, dq_acc, BH, N, N_pad, d_io);
+    bwd_pre_kernel<64><<<grid, 256, 0, s>>>(o, dout, lse, lse2, delta, dq_acc, bias, inv_scale, BH, N, N_pad, d_io);
   else
-    bwd_pre_kernel<128><<<grid, 256, 0, s>>>(o, dout, lse, lse2, delta, dq_acc, BH, N, N_pad, d_io);
+    bwd_pre_kernel<128><<<grid, 256, 0, s>>>(o, dout, lse, lse2, delta, dq_acc, nullptr, 0.f, BH, N, N_pad, d_io);
   return cudaGetLastError();
 }
 
 cudaError_t launch_bwd_main(int d, int dm, const CUtensorMap& tq, const CUtensorMap& tk,
                             const CUtensorMap& tv, const CUtensorMap& tdo, const CUtensorMap& tdq,
-                            const BwdParams& p, cudaStream_t s) {
-  if (d == 64) return launch_bwd_main_t<64, 64>(tq, tk, tv, tdo, tdq, p, s);
-  if (dm == 80) return launch_bwd_main_t<128, 80>(tq, tk, tv, tdo, tdq, p, s);
-  return launch_bwd_main_t<128, 128>(tq, tk, tv, tdo, tdq, p, s);
+                            const CUtensorMap& tbias, const BwdParams& p, cudaStream_t s) {
+  if (d == 64) return launch_bwd_main_t<64, 64>(tq, tk, tv, tdo, tdq, tbias, p, s);
+  if (dm == 80) return launch_bwd_main_t<128, 80>(tq, tk, tv, tdo, tdq, tbias, p, s);
+  return launch_bwd_main_t<128, 128>(tq, tk, tv, tdo, tdq, tbias, p, s);
 }
 
 cudaError_t launch_bwd_post(int d, int d_io, const float* dq_acc, __nv_bfloat16* dq, float scale,

@@ -136,15 +136,20 @@ cudaError_t launch_fwd(int d, int dm, const CUtensorMap& tq, const CUtensorMap& 
 cudaError_t launch_combine(int d, int d_io, const float* o_part, const float* lse_part,
                            __nv_bfloat16* o, float* lse, int splits, int BH, int rows,
                            const CommitJob& cj, cudaStream_t s);
+// bias (d = 64, else null): per padded row 8 floats (hi, lo of -LSE/scale;
+// hi, lo of -D; 4 zeros), the B operand of the tf32 MMAs that add those
+// per-query terms to S^T and dP^T
 cudaError_t launch_bwd_pre(int d, int d_io, const __nv_bfloat16* o, const __nv_bfloat16* dout,
-                           const float* lse, float* lse2, float* delta, float* dq_acc, int BH,
-                           int N, int N_pad, cudaStream_t s);
+                           const float* lse, float* lse2, float* delta, float* dq_acc,
+                           float* bias, float inv_scale, int BH, int N, int N_pad, cudaStream_t s);
 // tdq: f32 map over dQacc [BH, N_pad, d] with 32 x 32 boxes (128-byte
 // swizzle), the target of the d = 64 kernel's TMA reduce-adds
 // dm: MMA width as for launch_fwd
+// tbias (d = 64): f32 map over the bias rows [BH, N_pad, 8], 8 x 128 boxes,
+// 32-byte swizzle (d = 128: any map, unused)
 cudaError_t launch_bwd_main(int d, int dm, const CUtensorMap& tq, const CUtensorMap& tk,
                             const CUtensorMap& tv, const CUtensorMap& tdo, const CUtensorMap& tdq,
-                            const BwdParams& p, cudaStream_t s);
+                            const CUtensorMap& tbias, const BwdParams& p, cudaStream_t s);
 cudaError_t launch_bwd_post(int d, int d_io, const float* dq_acc, __nv_bfloat16* dq, float scale,
                             int BH, int N, int N_pad, cudaStream_t s);
 // d: any multiple of 8 (rows are copied in 16-byte pieces)

@@ -82,8 +82,9 @@ def test_bwd_rejects_bad_arguments_and_workspace(mw):
     lib = mw.library()
     B, H, n, T, d = 1, 2, 3, 50, 64
     need = lib.mw_bca_bwd_workspace_size(B, H, n, T, d)
-    # dQ accumulator (fp32, rows padded to 128) + two fp32 row vectors, 256-byte aligned
-    assert need == 2 * 256 * 64 * 4 + 2 * 256 * 4 + 2 * 256 * 4
+    # dQ accumulator (fp32, rows padded to 128) + two fp32 row vectors, 256-byte
+    # aligned, + the d = 64 bias rows of the MMA-folded LSE and D terms (32 bytes a row)
+    assert need == 2 * 256 * 64 * 4 + 2 * 256 * 4 + 2 * 256 * 4 + 2 * 256 * 32
     assert lib.mw_bca_bwd_workspace_size(B, H, n, T, 100) == 0
     # a padded head dim (72) keeps a 128-wide fp32 accumulator
     assert lib.mw_bca_bwd_workspace_size(B, H, n, T, 72) == 2 * 256 * 128 * 4 + 2 * 256 * 4 + 2 * 256 * 4
