@@ -233,6 +233,46 @@ def dq_rows(q: torch.Tensor, k: torch.Tensor, v: torch.Tensor, do: torch.Tensor,
     return torch.stack(out)
 
 
+def dkv_rows(q: torch.Tensor, k: torch.Tensor, v: torch.Tensor, do: torch.Tensor, T: int,
+             scale: float, rows: Sequence[int], block: int = 256
+             ) -> Tuple[torch.Tensor, torch.Tensor]:
+    """(dK, dV) of selected key rows of one head (Q,K,V,dO [N,d]).
+
+    Key j is seen by the queries i with chunk(i) >= chunk(j).  Each such
+    query needs its own LSE_i and D_i = <dO_i, O_i> over its visible keys
+    [0, (chunk(i)+1) T); then P_ij = exp(s_ij - LSE_i),
+    dS_ij = P_ij (<dO_i, v_j> - D_i), dV_j = sum_i P_ij dO_i and
+    dK_j = scale * sum_i dS_ij q_i.  The queries are taken ``block`` rows at a
+    time (rows of one block share no state), starting at the first query that
+    sees the earliest selected key, so sampling late keys stays cheap.
+    """
+    q, k, v, do = q.to(F64), k.to(F64), v.to(F64), do.to(F64)
+    N = q.shape[0]
+    rows = list(rows)
+    sel = torch.tensor(rows, dtype=torch.long)
+    sel_chunk = sel // T
+    dk = torch.zeros(len(rows), k.shape[1], dtype=F64)
+    dv = torch.zeros(len(rows), v.shape[1], dtype=F64)
+    i0 = int(sel_chunk.min()) * T
+    for c in range(i0 // T, N // T):
+        end = (c + 1) * T                      # keys visible to chunk c
+        for b0 in range(c * T, end, block):
+            qi, doi = q[b0:min(end, b0 + block)], do[b0:min(end, b0 + block)]
+            s = scale * (qi @ k[:end].T)
+            lse = _row_lse(s)
+            p = torch.exp(s - lse.unsqueeze(-1))
+            D = (doi * (p @ v[:end])).sum(-1)
+            seen = sel_chunk <= c              # selected keys this chunk sees
+            if not bool(seen.any()):
+                continue
+            idx = sel[seen]
+            ps = p[:, idx]
+            ds = ps * (doi @ v[idx].T - D.unsqueeze(-1))
+            dv[seen] += ps.T @ doi
+            dk[seen] += scale * (ds.T @ qi)
+    return dk, dv
+
+
 # --------------------------------------------------------------------------
 # rolling KV cache (Sec. 3.5): ring of committed chunks + in-flight chunks
 # --------------------------------------------------------------------------

@@ -261,6 +261,20 @@ def test_dq_rows_matches_the_full_backward():
     assert torch.allclose(got, dq[0, 0, rows], atol=1e-13, rtol=0)
 
 
+def test_dkv_rows_matches_the_full_backward():
+    """The row-by-row dK/dV (used for long sequences) equals the full
+    backward's dK/dV rows, itself pinned by finite differences and autograd;
+    small query blocks make several blocks per chunk and a ragged last one."""
+    N, T, d = 28, 7, 5
+    q, k, v, do = (_rand(1, 1, N, d, seed=s)[0, 0] for s in (130, 131, 132, 133))
+    _, dk, dv = oracle.bwd(q.view(1, 1, N, d), k.view(1, 1, N, d), v.view(1, 1, N, d),
+                           do.view(1, 1, N, d), T, 0.6)
+    for rows in ([0, 6, 7, 13, 20, 27], [27, 21], [9]):
+        gk, gv = oracle.dkv_rows(q, k, v, do, T, 0.6, rows, block=3)
+        assert torch.allclose(gk, dk[0, 0, rows], atol=1e-13, rtol=0)
+        assert torch.allclose(gv, dv[0, 0, rows], atol=1e-13, rtol=0)
+
+
 # ---------------------------------------------------------------- rolling cache
 
 def _cache_case(W, T, cap, length, head, d=8, seed=70, B=1, H=2):
