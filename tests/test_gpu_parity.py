@@ -83,6 +83,7 @@ SMALL = [
     (1, 2, 20, 16, 128, 2.0),
     (1, 1, 2, 880, 128, 4.0),    # one latent frame per chunk, peaky logits
     (1, 3, 5, 200, 64, 1.0),
+    (1, 2, 4, 160, 64, 4.0),     # peaky logits at d = 64 (the running max jumps: O rescaled)
     (2, 2, 1, 600, 128, 1.0),    # a single chunk: full bidirectional attention
     (1, 20, 3, 96, 128, 1.0),    # the 3B head layout (20 heads of 128)
     (1, 2, 3, 100, 72, 1.0),     # the 0.5B head dim (72: 80-wide MMAs on 128-wide tiles)
@@ -135,10 +136,11 @@ def test_full_size_training_configs(mw, name):
 
 @pytest.mark.parametrize("d,N,T", [(64, 65536, 4096), (128, 32768, 2048)])
 def test_long_sequence_sampled_rows_and_invariants(mw, d, N, T):
-    """A long sequence (16 chunks): O, LSE and dQ on sampled rows against the
-    oracle's row-by-row forms; dK and dV through identities that hold at any
-    size: sum_j dK_j = 0 (each row of dS sums to zero) and sum_j dV_j =
-    sum_i dO_i (each row of P sums to one)."""
+    """A long sequence (16 chunks): O, LSE and dQ on sampled query rows and dK,
+    dV on sampled key rows (from the second half, so that the oracle only
+    needs the later queries) against the oracle's row-by-row forms; plus two
+    identities that hold at any size: sum_j dK_j = 0 (each row of dS sums to
+    zero) and sum_j dV_j = sum_i dO_i (each row of P sums to one)."""
     q, k, v, do = _inputs(1, 1, N // T, T, d, seed=55)
     sc = 1.0 / math.sqrt(d)
     qc, kc, vc, doc = (t.cuda() for t in (q, k, v, do))
@@ -153,6 +155,11 @@ def test_long_sequence_sampled_rows_and_invariants(mw, d, N, T):
     check_o(o[0, 0, rows], o_ref, f"long d{d} sampled O")
     check_lse(lse[0, 0, rows], lse_ref, f"long d{d} sampled LSE")
     check_grad(dq[0, 0, rows], oracle.dq_rows(q1, k1, v1, do1, T, sc, rows), f"long d{d} sampled dQ")
+    krows = sorted(set([N // 2, N // 2 + T - 1, N - T - 1, N - T, N - 1] +
+                       torch.randint(N // 2, N, (11,), generator=g).tolist()))
+    dk_ref, dv_ref = oracle.dkv_rows(q1, k1, v1, do1, T, sc, krows)
+    check_grad(dk[0, 0, krows], dk_ref, f"long d{d} sampled dK")
+    check_grad(dv[0, 0, krows], dv_ref, f"long d{d} sampled dV")
     dk64, dv64 = dk[0, 0].double().cpu(), dv[0, 0].double().cpu()
     assert float(dk64.sum(0).norm() / dk64.norm()) < 2e-2
     sum_do = do1.double().sum(0)
@@ -408,25 +415,34 @@ def test_programmatic_launch_changes_nothing(mw):
 
 
 def test_rolling_cache_config_steps(mw):
-    """The streaming workload: one 880-token chunk against an 8-chunk ring
-    whose head wraps mid-buffer; each step commits the chunk (FIFO eviction)."""
+    """The streaming workload over its full length: one 880-token chunk
+    against an 8-chunk ring whose head wraps mid-buffer, 64 steps, each
+    committing the chunk (FIFO eviction), so the head laps the ring eight
+    times.  Every step's O and LSE are checked on two sampled heads (the
+    first and the last) against the oracle run on the oracle's own ring; the
+    full O of the first three steps, and the whole ring at the end (bit-exact)."""
     cfg = CACHE_CONFIGS["rolling_cache"]
-    steps = 3
-    x = gen_cache(cfg, steps=steps)
+    x = gen_cache(cfg)
+    steps = cfg.steps
+    assert steps == 64
     kr, vr = x["k_ring"].clone(), x["v_ring"].clone()
     krg, vrg = kr.cuda(), vr.cuda()
     head, length = cfg.head, cfg.length
+    heads = (slice(0, 1), slice(cfg.H - 1, cfg.H))
     for s in range(steps):
         q, kn, vn = x["q"][s], x["k_new"][s], x["v_new"][s]
         o, lse = mw.mw_bca_cache_fwd(q.cuda(), kn.cuda(), vn.cuda(), krg, vrg, head, length,
                                      cfg.T, cfg.scale)
-        o_ref, lse_ref = oracle.cache_fwd(q, kn, vn, kr, vr, cfg.cap, head, length, cfg.T,
-                                          cfg.scale)
-        check_o(o, o_ref, f"step {s}")
-        check_lse(lse, lse_ref, f"step {s}")
+        for hs in ((slice(None),) if s < 3 else heads):
+            sl = (slice(None), hs)
+            o_ref, lse_ref = oracle.cache_fwd(q[sl], kn[sl], vn[sl], kr[sl], vr[sl], cfg.cap,
+                                              head, length, cfg.T, cfg.scale)
+            check_o(o[sl], o_ref, f"step {s} heads {hs}")
+            check_lse(lse[sl], lse_ref, f"step {s} heads {hs}")
         slot, head, length = oracle.ring_advance(cfg.cap, head, length, cfg.T)
         mw.mw_bca_cache_commit(krg, vrg, slot, kn.cuda(), vn.cuda())
         kr, vr = oracle.cache_commit(kr, vr, cfg.cap, slot, kn, vn)
+    assert (head, length) == ((cfg.head + steps * cfg.T) % cfg.cap, cfg.cap)
     assert torch.equal(krg.cpu(), kr) and torch.equal(vrg.cpu(), vr)
     assert mw.mw_device_status() == 0
 
