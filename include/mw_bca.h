@@ -282,9 +282,11 @@ mw_status mw_qkv_rope_split(const void* qkv, void* q, void* k, void* v, int B, i
  *   that first call before any stream capture.
  *   All calls share the one array and it keeps the last call's contents.
  *   Each call writes every partial it later reads, so nothing has to start at
- *   zero, but calls whose kernels overlap on the GPU (different streams, or
- *   different host threads without ordering) race on the array: serialise
- *   them, e.g. on one stream.
+ *   zero; a kernel that cannot run (mw_device_status then reports it) writes
+ *   its rows as O = 0, LSE = -inf rather than leaving an earlier call's
+ *   partials to be merged.  Calls whose kernels overlap on the GPU (different
+ *   streams, or different host threads without ordering) race on the array:
+ *   serialise them, e.g. on one stream.
  */
 mw_status mw_bca_cache_fwd_noalloc(const void* q, const void* k_new, const void* v_new,
                                    const void* k_cache, const void* v_cache, int cache_cap,

@@ -135,8 +135,30 @@ __global__ void __launch_bounds__(FwdLayout<D, DM>::THREADS, 1)
   constexpr int QT = L::QT;
   constexpr int NS = L::STAGES;
   extern __shared__ __align__(1024) uint8_t smem[];
+  // ---- work item: longest query blocks first (they see the most keys)
+  int x = blockIdx.x;
+  const int split = x % p.num_splits;
+  x /= p.num_splits;
+  const int bh = x % p.BH;
+  const int qb = p.n_qblocks - 1 - x / p.BH;
+  const int r0 = qb * kFwdBlockRows;
   if ((smem_u32(smem) & 1023u) != 0u) {
+    // nothing runs without aligned shared memory: report it, and give this
+    // CTA's rows a defined result (O = 0, LSE = -inf; as split partials, a
+    // -inf LSE that the combine skips) instead of leaving stale values behind
     if (threadIdx.x == 0) atomicOr(p.status, kDevMisaligned);
+    const int row = r0 + static_cast<int>(threadIdx.x);
+    if (threadIdx.x < kFwdBlockRows && row < p.rows_q) {
+      const size_t row_off = static_cast<size_t>(bh) * p.rows_q + row;
+      if (p.num_splits == 1) {
+        const int d_io = (D == 64) ? D : p.d_io;
+        uint4* dst = reinterpret_cast<uint4*>(p.o + row_off * d_io);
+        for (int c = 0; c < d_io / 8; ++c) dst[c] = make_uint4(0u, 0u, 0u, 0u);
+        if (p.lse) p.lse[row_off] = -INFINITY;
+      } else {
+        p.lse_part[static_cast<size_t>(split) * p.BH * p.rows_q + row_off] = -INFINITY;
+      }
+    }
     return;  // uniform across the CTA, before any barrier or TMEM use
   }
   uint64_t* bars = reinterpret_cast<uint64_t*>(smem + L::OFF_BAR);
@@ -157,13 +179,6 @@ __global__ void __launch_bounds__(FwdLayout<D, DM>::THREADS, 1)
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
 
-  // ---- work item: longest query blocks first (they see the most keys)
-  int x = blockIdx.x;
-  const int split = x % p.num_splits;
-  x /= p.num_splits;
-  const int bh = x % p.BH;
-  const int qb = p.n_qblocks - 1 - x / p.BH;
-  const int r0 = qb * kFwdBlockRows;
   // query tiles of the block that hold rows (the last block may hold one)
   const int qt_n = (r0 + kTileRows < p.rows_q) ? QT : 1;
   const int last_row = min(r0 + kFwdBlockRows - 1, p.rows_q - 1);

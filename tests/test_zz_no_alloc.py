@@ -4,22 +4,26 @@ Some callers cannot allocate device memory: hosts that only hand the library
 their own input/output buffers, and real-time streaming loops that must not
 call cudaMalloc/cudaFree (those can synchronise the device).  For them the
 library keeps its split-KV scratch in a fixed static device array.  These
-tests call the new entry point through the C ABI and check that it returns
-what the workspace-taking mw_bca_cache_fwd returns, on consecutive calls that
-share the one scratch array, and that oversized requests are refused.
+tests call the new entry point through the C ABI and check its results
+against the fp64 oracle (and bit for bit against the workspace-taking
+mw_bca_cache_fwd, which runs the same kernels and split plan) on consecutive
+calls that share the one scratch array, on a request that fills the array to
+within 4 KB, and that requests beyond it are refused before anything runs.
 
 This file is collected last so that a run stopping at the first failure has
 already run every other test; it also passes alone in a fresh process.
 """
-import ctypes
 import math
 
 import pytest
 import torch
 
+import oracle
+
 pytestmark = pytest.mark.gpu
 
 O_MAX_ABS, O_REL, LSE_REL = 2e-2, 5e-3, 1e-3
+MW_NOALLOC_SCRATCH_BYTES = 64 << 20  # include/mw_bca.h
 
 
 @pytest.fixture(scope="module")
@@ -54,14 +58,33 @@ def _noalloc(mw, q, kn, vn, kr, vr, head, length, T, scale):
 
 
 def _close(o, lse, o_ref, lse_ref):
-    a, b = o.double(), o_ref.double()
+    a, b = o.double().cpu(), o_ref.double()
     assert torch.isfinite(a).all() and torch.isfinite(lse).all()
     assert float((a - b).abs().max()) <= O_MAX_ABS
     assert float((a - b).norm() / b.norm()) <= O_REL
-    assert float(((lse - lse_ref).abs() / lse_ref.abs().clamp_min(1.0)).max()) <= LSE_REL
+    err = (lse.double().cpu() - lse_ref).abs() / lse_ref.abs().clamp_min(1.0)
+    assert float(err.max()) <= LSE_REL
 
 
-def test_noalloc_matches_workspace_entry_point_on_consecutive_calls(mw):
+def _check(mw, case, inputs, heads):
+    """One allocation-free call: bit-identical to the workspace entry point,
+    and within the tolerances of the oracle on the sampled heads."""
+    B, H, W, T, cap, length, head, d = case
+    q, kn, vn, kr, vr = inputs
+    scale = 1.0 / math.sqrt(d)
+    code, o, lse = _noalloc(mw, q, kn, vn, kr, vr, head, length, T, scale)
+    assert code == 0, mw.library().mw_last_error().decode()
+    o_ws, lse_ws = mw.mw_bca_cache_fwd(q, kn, vn, kr, vr, head, length, T, scale)
+    torch.cuda.synchronize()
+    assert torch.equal(o, o_ws) and torch.equal(lse, lse_ws)
+    for h in heads:
+        sl = (slice(None), slice(h, h + 1))
+        o_ref, lse_ref = oracle.cache_fwd(q[sl].cpu(), kn[sl].cpu(), vn[sl].cpu(), kr[sl].cpu(),
+                                          vr[sl].cpu(), cap, head, length, T, scale)
+        _close(o[sl], lse[sl], o_ref, lse_ref)
+
+
+def test_noalloc_matches_the_oracle_on_consecutive_calls(mw):
     # two different workloads back to back: the second call reuses the scratch
     # the first one left behind; then the first workload again
     cases = [
@@ -73,26 +96,49 @@ def test_noalloc_matches_workspace_entry_point_on_consecutive_calls(mw):
     for i in (0, 1, 0):
         B, H, W, T, cap, length, head, d = cases[i]
         assert mw.mw_bca_cache_workspace_size(B, H, W, T, d, length) > 0
-        q, kn, vn, kr, vr = inputs[i]
-        scale = 1.0 / math.sqrt(d)
-        o_ref, lse_ref = mw.mw_bca_cache_fwd(q, kn, vn, kr, vr, head, length, T, scale)
-        code, o, lse = _noalloc(mw, q, kn, vn, kr, vr, head, length, T, scale)
-        assert code == 0, mw.library().mw_last_error().decode()
-        torch.cuda.synchronize()
-        _close(o, lse, o_ref, lse_ref)
+        _check(mw, cases[i], inputs[i], heads=(0, H - 1))
     assert mw.mw_device_status() == 0
 
 
-def test_noalloc_refuses_sizes_beyond_the_scratch(mw):
-    lib = mw.library()
+def test_noalloc_fills_the_scratch_to_the_limit(mw):
+    # 16 forced splits of 16 heads x 508 rows at d = 128: the partials take
+    # 4 KB less than the whole array
+    case = (1, 16, 2, 254, 2048, 2048, 1000, 128)
+    B, H, W, T, cap, length, head, d = case
     try:
-        mw.mw_set_option("cache_splits", 16)   # 16 partials of a 3520-row, 16-head window
-        need = lib.mw_bca_cache_workspace_size(1, 16, 4, 880, 128, 10560)
-        assert need > (64 << 20)
-        fake = ctypes.c_void_p(0x10000)
-        code = lib.mw_bca_cache_fwd_noalloc(fake, fake, fake, fake, fake, 10560, 0, 10560, fake,
-                                            None, 1, 16, 4, 880, 128, 0.088, None)
+        mw.mw_set_option("cache_splits", 16)
+        need = mw.mw_bca_cache_workspace_size(B, H, W, T, d, length)
+        assert MW_NOALLOC_SCRATCH_BYTES - 4096 <= need <= MW_NOALLOC_SCRATCH_BYTES
+        _check(mw, case, _case(B, H, W, T, cap, d, seed=31), heads=(0, 7, H - 1))
+    finally:
+        mw.mw_set_option("cache_splits", 0)
+    assert mw.mw_device_status() == 0
+
+
+@pytest.mark.parametrize("splits,B,H,W,T,cap,d", [
+    (16, 1, 16, 4, 880, 10560, 128),   # far beyond: 16 partials of a 16-head window
+    (2, 1, 4, 1, 32265, 512, 64),      # 2560 bytes beyond
+])
+def test_noalloc_refuses_sizes_beyond_the_scratch(mw, splits, B, H, W, T, cap, d):
+    # real buffers of the full sizes, so that even a broken size check could
+    # only read and write memory that belongs to this test
+    lib = mw.library()
+    q, kn, vn, kr, vr = (torch.zeros(B, H, r, d, dtype=torch.bfloat16, device="cuda")
+                         for r in (W * T, W * T, W * T, cap, cap))
+    o = torch.zeros_like(q)
+    lse = torch.zeros(B, H, W * T, dtype=torch.float32, device="cuda")
+    try:
+        mw.mw_set_option("cache_splits", splits)
+        need = lib.mw_bca_cache_workspace_size(B, H, W, T, d, cap)
+        assert need > MW_NOALLOC_SCRATCH_BYTES
+        code = lib.mw_bca_cache_fwd_noalloc(q.data_ptr(), kn.data_ptr(), vn.data_ptr(),
+                                            kr.data_ptr(), vr.data_ptr(), cap, 0, cap,
+                                            o.data_ptr(), lse.data_ptr(), B, H, W, T, d,
+                                            1.0 / math.sqrt(d),
+                                            torch.cuda.current_stream().cuda_stream)
         assert code == 5  # MW_ERR_WORKSPACE, before anything is enqueued
         assert str(need) in lib.mw_last_error().decode()
+        torch.cuda.synchronize()
+        assert not o.any() and not lse.any()  # nothing ran
     finally:
         mw.mw_set_option("cache_splits", 0)
