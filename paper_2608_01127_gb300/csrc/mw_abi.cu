@@ -4,6 +4,7 @@
 // errors are reported without touching the device.
 #include <cudaTypedefs.h>
 
+#include <algorithm>
 #include <climits>
 #include <cstdarg>
 #include <cstdio>
@@ -348,6 +349,14 @@ mw_status fwd_common(const void* q, const void* k, const void* v, const void* kr
   p.d_io = d;
   p.T = T;
   p.n_qblocks = ceil_div(rows_q, mw::kFwdBlockRows);
+  // head groups of about four waves of CTAs each: a group's K/V stay in L2
+  // while its query blocks run, and the longest blocks of each group start
+  // first; groups of (nearly) equal size keep the last one from ending late
+  {
+    const int per_group = std::max(1, std::min(BH, ceil_div(4LL * sm_count(),
+                                                            static_cast<long long>(p.n_qblocks) * splits)));
+    p.head_groups = ceil_div(BH, per_group);
+  }
   p.ring_cap = len > 0 ? cap : 1;
   p.ring_head = len > 0 ? head : 0;
   p.ring_len = len;

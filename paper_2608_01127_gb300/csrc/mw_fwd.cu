@@ -135,12 +135,28 @@ __global__ void __launch_bounds__(FwdLayout<D, DM>::THREADS, 1)
   constexpr int QT = L::QT;
   constexpr int NS = L::STAGES;
   extern __shared__ __align__(1024) uint8_t smem[];
-  // ---- work item: longest query blocks first (they see the most keys)
+  // ---- work item: p.head_groups groups of heads one after another (sizes
+  // differ by at most one, the larger first), so that the CTAs running
+  // together share a few heads' K/V in L2; inside a group the longest query
+  // blocks (they see the most keys) come first
   int x = blockIdx.x;
   const int split = x % p.num_splits;
   x /= p.num_splits;
-  const int bh = x % p.BH;
-  const int qb = p.n_qblocks - 1 - x / p.BH;
+  const int g_base = p.BH / p.head_groups, g_rem = p.BH % p.head_groups;
+  const int big = (g_base + 1) * p.n_qblocks;  // CTAs of one larger group
+  int in_grp, gsize, h0;
+  if (x < g_rem * big) {
+    gsize = g_base + 1;
+    h0 = (x / big) * gsize;
+    in_grp = x % big;
+  } else {
+    const int y = x - g_rem * big;
+    gsize = g_base;
+    h0 = g_rem * (g_base + 1) + (y / (g_base * p.n_qblocks)) * g_base;
+    in_grp = y % (g_base * p.n_qblocks);
+  }
+  const int bh = h0 + in_grp % gsize;
+  const int qb = p.n_qblocks - 1 - in_grp / gsize;
   const int r0 = qb * kFwdBlockRows;
   if ((smem_u32(smem) & 1023u) != 0u) {
     // nothing runs without aligned shared memory: report it, and give this

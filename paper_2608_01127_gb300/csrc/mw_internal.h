@@ -39,6 +39,7 @@ struct FwdParams {
                     // TMA maps zero-fill the columns in between)
   int T;            // chunk length in tokens
   int n_qblocks;    // ceil(rows_q / kFwdBlockRows)
+  int head_groups;  // the heads are scheduled in this many groups (1..BH)
   int ring_cap;
   int ring_head;
   int ring_len;
