@@ -129,7 +129,7 @@ __global__ void __launch_bounds__(FwdLayout<D, DM>::THREADS, 1)
     bca_fwd_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_k,
                    const __grid_constant__ CUtensorMap tm_v, const __grid_constant__ CUtensorMap tm_kr,
                    const __grid_constant__ CUtensorMap tm_vr, const __grid_constant__ CUtensorMap tm_ks,
-                   const __grid_constant__ CUtensorMap tm_vs, const FwdParams p,
+                   const __grid_constant__ CUtensorMap tm_vs, const __grid_constant__ FwdParams p,
                    const __grid_constant__ RopeFreq rope_om) {
   using L = FwdLayout<D, DM, ROPE>;
   constexpr int QT = L::QT;
