@@ -377,6 +377,30 @@ def cache_fwd(q: torch.Tensor, k_new: torch.Tensor, v_new: torch.Tensor,
     return o, lse
 
 
+def cache_fwd_reshift(q: torch.Tensor, k_new: torch.Tensor, v_new: torch.Tensor,
+                      k_ring: torch.Tensor, v_ring: torch.Tensor, cap: int, head: int,
+                      length: int, T: int, scale: float, k_sink: torch.Tensor,
+                      v_sink: torch.Tensor, rope_dims: int, base: float,
+                      shift: int) -> Tuple[torch.Tensor, torch.Tensor]:
+    """(O, LSE) of the streaming forward with RoPE re-shifting (Sec. 3.5).
+
+    The inputs carry their temporal RoPE: queries, in-flight keys and ring
+    keys at their stream positions (frames counted from the start of the
+    stream), the sink anchor at its own first position(s).  ``shift`` frames
+    have been evicted from the FIFO.  Re-shifting subtracts that offset from
+    the positions of the retained keys, and the active window (queries and
+    in-flight keys) is re-indexed with them, so that every position stays in
+    the trained range; the sink keeps its position.  Here that is done
+    literally: the non-sink rows are turned back by ``shift`` frames, then the
+    sink-anchored cache forward runs on the re-indexed tensors.
+    """
+    back = torch.full((1,), -int(shift))
+    qs = rope_rotate(q, back, rope_dims, base)
+    kns = rope_rotate(k_new, back, rope_dims, base)
+    krs = rope_rotate(k_ring, back, rope_dims, base)
+    return cache_fwd(qs, kns, v_new, krs, v_ring, cap, head, length, T, scale, k_sink, v_sink)
+
+
 def cache_commit(k_ring: torch.Tensor, v_ring: torch.Tensor, cap: int, slot: int,
                  k_src: torch.Tensor, v_src: torch.Tensor) -> Tuple[torch.Tensor, torch.Tensor]:
     """New ring contents after writing ``rows`` tokens at physical rows (slot+r) mod cap.

@@ -422,6 +422,72 @@ def test_rope_ring_equals_prerotated_ring():
     assert torch.equal(o, o2) and torch.equal(lse, lse2)
 
 
+def _reshift_case(seed=150, W=2, T=4, cap_chunks=3, head=5, S=3, d=8):
+    cap = cap_chunks * T
+    q, kn, vn, kr, vr = _cache_case(W, T, cap, cap, head, d=d, seed=seed)
+    ks, vs = _rand(1, 2, S, d, seed=seed + 7), _rand(1, 2, S, d, seed=seed + 8)
+    return W, T, cap, head, q, kn, vn, kr, vr, ks, vs
+
+
+def test_reshift_without_evictions_is_the_plain_sink_forward():
+    W, T, cap, head, q, kn, vn, kr, vr, ks, vs = _reshift_case()
+    o, lse = oracle.cache_fwd_reshift(q, kn, vn, kr, vr, cap, head, cap, T, 0.5, ks, vs, 6, 50.0, 0)
+    o2, lse2 = oracle.cache_fwd(q, kn, vn, kr, vr, cap, head, cap, T, 0.5, ks, vs)
+    assert torch.equal(o, o2) and torch.equal(lse, lse2)
+
+
+def test_reshift_only_moves_the_sink_relative_to_the_window():
+    """Turning every non-sink row back by the same angle keeps their mutual
+    scores; without a sink the shift therefore changes nothing, and with one
+    it equals turning only the sink forward by the shift (the form the
+    kernels use)."""
+    W, T, cap, head, q, kn, vn, kr, vr, ks, vs = _reshift_case()
+    empty = ks[:, :, :0]
+    for shift in (1, 7, 1000):
+        o, lse = oracle.cache_fwd_reshift(q, kn, vn, kr, vr, cap, head, cap, T, 0.5, empty,
+                                          vs[:, :, :0], 6, 50.0, shift)
+        o2, lse2 = oracle.cache_fwd(q, kn, vn, kr, vr, cap, head, cap, T, 0.5)
+        assert torch.allclose(o, o2, atol=1e-12, rtol=0) and torch.allclose(lse, lse2, atol=1e-12, rtol=0)
+        o, lse = oracle.cache_fwd_reshift(q, kn, vn, kr, vr, cap, head, cap, T, 0.5, ks, vs, 6,
+                                          50.0, shift)
+        ks_fwd = oracle.rope_rotate(ks, torch.full((1,), shift), 6, 50.0)
+        o3, lse3 = oracle.cache_fwd(q, kn, vn, kr, vr, cap, head, cap, T, 0.5, ks_fwd, vs)
+        assert torch.allclose(o, o3, atol=1e-12, rtol=0) and torch.allclose(lse, lse3, atol=1e-12, rtol=0)
+        # the direction matters: turning the sink back instead gives other scores
+        ks_bad = oracle.rope_rotate(ks, torch.full((1,), -shift), 6, 50.0)
+        o4, _ = oracle.cache_fwd(q, kn, vn, kr, vr, cap, head, cap, T, 0.5, ks_bad, vs)
+        assert (o4 - o).abs().max() > 1e-6
+
+
+def test_reshift_equals_window_positions():
+    """Keys rotated at stream positions and re-shifted by the evicted frames
+    give the attention of the same keys rotated at their window positions
+    (ring token t at frame first + t // P, the window counted from the
+    oldest retained chunk; the sink at frame 0)."""
+    W, T, cap, head, q0, kn0, vn, kr0, vr, ks0, vs = _reshift_case(seed=170)
+    P, first, shift, dims, base = 2, 1, 9, 6, 50.0
+    logical = torch.arange(cap)
+    ring_window = first + logical // P                    # logical order
+    win_frames = first + cap // P + torch.arange(W * T) // P
+    # stream-rotated inputs (what the caller holds): window frame + shift
+    phys = torch.tensor([(head + t) % cap for t in range(cap)])
+    inv = torch.empty_like(phys)
+    inv[phys] = logical                                   # physical row -> logical index
+    kr_stream = oracle.rope_rotate(kr0, ring_window[inv] + shift, dims, base)
+    q_s = oracle.rope_rotate(q0, win_frames + shift, dims, base)
+    kn_s = oracle.rope_rotate(kn0, win_frames + shift, dims, base)
+    ks = oracle.rope_rotate(ks0, torch.zeros(ks0.shape[-2], dtype=torch.long), dims, base)
+    o, lse = oracle.cache_fwd_reshift(q_s, kn_s, vn, kr_stream, vr, cap, head, cap, T, 0.5, ks, vs,
+                                      dims, base, shift)
+    # the window-position form: queries and in-flight keys at window frames,
+    # the ring turned on read from its unrotated keys
+    q_w = oracle.rope_rotate(q0, win_frames, dims, base)
+    kn_w = oracle.rope_rotate(kn0, win_frames, dims, base)
+    o2, lse2 = oracle.cache_fwd(q_w, kn_w, vn, kr0, vr, cap, head, cap, T, 0.5, ks, vs,
+                                rope=(dims, base, P, first))
+    assert torch.allclose(o, o2, atol=1e-12, rtol=0) and torch.allclose(lse, lse2, atol=1e-12, rtol=0)
+
+
 def test_ring_rotation_is_invisible():
     W, T, cap = 2, 3, 12
     q, kn, vn, kr, vr = _cache_case(W, T, cap, cap, 4)
