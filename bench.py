@@ -678,12 +678,16 @@ def bench_rolling(mw, dev, peaks):
                    "commit as two API calls. The ring (57.7 MB) stays L2-resident across "
                    "steps, as in streaming"}
     res.update(_cache_roofline(cfg, g_us, peaks))
-    # the same stream with the ring's RoPE re-shift fused into its read (32
-    # rotated channels, 440 tokens per frame; the ring holds unrotated keys)
+    # the same stream through the RoPE re-shift entry point (32 rotated
+    # channels; keys stored as rotated at their stream frames, two 440-token
+    # frames per chunk, so each step's eviction moves the window by two
+    # frames): without a sink no score changes, and the call is the plain
+    # forward
     def step_rope(s):
         h, ln, slot = plan[s]
         mw.mw_bca_cache_fwd_rope(qs[s], ks[s], vs[s], None, None, kr, vr, h, ln, cfg.T, 32,
-                                 10000.0, 440, 0, cfg.scale, need_lse=False, workspace=ws, out=o)
+                                 10000.0, 2 * (s + 1), cfg.scale, need_lse=False, workspace=ws,
+                                 out=o)
         mw.mw_bca_cache_commit(kr, vr, slot, ks[s], vs[s])
 
     for s in range(3):
@@ -737,17 +741,18 @@ def bench_sink(mw, dev, peaks, flush):
     med = statistics.median(ts) * 1e3
     res = {"us_median": round(med, 2), "l2": "flushed between runs", "sink_tokens": cfg.sink}
     res.update(_cache_roofline(cfg, med, peaks))
-    # the same call with the ring's RoPE re-shift fused into its read: the
-    # first 32 channels carry the temporal rotation, 440 tokens per frame, the
-    # ring starting at frame 1 behind the one-frame sink
+    # the same call with RoPE re-shifting: the first 32 channels carry the
+    # temporal rotation, every key rotated at its stream frame, and 24 frames
+    # (12 chunks of two 440-token frames) already evicted, so the one-frame
+    # sink turns by 24 frames as it is read
     ts = time_repeated(lambda: mw.mw_bca_cache_fwd_rope(q, kn, vn, ks, vs, kr, vr, cfg.head,
-                                                        cfg.length, cfg.T, 32, 10000.0, 440, 1,
+                                                        cfg.length, cfg.T, 32, 10000.0, 24,
                                                         cfg.scale, need_lse=False, workspace=ws,
                                                         out=o),
                        20, flush=flush)
     med_r = statistics.median(ts) * 1e3
-    res["rope_reshift"] = {"us_median": round(med_r, 2), "rope_dims": 32,
-                           "tokens_per_frame": 440, **_cache_roofline(cfg, med_r, peaks)}
+    res["rope_reshift"] = {"us_median": round(med_r, 2), "rope_dims": 32, "shift_frames": 24,
+                           "overhead": round(med_r / med - 1, 4), **_cache_roofline(cfg, med_r, peaks)}
     return res
 
 

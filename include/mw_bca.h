@@ -157,34 +157,37 @@ mw_status mw_bca_cache_fwd_sink(const void* q, const void* k_new, const void* v_
                                 int T_chunk, int d, float scale, void* stream);
 
 /*
- * The same forward with RoPE re-shifting of the ring fused into its read
- * (Sec. 3.5, RoPE re-shifting: after each cache update the retained keys are
- * re-indexed from the start of the window by subtracting the temporal offset
- * of the evicted chunks; the sink anchor keeps the first position).  Instead
- * of rewriting the ring, the ring holds keys without their temporal rotation
- * and each is rotated as it is read:
- *   ring token t (logical order, oldest = 0) is at frame
- *       f(t) = first_frame + t / tokens_per_frame   (integer division)
- *   channel pair (2i, 2i+1), 0 <= i < rope_dims / 2, of its key turns by
- *       f(t) * rope_base^(-2i / rope_dims):
- *       (x, y) -> (x cos - y sin, x sin + y cos)
- * The rotated key is rounded to bf16 before QK^T.  Sink and in-flight keys
- * (and all queries) are used as given: the caller rotates them to their
- * window positions.  The paper states neither the channel layout nor the
- * frequencies of its RoPE, so they are arguments.
- *   rope_dims        : even, 0 <= rope_dims <= d (0: no rotation, i.e.
- *                      mw_bca_cache_fwd_sink)
- *   rope_base        : > 1
- *   tokens_per_frame : >= 1
- *   first_frame      : >= 0, and first_frame + (cache_len - 1) / tokens_per_frame
- *                      <= 2^24 (the angle reduction is exact up to there)
+ * The same forward with RoPE re-shifting (Sec. 3.5, RoPE re-shifting: after
+ * each cache update the retained keys are re-indexed from the start of the
+ * window by subtracting the temporal offset of the evicted chunks, so that
+ * positions stay in the trained range; the sink anchor keeps the first
+ * position and is excluded).
+ *   The inputs carry their temporal rotation: queries, in-flight keys and the
+ *   ring's keys at their stream positions (each key rotated once, when its
+ *   chunk was projected, e.g. by mw_qkv_rope_split, and committed as it
+ *   is), the sink's keys at the sink's own position(s).  shift_frames frames
+ *   have been evicted.  Re-indexing moves the queries and every non-sink key
+ *   back by the same offset, which leaves their mutual scores unchanged (RoPE
+ *   scores depend on position differences only); what it changes are the
+ *   query-sink scores.  This call computes exactly that: the sink's keys turn
+ *   forward by shift_frames frames as they are read, rounded to bf16 before
+ *   QK^T, and nothing else is rotated:
+ *     channel pair (2i, 2i+1), 0 <= i < rope_dims / 2, turns by
+ *     shift_frames * rope_base^(-2i / rope_dims):  (x, y) -> (x cos - y sin, x sin + y cos)
+ *   Without a sink, or with shift_frames 0, the result is that of
+ *   mw_bca_cache_fwd_sink.  The paper states neither the channel layout nor
+ *   the frequencies of its RoPE, so they are arguments.
+ *   rope_dims    : even, 0 <= rope_dims <= d (0: no rotation)
+ *   rope_base    : > 1
+ *   shift_frames : frames evicted so far, 0 <= shift_frames <= 2^24 (the
+ *                  angle reduction is exact up to there)
  * Every other argument is as for mw_bca_cache_fwd_sink.
  */
 mw_status mw_bca_cache_fwd_rope(const void* q, const void* k_new, const void* v_new,
                                 const void* k_sink, const void* v_sink, int sink_len,
                                 const void* k_cache, const void* v_cache, int cache_cap,
                                 int cache_head, int cache_len, int rope_dims, float rope_base,
-                                int tokens_per_frame, int first_frame, void* o, float* lse,
+                                int shift_frames, void* o, float* lse,
                                 void* workspace, size_t ws_bytes, int B, int H, int n_q_chunks,
                                 int T_chunk, int d, float scale, void* stream);
 

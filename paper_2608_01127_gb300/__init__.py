@@ -12,7 +12,7 @@ Entry points (same names as the C ABI, taking torch tensors):
                    T_chunk, scale=None, need_lse=True) -> (o, lse)
   mw_bca_cache_fwd_sink(q, k_new, v_new, k_sink, v_sink, k_cache, v_cache,
                         cache_head, cache_len, T_chunk, ...) -> (o, lse)
-  mw_bca_cache_fwd_rope(..., rope_dims, rope_base, tokens_per_frame, first_frame)
+  mw_bca_cache_fwd_rope(..., rope_dims, rope_base, shift_frames)
   mw_bca_cache_commit(k_cache, v_cache, slot_start, k_src, v_src)
   mw_device_status(clear=True), mw_set_option(name, value)
 Tensors are contiguous bf16 [B, H, rows, d] on the current CUDA device.
@@ -88,7 +88,7 @@ def library() -> ctypes.CDLL:
                                   _I, _I, _I, _I, _I, _F, _P]),
         "mw_bca_cache_fwd_sink": (_I, [_P, _P, _P, _P, _P, _I, _P, _P, _I, _I, _I, _P, _P, _P,
                                        _Z, _I, _I, _I, _I, _I, _F, _P]),
-        "mw_bca_cache_fwd_rope": (_I, [_P, _P, _P, _P, _P, _I, _P, _P, _I, _I, _I, _I, _F, _I, _I,
+        "mw_bca_cache_fwd_rope": (_I, [_P, _P, _P, _P, _P, _I, _P, _P, _I, _I, _I, _I, _F, _I,
                                        _P, _P, _P, _Z, _I, _I, _I, _I, _I, _F, _P]),
         "mw_bca_cache_commit": (_I, [_P, _P, _I, _I, _P, _P, _I, _I, _I, _I, _P]),
         "mw_qkv_rope_split": (_I, [_P, _P, _P, _P, _I, _I, _I, _I, _I, _F, _I, _I, _P]),
@@ -289,15 +289,17 @@ def mw_bca_cache_fwd_sink(q, k_new, v_new, k_sink, v_sink, k_cache, v_cache, cac
 
 def mw_bca_cache_fwd_rope(q, k_new, v_new, k_sink, v_sink, k_cache, v_cache, cache_head: int,
                           cache_len: int, T_chunk: int, rope_dims: int, rope_base: float,
-                          tokens_per_frame: int, first_frame: int, scale: Optional[float] = None,
+                          shift_frames: int, scale: Optional[float] = None,
                           need_lse: bool = True, workspace: Optional[torch.Tensor] = None,
                           out: Optional[torch.Tensor] = None):
-    """As mw_bca_cache_fwd_sink (k_sink may be None) with the ring's keys rotated
-    on read to window frames first_frame + t // tokens_per_frame (RoPE
-    re-shifting, Sec. 3.5); returns (O, LSE or None)."""
+    """As mw_bca_cache_fwd_sink (k_sink may be None) with RoPE re-shifting
+    (Sec. 3.5): queries, in-flight and ring keys rotated at their stream
+    positions, the sink at its own, ``shift_frames`` frames evicted; the
+    sink's keys turn forward by the shift as they are read.  Returns
+    (O, LSE or None)."""
     return _cache_fwd(q, k_new, v_new, k_sink, v_sink, k_cache, v_cache, cache_head, cache_len,
                       T_chunk, scale, need_lse, workspace, out,
-                      rope=(rope_dims, rope_base, tokens_per_frame, first_frame))
+                      rope=(rope_dims, rope_base, shift_frames))
 
 
 def _cache_fwd(q, k_new, v_new, k_sink, v_sink, k_cache, v_cache, cache_head, cache_len,
@@ -342,7 +344,7 @@ def _cache_fwd(q, k_new, v_new, k_sink, v_sink, k_cache, v_cache, cache_head, ca
         _check(library().mw_bca_cache_fwd_rope(
             _ptr(q), _ptr(k_new), _ptr(v_new), _ptr(k_sink), _ptr(v_sink), sink_len,
             _ptr(k_cache), _ptr(v_cache), cap, cache_head, cache_len, int(rope[0]),
-            float(rope[1]), int(rope[2]), int(rope[3]), _ptr(o), _ptr(lse),
+            float(rope[1]), int(rope[2]), _ptr(o), _ptr(lse),
             _ptr(workspace), ws_bytes, B, H, W, T_chunk, d,
             _scale(scale, d), _stream()))
     elif k_sink is None:

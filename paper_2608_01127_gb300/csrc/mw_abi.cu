@@ -300,8 +300,7 @@ mw_status launch_status(cudaError_t e, const char* what) {
 struct RopeArgs {
   int dims = 0;          // 0: off
   mw::RopeFreq omega{};
-  int per_frame = 1;
-  int first_frame = 0;
+  int shift = 0;         // frames the sink anchor's keys turn forward
 };
 
 // omega_i = base^(-2i / dims) in fp64, split into float hi + lo
@@ -361,9 +360,8 @@ mw_status fwd_common(const void* q, const void* k, const void* v, const void* kr
   p.ring_head = len > 0 ? head : 0;
   p.ring_len = len;
   p.sink_len = sink_len;
-  p.rope_dims = len > 0 ? rope.dims : 0;
-  p.rope_per_frame = rope.per_frame;
-  p.rope_first_frame = rope.first_frame;
+  p.rope_dims = sink_len > 0 ? rope.dims : 0;
+  p.rope_shift = rope.shift;
   p.num_splits = splits;
   p.scale_log2 = scale * 1.4426950408889634f;
   p.o = static_cast<__nv_bfloat16*>(o);
@@ -578,7 +576,7 @@ mw_status mw_bca_cache_fwd_sink(const void* q, const void* k_new, const void* v_
                                 void* workspace, size_t ws_bytes, int B, int H, int n_q_chunks,
                                 int T_chunk, int d, float scale, void* stream) {
   return mw_bca_cache_fwd_rope(q, k_new, v_new, k_sink, v_sink, sink_len, k_cache, v_cache,
-                               cache_cap, cache_head, cache_len, 0, 0.f, 1, 0, o, lse, workspace,
+                               cache_cap, cache_head, cache_len, 0, 0.f, 0, o, lse, workspace,
                                ws_bytes, B, H, n_q_chunks, T_chunk, d, scale, stream);
 }
 
@@ -588,7 +586,7 @@ static mw_status cache_fwd_impl(const void* q, const void* k_new, const void* v_
                                 const void* k_sink, const void* v_sink, int sink_len,
                                 const void* k_cache, const void* v_cache, int cache_cap,
                                 int cache_head, int cache_len, int rope_dims, float rope_base,
-                                int tokens_per_frame, int first_frame, void* o, float* lse,
+                                int shift_frames, void* o, float* lse,
                                 void* workspace, size_t ws_bytes, int B, int H, int n_q_chunks,
                                 int T_chunk, int d, float scale, const mw::CommitJob& commit,
                                 void* stream) {
@@ -613,17 +611,15 @@ static mw_status cache_fwd_impl(const void* q, const void* k_new, const void* v_
       return fail(MW_ERR_INVALID_ARG, "rope_dims=%d must be even and in [0, d=%d]", rope_dims, d);
     if (!(rope_base > 1.f) || !(rope_base < 1e30f))
       return fail(MW_ERR_INVALID_ARG, "rope_base must be > 1 and finite");
-    if (tokens_per_frame < 1)
-      return fail(MW_ERR_INVALID_ARG, "tokens_per_frame=%d must be >= 1", tokens_per_frame);
-    if (first_frame < 0 ||
-        static_cast<long long>(first_frame) + (cache_len > 0 ? (cache_len - 1) / tokens_per_frame : 0) >
-            (1 << 24))
-      return fail(MW_ERR_INVALID_ARG,
-                  "first_frame=%d: ring frame positions must stay in [0, 2^24]", first_frame);
-    rope.dims = rope_dims;
-    rope.omega = rope_freq(rope_dims, rope_base);
-    rope.per_frame = tokens_per_frame;
-    rope.first_frame = first_frame;
+    if (shift_frames < 0 || shift_frames > (1 << 24))
+      return fail(MW_ERR_INVALID_ARG, "shift_frames=%d not in [0, 2^24]", shift_frames);
+    // only the sink's angles change, so without a sink or a shift this is the
+    // plain forward
+    if (sink_len > 0 && shift_frames > 0) {
+      rope.dims = rope_dims;
+      rope.omega = rope_freq(rope_dims, rope_base);
+      rope.shift = shift_frames;
+    }
   }
   MW_TRY(check_ptr(q, "q"));
   MW_TRY(check_ptr(k_new, "k_new"));
@@ -659,11 +655,11 @@ mw_status mw_bca_cache_fwd_rope(const void* q, const void* k_new, const void* v_
                                 const void* k_sink, const void* v_sink, int sink_len,
                                 const void* k_cache, const void* v_cache, int cache_cap,
                                 int cache_head, int cache_len, int rope_dims, float rope_base,
-                                int tokens_per_frame, int first_frame, void* o, float* lse,
+                                int shift_frames, void* o, float* lse,
                                 void* workspace, size_t ws_bytes, int B, int H, int n_q_chunks,
                                 int T_chunk, int d, float scale, void* stream) {
   return cache_fwd_impl(q, k_new, v_new, k_sink, v_sink, sink_len, k_cache, v_cache, cache_cap,
-                        cache_head, cache_len, rope_dims, rope_base, tokens_per_frame, first_frame,
+                        cache_head, cache_len, rope_dims, rope_base, shift_frames,
                         o, lse, workspace, ws_bytes, B, H, n_q_chunks, T_chunk, d, scale,
                         mw::CommitJob{}, stream);
 }
@@ -696,7 +692,7 @@ mw_status mw_bca_cache_step(const void* q, const void* k_new, const void* v_new,
     job.BH = B * H;
   }
   return cache_fwd_impl(q, k_new, v_new, nullptr, nullptr, 0, k_cache, v_cache, cache_cap,
-                        cache_head, cache_len, 0, 0.f, 1, 0, o, lse, workspace, ws_bytes, B, H,
+                        cache_head, cache_len, 0, 0.f, 0, o, lse, workspace, ws_bytes, B, H,
                         n_q_chunks, T_chunk, d, scale, job, stream);
 }
 

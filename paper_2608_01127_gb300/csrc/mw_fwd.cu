@@ -11,9 +11,9 @@
 //   warps 0-3 / 4-7  softmax of query tile 0 / 1 (one thread per row = TMEM lane)
 //   warp 8           TMA producer (Q once, then K/V tiles through a ring of stages)
 //   warp 9           tcgen05 issuer (S = Q K^T into TMEM, O += P V with P in TMEM)
-//   warps 10-11      RoPE re-shift of ring key tiles in shared memory when it
-//                    is enabled (otherwise idle; they complete warpgroup 2 for
-//                    the register re-split)
+//   warps 10-11      RoPE re-shift of the sink anchor's key tiles in shared
+//                    memory when it is enabled (otherwise idle; they complete
+//                    warpgroup 2 for the register re-split)
 // TMEM (512 columns): S_t at column 128 t (P_t, bf16, overwrites its first 64
 // columns), O_t at 256 + D t.
 #include "mw_internal.h"
@@ -50,12 +50,10 @@ struct FwdLayout {
   static constexpr int SUM_COL = DM;                  // first row-sum column of O
   static constexpr int OFF_ONES = OFF_V + STAGES * TILE_BYTES;
   static constexpr int ONES_BYTES = (D == 64) ? REGION_BYTES : 0;
-  // RoPE re-shift: per-pair frequencies, then (cos, sin) per (frame, pair) for
-  // up to ROPE_FRAMES frames of the tile being rotated
-  // (one copy per rotating warp)
-  static constexpr int ROPE_FRAMES = 4;
+  // RoPE re-shift: (cos, sin) of the shift per channel pair (one copy per
+  // rotating warp)
   static constexpr int OFF_ROPE = OFF_ONES + ONES_BYTES;
-  static constexpr int ROPE_WARP_BYTES = 2 * (D / 2) * 4 + ROPE_FRAMES * (D / 2) * 8;
+  static constexpr int ROPE_WARP_BYTES = (D / 2) * 8;
   static constexpr int ROPE_BYTES = 2 * ROPE_WARP_BYTES;
   static constexpr int OFF_BAR = OFF_ROPE + ROPE_BYTES;
   static constexpr int NBAR = 1 + 6 * STAGES + 3 * QT + 1;
@@ -121,9 +119,9 @@ __device__ __forceinline__ TileSrc tile_src(const Segs& g, int j) {
   return s;
 }
 
-// ROPE: the cache form with the ring's RoPE re-shift (warps 10-11 rotate ring
-// key tiles before the MMAs read them); the training and plain cache forms
-// are compiled without it.
+// ROPE: the cache form with the RoPE re-shift of the sink anchor (warps 10-11
+// turn its key tiles before the MMAs read them); the training and plain
+// cache forms are compiled without it.
 template <int D, int DM, bool ROPE>
 __global__ void __launch_bounds__(FwdLayout<D, DM>::THREADS, 1)
     bca_fwd_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_k,
@@ -347,7 +345,9 @@ __global__ void __launch_bounds__(FwdLayout<D, DM>::THREADS, 1)
         const uint32_t ph = (i / NS) & 1;
         const int stp = (i + NS - 1) % NS;
         const uint32_t php = ((i - 1) / NS) & 1;
-        if (!(ok = warp_wait(ROPE ? &k_rdy[st] : &k_full[st], ph, ctl))) break;
+        // with the re-shift, a sink tile is read once warps 10-11 have turned it
+        const bool turned = ROPE && j0 + i < g.nS;
+        if (!(ok = warp_wait(turned ? &k_rdy[st] : &k_full[st], ph, ctl))) break;
         tc_fence_after();
         // unrolled over the compile-time tile count, so every descriptor
         // offset stays a constant (a runtime trip count here slows the whole
@@ -394,23 +394,21 @@ __global__ void __launch_bounds__(FwdLayout<D, DM>::THREADS, 1)
       }
     }
   } else if (ROPE && (warp == 10 || warp == 11) && n_local > 0) {
-    // ------------------------------------------------------------ RoPE re-shift
-    // Ring keys are stored without their temporal rotation; after evictions the
-    // window is re-indexed from its start (Sec. 3.5), so ring token t (logical
-    // order) is rotated to frame first_frame + t / per_frame here, in shared
-    // memory, between the TMA copy and the MMAs that read the tile.  Channel
-    // pair (2i, 2i+1), i < rope_dims / 2, turns by frame * base^(-2i/rope_dims).
-    // Each of the two warps turns its own half of every ring tile (rows
+    // ------------------------------------------------------------ RoPE re-shift of the sink
+    // Queries, in-flight keys and ring keys carry their temporal rotation at
+    // stream positions.  Re-shifting (Sec. 3.5) moves the window back by the
+    // evicted frames and leaves the sink anchor at its position; since the
+    // scores depend only on position differences, that changes just the
+    // query-sink angles, exactly as turning the sink's keys forward by
+    // rope_shift frames does.  That happens here, in shared memory, between
+    // the TMA copy of a sink tile and the MMAs that read it: channel pair
+    // (2i, 2i+1), i < rope_dims / 2, turns by rope_shift * base^(-2i/rope_dims).
+    // Each of the two warps turns its own half of every sink tile (rows
     // [64 h, 64 h + 64)), so they never wait for each other.
     const int half = warp - 10;
-    float* omega = reinterpret_cast<float*>(smem + L::OFF_ROPE + half * L::ROPE_WARP_BYTES);
-    float* omega_lo = omega + D / 2;
-    float2* table = reinterpret_cast<float2*>(omega + D);  // [ROPE_FRAMES][4 n_ch]
+    float2* cs = reinterpret_cast<float2*>(smem + L::OFF_ROPE + half * L::ROPE_WARP_BYTES);
     const int pairs = p.rope_dims / 2;
-    for (int i = lane; i < pairs; i += 32) {
-      omega[i] = rope_om.hi[i];
-      omega_lo[i] = rope_om.lo[i];
-    }
+    for (int i = lane; i < pairs; i += 32) cs[i] = rope_cos_sin(p.rope_shift, rope_om.hi[i], rope_om.lo[i]);
     __syncwarp();
     // lane -> (row within a pass, 16-byte chunk of 8 channels = 4 pairs)
     const int n_ch = (pairs + 3) / 4;
@@ -421,67 +419,31 @@ __global__ void __launch_bounds__(FwdLayout<D, DM>::THREADS, 1)
     const int np = min(4, pairs - 4 * my_ch);        // pairs of the chunk that turn
     const int region_off = (c0 >> 6) * L::REGION_BYTES;
     const int cidx = (c0 & 63) >> 3;                 // chunk index within the 128-byte row
-    auto angle_cs = [&](int f, int pi) { return rope_cos_sin(f, omega[pi], omega_lo[pi]); };
-    auto turn = [](uint32_t w, float2 csn) { return rope_turn(w, csn); };
-    for (int i = 0; i < n_local; ++i) {
+    const float4 c01 = reinterpret_cast<const float4*>(cs)[2 * my_ch];
+    const float4 c23 = reinterpret_cast<const float4*>(cs)[2 * my_ch + 1];
+    const int n_sink = min(n_local, g.nS - j0);     // a block visits the sink first
+    for (int i = 0; i < n_sink; ++i) {
       const int st = i % NS;
       if (!warp_wait(&k_full[st], (i / NS) & 1, ctl)) break;
       const TileSrc src = tile_src(g, j0 + i);
       const int r_lo = 64 * half;
       const int nrows = min(64, src.end - src.row0 - r_lo);  // valid rows of this half
-      if (src.seg == kSegRing && nrows > 0) {
+      if (active && nrows > 0) {
         uint8_t* tile = sK + st * L::TILE_BYTES + region_off;
-        const int t_lo = src.t0 + r_lo;
-        const int f_lo = p.rope_first_frame + t_lo / p.rope_per_frame;
-        const int nf = p.rope_first_frame + (t_lo + nrows - 1) / p.rope_per_frame - f_lo + 1;
-        const bool tabled = nf <= L::ROPE_FRAMES;
-        if (tabled) {  // (cos, sin) once per frame and pair; rows of 4 n_ch pairs (32-byte aligned)
-          for (int e = lane; e < nf * pairs; e += 32)
-            table[(e / pairs) * (4 * n_ch) + e % pairs] = angle_cs(f_lo + e / pairs, e % pairs);
-          __syncwarp();
-        }
-        if (active && tabled) {
-          // rows before the first frame boundary use table row 0, the next
-          // per_frame rows row 1, ... (no division per row)
-          const int b0 = (f_lo + 1 - p.rope_first_frame) * p.rope_per_frame - t_lo;
-          const int P = p.rope_per_frame;
-          const int pi0 = 4 * my_ch;
 #pragma unroll 2
-          for (int rr = my_r; rr < nrows; rr += rpp) {
-            const int r = r_lo + rr;
-            const int fi = (rr >= b0) + (rr >= b0 + P) + (rr >= b0 + 2 * P);
-            const float4* cs = reinterpret_cast<const float4*>(table + fi * (4 * n_ch) + pi0);
-            // 128-byte swizzle: 16-byte chunk index ^ (row mod 8)
-            uint4* a = reinterpret_cast<uint4*>(tile + r * 128 + ((cidx ^ (r & 7)) << 4));
-            uint4 v = *a;
-            const float4 c01 = cs[0];
-            v.x = turn(v.x, make_float2(c01.x, c01.y));
-            if (np > 1) v.y = turn(v.y, make_float2(c01.z, c01.w));
-            if (np > 2) {
-              const float4 c23 = cs[1];
-              v.z = turn(v.z, make_float2(c23.x, c23.y));
-              if (np > 3) v.w = turn(v.w, make_float2(c23.z, c23.w));
-            }
-            *a = v;
-          }
-        } else if (active) {  // many frames in one tile (short frames): angles per row
-#pragma unroll 1
-          for (int rr = my_r; rr < nrows; rr += rpp) {
-            const int r = r_lo + rr;
-            const int f = p.rope_first_frame + (t_lo + rr) / p.rope_per_frame;
-            const int pi0 = 4 * my_ch;
-            uint4* a = reinterpret_cast<uint4*>(tile + r * 128 + ((cidx ^ (r & 7)) << 4));
-            uint4 v = *a;
-            v.x = turn(v.x, angle_cs(f, pi0));
-            if (np > 1) v.y = turn(v.y, angle_cs(f, pi0 + 1));
-            if (np > 2) v.z = turn(v.z, angle_cs(f, pi0 + 2));
-            if (np > 3) v.w = turn(v.w, angle_cs(f, pi0 + 3));
-            *a = v;
-          }
+        for (int rr = my_r; rr < nrows; rr += rpp) {
+          const int r = r_lo + rr;
+          // 128-byte swizzle: 16-byte chunk index ^ (row mod 8)
+          uint4* a = reinterpret_cast<uint4*>(tile + r * 128 + ((cidx ^ (r & 7)) << 4));
+          uint4 v = *a;
+          v.x = rope_turn(v.x, make_float2(c01.x, c01.y));
+          if (np > 1) v.y = rope_turn(v.y, make_float2(c01.z, c01.w));
+          if (np > 2) v.z = rope_turn(v.z, make_float2(c23.x, c23.y));
+          if (np > 3) v.w = rope_turn(v.w, make_float2(c23.z, c23.w));
+          *a = v;
         }
-        fence_proxy_async_smem();  // the tensor core reads the tile next
-        __syncwarp();              // every lane is done with the table
       }
+      fence_proxy_async_smem();  // the tensor core reads the tile next
       __syncwarp();
       if (lane == 0) mbar_arrive(&k_rdy[st]);
     }

@@ -44,12 +44,11 @@ struct FwdParams {
   int ring_head;
   int ring_len;
   int sink_len;     // tokens of the sink anchor, visited before the ring
-  // RoPE re-shift of ring keys on read (0 rope_dims: off): ring token t turns
-  // to frame rope_first_frame + t / rope_per_frame (the frequencies are a
-  // kernel parameter of their own)
+  // RoPE re-shift (0 rope_dims: off): the sink anchor's keys turn forward by
+  // rope_shift frames as they are read (the frequencies are a kernel
+  // parameter of their own)
   int rope_dims;
-  int rope_per_frame;
-  int rope_first_frame;
+  int rope_shift;
   int num_splits;   // 1: write bf16 O + LSE; >1: fp32 partials for the combine
   float scale_log2; // softmax scale * log2(e)
   __nv_bfloat16* o;

@@ -135,9 +135,9 @@ def test_sink_entry_rejects_bad_sink(mw):
 def test_rope_entry_rejects_bad_rope(mw):
     lib = mw.library()
 
-    def call(dims=32, base=1e4, per_frame=440, first=1):
+    def call(dims=32, base=1e4, shift=3):
         return lib.mw_bca_cache_fwd_rope(FAKE, FAKE, FAKE, None, None, 0, FAKE, FAKE, 1024, 0,
-                                         1024, dims, base, per_frame, first, FAKE, None, None, 0,
+                                         1024, dims, base, shift, FAKE, None, None, 0,
                                          1, 2, 1, 64, 128, 0.1, None)
 
     assert call(dims=-2) == INVALID
@@ -145,9 +145,8 @@ def test_rope_entry_rejects_bad_rope(mw):
     assert call(dims=130) == INVALID      # more than d
     assert call(base=1.0) == INVALID
     assert call(base=float("nan")) == INVALID
-    assert call(per_frame=0) == INVALID
-    assert call(first=-1) == INVALID
-    assert call(first=(1 << 24) - 1, per_frame=440) == INVALID  # ring frames past 2^24
+    assert call(shift=-1) == INVALID
+    assert call(shift=(1 << 24) + 1) == INVALID  # angles past 2^24 frames
 
 
 def test_step_rejects_bad_commit(mw):

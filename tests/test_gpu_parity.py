@@ -340,19 +340,21 @@ def test_qkv_split_rope_training_shape(mw):
         _check_qkv(qkv[:, sl].contiguous(), 32, 1e4, P, t0 // P, part)
 
 
-def test_qkv_split_rope_matches_the_fused_ring_rotation(mw):
-    """Keys turned by the split kernel and stored rotated give bit for bit the
-    same attention as un-rotated ring keys turned on read (both round the same
-    fp32 rotation to bf16; head 0 keeps the key tiles identical)."""
-    B, H, T, cap, d, P, first = 1, 2, 128, 1280, 64, 200, 5
+@pytest.mark.parametrize("d", [64, 128])
+def test_qkv_split_rope_matches_the_fused_sink_rotation(mw, d):
+    """Sink keys turned by the split kernel and stored rotated give bit for bit
+    the attention of the re-shift, which turns them as it reads them (both
+    round the same fp32 rotation to bf16)."""
+    B, H, T, cap, S, shift = 1, 2, 128, 1280, 300, 77
     g = torch.Generator().manual_seed(19)
     q, kn, vn = (torch.randn(B, H, T, d, generator=g).to(torch.bfloat16).cuda() for _ in range(3))
     kr, vr = (torch.randn(B, H, cap, d, generator=g).to(torch.bfloat16).cuda() for _ in range(2))
-    o1, l1 = mw.mw_bca_cache_fwd_rope(q, kn, vn, None, None, kr, vr, 0, cap, T, 32, 1e4, P, first)
-    qkv = torch.zeros(B, cap, 3, H, d, dtype=torch.bfloat16, device="cuda")
-    qkv[:, :, 1] = kr.permute(0, 2, 1, 3)
-    _, k_rot, _ = mw.mw_qkv_rope_split(qkv, 32, 1e4, P, first)
-    o2, l2 = mw.mw_bca_cache_fwd(q, kn, vn, k_rot, vr, 0, cap, T)
+    ks, vs = (torch.randn(B, H, S, d, generator=g).to(torch.bfloat16).cuda() for _ in range(2))
+    o1, l1 = mw.mw_bca_cache_fwd_rope(q, kn, vn, ks, vs, kr, vr, 100, cap, T, 32, 1e4, shift)
+    qkv = torch.zeros(B, S, 3, H, d, dtype=torch.bfloat16, device="cuda")
+    qkv[:, :, 1] = ks.permute(0, 2, 1, 3)
+    _, ks_rot, _ = mw.mw_qkv_rope_split(qkv, 32, 1e4, S, shift)  # every sink token at frame `shift`
+    o2, l2 = mw.mw_bca_cache_fwd_sink(q, kn, vn, ks_rot, vs, kr, vr, 100, cap, T)
     torch.cuda.synchronize()
     assert torch.equal(o1, o2) and torch.equal(l1, l2)
 
@@ -517,21 +519,25 @@ def test_sink_anchor_config(mw):
 
 
 ROPE_SMALL = [
-    # B, H, W, T, cap, length, head, sink, d, rope_dims, per_frame, first_frame, splits
-    (1, 2, 1, 64, 512, 512, 100, 0, 128, 32, 64, 1, 0),      # tiles span two frames
-    (1, 2, 2, 100, 1000, 300, 900, 32, 64, 64, 7, 0, 0),     # every channel, many frames per tile
-    (1, 1, 1, 880, 1760, 1760, 1759, 440, 128, 16, 440, 1, 3),  # one-frame sink, frames of 440
-    (2, 1, 2, 64, 640, 640, 0, 0, 64, 2, 1, 5, 0),           # one token per frame
-    (1, 2, 1, 64, 512, 512, 200, 16, 72, 24, 64, 1, 2),     # padded head dim, sink, splits
-    (1, 2, 1, 64, 512, 512, 300, 0, 64, 64, 2, (1 << 24) - 255, 0),  # the largest frames
+    # B, H, W, T, cap, length, head, sink, d, rope_dims, shift, splits (0 = automatic)
+    (1, 2, 1, 64, 512, 512, 100, 32, 128, 32, 8, 0),          # a quarter-tile sink
+    (1, 2, 2, 100, 1000, 300, 900, 32, 64, 64, 1000, 0),      # every channel, a large shift
+    (1, 1, 1, 880, 1760, 1760, 1759, 440, 128, 16, 4, 3),     # one-frame sink, forced splits
+    (2, 1, 2, 64, 640, 640, 0, 200, 64, 2, 1, 0),             # sink over two tiles, one pair
+    (1, 2, 1, 64, 512, 512, 200, 16, 72, 24, 7, 2),           # padded head dim, splits
+    (1, 2, 1, 64, 512, 512, 300, 130, 64, 64, (1 << 24) - 5, 0),  # the largest shifts
+    (1, 2, 1, 64, 512, 512, 300, 0, 64, 32, 50, 0),           # no sink: nothing turns
+    (1, 2, 1, 64, 512, 512, 300, 64, 64, 32, 0, 0),           # nothing evicted yet
 ]
 
 
-@pytest.mark.parametrize("B,H,W,T,cap,length,head,sink,d,rope_dims,per_frame,first,splits",
-                         ROPE_SMALL)
-def test_cache_forward_rope_reshift(mw, B, H, W, T, cap, length, head, sink, d, rope_dims,
-                                    per_frame, first, splits):
-    q, kn, vn, kr, vr = _ring_case(B, H, W, T, cap, d, seed=cap + rope_dims + per_frame)
+@pytest.mark.parametrize("B,H,W,T,cap,length,head,sink,d,rope_dims,shift,splits", ROPE_SMALL)
+def test_cache_forward_rope_reshift(mw, B, H, W, T, cap, length, head, sink, d, rope_dims, shift,
+                                    splits):
+    """Queries, in-flight and ring keys stand for keys rotated at stream
+    positions (any bf16 values are), the sink for keys at its own position;
+    the oracle re-indexes the window by the shift as Sec. 3.5 describes."""
+    q, kn, vn, kr, vr = _ring_case(B, H, W, T, cap, d, seed=cap + rope_dims + sink)
     g = torch.Generator().manual_seed(sink + 11)
     ks, vs = (torch.randn(B, H, sink, d, generator=g).to(torch.bfloat16) for _ in range(2))
     sc, base = 1.0 / math.sqrt(d), 10000.0
@@ -540,22 +546,22 @@ def test_cache_forward_rope_reshift(mw, B, H, W, T, cap, length, head, sink, d, 
         o, lse = mw.mw_bca_cache_fwd_rope(q.cuda(), kn.cuda(), vn.cuda(),
                                           ks.cuda() if sink else None, vs.cuda() if sink else None,
                                           kr.cuda(), vr.cuda(), head, length, T, rope_dims, base,
-                                          per_frame, first, sc)
+                                          shift, sc)
     finally:
         mw.mw_set_option("cache_splits", 0)
-    o_ref, lse_ref = oracle.cache_fwd(q, kn, vn, kr, vr, cap, head, length, T, sc,
-                                      ks if sink else None, vs if sink else None,
-                                      rope=(rope_dims, base, per_frame, first))
-    tag = f"rope{rope_dims} P{per_frame} first{first} sink{sink} len{length} splits{splits}"
+    o_ref, lse_ref = oracle.cache_fwd_reshift(q, kn, vn, kr, vr, cap, head, length, T, sc, ks, vs,
+                                              rope_dims, base, shift)
+    tag = f"rope{rope_dims} shift{shift} sink{sink} len{length} splits{splits}"
     check_o(o, o_ref, tag)
     check_lse(lse, lse_ref, tag)
 
 
 def test_rope_reshift_streaming(mw):
-    """Streaming with a sink and a FIFO ring whose keys are stored without their
-    temporal rotation: each step the in-flight chunk is rotated to the frames
-    after the window (test side), attends, and its unrotated keys are
-    committed; evictions re-index the window without rewriting the ring."""
+    """Streaming with a one-frame sink and a FIFO ring: every chunk's queries
+    and keys are rotated once, at their stream frames (frame 0 is the sink's,
+    the stream's tokens follow from frame 1), and the keys are committed as
+    they are; after evictions the window is re-indexed by the evicted frames,
+    which here only turns the sink as it is read."""
     B, H, T, d, P, cap, sink = 1, 2, 64, 128, 32, 256, 32
     rope_dims, base, sc = 32, 10000.0, 1.0 / math.sqrt(d)
     g = torch.Generator().manual_seed(41)
@@ -565,23 +571,27 @@ def test_rope_reshift_streaming(mw):
     vr = torch.zeros(B, H, cap, d, dtype=torch.bfloat16)
     ring = mw.RingState(cap, 0, 0)
     kr_g, vr_g = kr.cuda(), vr.cuda()
-    first = sink // P  # the ring starts right after the sink frame(s)
+    evicted = 0  # tokens that have left the ring
     for step in range(7):  # the ring fills after 4 steps, then evicts
         q_raw, k_raw, v_new = (torch.randn(B, H, T, d, generator=g).to(torch.bfloat16)
                                for _ in range(3))
-        frames = first + ring.length // P + torch.arange(T) // P
+        frames = 1 + (step * T + torch.arange(T)) // P
         q = oracle.rope_rotate(q_raw, frames, rope_dims, base).to(torch.bfloat16)
         k = oracle.rope_rotate(k_raw, frames, rope_dims, base).to(torch.bfloat16)
+        shift = evicted // P
         o, lse = mw.mw_bca_cache_fwd_rope(q.cuda(), k.cuda(), v_new.cuda(), ks.cuda(), vs.cuda(),
                                           kr_g, vr_g, ring.head, ring.length, T, rope_dims, base,
-                                          P, first, sc)
-        o_ref, lse_ref = oracle.cache_fwd(q, k, v_new, kr, vr, cap, ring.head, ring.length, T, sc,
-                                          ks, vs, rope=(rope_dims, base, P, first))
-        check_o(o, o_ref, f"stream step {step}")
+                                          shift, sc)
+        o_ref, lse_ref = oracle.cache_fwd_reshift(q, k, v_new, kr, vr, cap, ring.head, ring.length,
+                                                  T, sc, ks, vs, rope_dims, base, shift)
+        check_o(o, o_ref, f"stream step {step} shift {shift}")
         check_lse(lse, lse_ref, f"stream step {step}")
+        before = ring.length
         slot = ring.commit(T)
-        mw.mw_bca_cache_commit(kr_g, vr_g, slot, k_raw.cuda(), v_new.cuda())
-        kr, vr = oracle.cache_commit(kr, vr, cap, slot, k_raw, v_new)
+        evicted += before + T - ring.length
+        mw.mw_bca_cache_commit(kr_g, vr_g, slot, k.cuda(), v_new.cuda())
+        kr, vr = oracle.cache_commit(kr, vr, cap, slot, k, v_new)
+    assert evicted == 3 * T
 
 
 def test_device_status_is_clean(mw):
