@@ -240,6 +240,54 @@ def oracle_sample(seconds: float, rank_seed: int = 0, max_heads: int = 24):
     return per_head * heads / dt / 1e12, heads, dt
 
 
+def oracle_config_baselines(seconds: float = 5.0):
+    """The fp64 oracle, as it stands, on the host cores for the other
+    workloads: whole (b, h) heads until about `seconds` have passed (at least
+    one), scaled to the metric of each (TFLOP/s for training fwd+bwd; for the
+    cache workloads the time of one full call, all heads, in microseconds)."""
+    import oracle
+    res = {}
+    cfg = TRAIN_CONFIGS["train_h16_d128_peaky"]
+    x = gen_train(cfg)
+    per_head = (fwd_flops(train_pairs(cfg), cfg.d) + bwd_flops(train_pairs(cfg), cfg.d)) / (cfg.B * cfg.H)
+    t0, heads = time.perf_counter(), 0
+    while heads < cfg.B * cfg.H:
+        b, h = divmod(heads, cfg.H)
+        sl = (slice(b, b + 1), slice(h, h + 1))
+        q, k, v, do = (x[n][sl] for n in ("q", "k", "v", "do"))
+        oracle.fwd(q, k, v, cfg.T, cfg.scale)
+        oracle.bwd(q, k, v, do, cfg.T, cfg.scale)
+        heads += 1
+        if time.perf_counter() - t0 >= seconds:
+            break
+    dt = time.perf_counter() - t0
+    res["train_h16_d128_peaky"] = {
+        "value": round(per_head * heads / dt / 1e12, 6), "unit": "TFLOP/s (fwd+bwd)",
+        "cores": torch.get_num_threads(), "kind": "oracle",
+        "sample": f"fp64 oracle fwd+bwd of {heads} of {cfg.B * cfg.H} heads ({dt:.1f} s)"}
+    for name in ("rolling_cache", "pipelined"):
+        cfg = CACHE_CONFIGS[name]
+        x = gen_cache(cfg, steps=1)
+        q, kn, vn, kr, vr = x["q"][0], x["k_new"][0], x["v_new"][0], x["k_ring"], x["v_ring"]
+        t0, heads = time.perf_counter(), 0
+        while heads < cfg.B * cfg.H:
+            b, h = divmod(heads, cfg.H)
+            sl = (slice(b, b + 1), slice(h, h + 1))
+            oracle.cache_fwd(q[sl], kn[sl], vn[sl], kr[sl], vr[sl], cfg.cap, cfg.head, cfg.length,
+                             cfg.T, cfg.scale)
+            heads += 1
+            if time.perf_counter() - t0 >= seconds:
+                break
+        dt = time.perf_counter() - t0
+        us = dt / heads * cfg.B * cfg.H * 1e6
+        res[name] = {"value": round(us, 1), "unit": "us per call (all heads)",
+                     "tflops": round(fwd_flops(cache_pairs(cfg), cfg.d) / (us / 1e6) / 1e12, 6),
+                     "cores": torch.get_num_threads(), "kind": "oracle",
+                     "sample": f"fp64 oracle cache forward of {heads} of {cfg.B * cfg.H} heads, "
+                               f"scaled to all heads ({dt:.1f} s)"}
+    return res
+
+
 def cpu_cores() -> int:
     try:
         return len(os.sched_getaffinity(0))
@@ -403,7 +451,9 @@ def run_ours(args):
     out["clocks"] = clk.summary()
     out["e2e"] = run_e2e(mw, cfg, dev, args, world, step_flops)
     if rank == 0 and world == 1 and not args.no_extras:
-        out["extra"] = run_extras(mw, dev, peaks)
+        out["extra"] = run_extras(mw, dev, peaks, args=args)
+        if not args.no_cpu_baseline:
+            out["extra"]["cpu_baseline_per_config"] = oracle_config_baselines()
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         tf, heads, dt = oracle_sample(args.cpu_seconds)
         out["cpu_baseline"] = {"value": round(tf, 6), "unit": "TFLOP/s", "cores": torch.get_num_threads(),
@@ -526,7 +576,7 @@ EXTRA_NAMES = ("train_h16_d128_peaky", "train_1b_32x600", "train_05b_d72", "roll
                "pipelined", "sink_anchor", "qkv_rope_split")
 
 
-def run_extras(mw, dev, peaks, only=None):
+def run_extras(mw, dev, peaks, only=None, args=None):
     """The secondary workloads (all, or the names in `only`)."""
     flush_buf = torch.empty(L2_FLUSH_BYTES, dtype=torch.uint8, device=dev)
     flush = flush_buf.zero_
@@ -556,6 +606,27 @@ def run_extras(mw, dev, peaks, only=None):
             "fwd_tflops": round(fwd_flops(pairs, cfg.d) / fm / 1e9, 2),
             "fwd_bwd_tflops": round((fwd_flops(pairs, cfg.d) + bwd_flops(pairs, cfg.d))
                                     / (fm + bm) / 1e9, 2)}
+        if name == "train_h16_d128_peaky":
+            # the largest training workload, reported like the headline: its
+            # dominant kernel (the backward key-tile kernel, timed alone) and
+            # the step end to end through the API with host buffers
+            mw.mw_bca_bwd(q, k, v, o, lse, do, cfg.T, cfg.scale, workspace=ws, out=grads, stage=1)
+            tm = time_repeated(lambda: mw.mw_bca_bwd(q, k, v, o, lse, do, cfg.T, cfg.scale,
+                                                     workspace=ws, out=grads, stage=2), 10, flush=flush)
+            mm = statistics.median(tm)
+            ach = bwd_flops(pairs, cfg.d) / mm / 1e9
+            extra[name]["roofline"] = {
+                "kernel": f"bca_bwd_kernel<{cfg.d}, {cfg.d}> (backward key-tile kernel)",
+                "bound": "tensor", "achieved": round(ach, 2), "peak": peaks["bf16_tflops"],
+                "peak_source": peaks["source"] + " bf16 burst", "unit": "TFLOP/s",
+                "frac": round(ach / peaks["bf16_tflops"], 4),
+                "frac_of_sustained": round(ach / peaks["bf16_tflops_sustained"], 4),
+                "traffic": profiled_traffic(f"bca_bwd_kernel<{cfg.d},{cfg.d}>", name),
+                "algorithmic_bytes": bwd_main_bytes(cfg), "ms_per_launch": round(mm, 4),
+                "share_of_step": round(mm / (fm + bm), 4)}
+            if args is not None:
+                extra[name]["e2e"] = run_e2e(mw, cfg, dev, args, 1,
+                                             fwd_flops(pairs, cfg.d) + bwd_flops(pairs, cfg.d))
         del q, k, v, do, o, lse, ws, grads
     if "rolling_cache" in want:
         extra["rolling_cache"] = bench_rolling(mw, dev, peaks)
