@@ -166,6 +166,25 @@ def test_long_sequence_sampled_rows_and_invariants(mw, d, N, T):
     assert float((dv64.sum(0) - sum_do).norm() / sum_do.norm()) < 2e-2
 
 
+def test_head_groups_of_unequal_size(mw):
+    """Seven heads of 64K tokens: the forward schedules its query blocks in
+    head groups of about four waves of CTAs (here 3 + 2 + 2 heads), the
+    larger group first; every head's rows come out as the oracle's (sampled
+    rows of a head from each group)."""
+    B, H, N, T, d = 1, 7, 65536, 4096, 64
+    q, k, v, _ = _inputs(B, H, N // T, T, d, seed=61)
+    sc = 1.0 / math.sqrt(d)
+    o, lse = mw.mw_bca_fwd(q.cuda(), k.cuda(), v.cuda(), T, sc)
+    torch.cuda.synchronize()
+    g = torch.Generator().manual_seed(13)
+    rows = sorted(set([0, T - 1, N // 2, N - 1] + torch.randint(0, N, (8,), generator=g).tolist()))
+    for h in (0, 2, 3, 6):
+        o_ref, lse_ref = oracle.fwd_rows(q[0, h], k[0, h], v[0, h], T, sc, rows)
+        check_o(o[0, h, rows], o_ref, f"head {h}")
+        check_lse(lse[0, h, rows], lse_ref, f"head {h}")
+    assert mw.mw_device_status() == 0
+
+
 def test_forward_is_deterministic_and_stays_in_bounds(mw):
     B, H, n, T, d = 1, 2, 3, 100, 64
     q, k, v, _ = _inputs(B, H, n, T, d, seed=7)
