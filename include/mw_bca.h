@@ -318,6 +318,12 @@ mw_status mw_device_status(void* stream, int clear);
  *                      (default 2000)
  *   "debug_skip_q_load" non-zero: forward kernels never load Q, so their
  *                      first wait expires; for testing the timeout path only
+ *   "fwd_group_waves"  forward CTAs per head group, in multiples of the SM
+ *                      count (default 2; 0 restores it): the query blocks of
+ *                      a group's heads run together and share their K/V in L2
+ *   "pdl"              0 launches the forward, the split combine and the
+ *                      commit without programmatic dependent launch
+ *                      (default 1)
  * Returns MW_ERR_INVALID_ARG for an unknown name or a negative value.
  */
 mw_status mw_set_option(const char* name, long long value);

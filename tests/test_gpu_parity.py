@@ -168,8 +168,8 @@ def test_long_sequence_sampled_rows_and_invariants(mw, d, N, T):
 
 def test_head_groups_of_unequal_size(mw):
     """Seven heads of 64K tokens: the forward schedules its query blocks in
-    head groups of about four waves of CTAs (here 3 + 2 + 2 heads), the
-    larger group first; every head's rows come out as the oracle's (sampled
+    head groups of about two waves of CTAs (here 2 + 2 + 2 + 1 heads), the
+    larger groups first; every head's rows come out as the oracle's (sampled
     rows of a head from each group)."""
     B, H, N, T, d = 1, 7, 65536, 4096, 64
     q, k, v, _ = _inputs(B, H, N // T, T, d, seed=61)
@@ -178,7 +178,7 @@ def test_head_groups_of_unequal_size(mw):
     torch.cuda.synchronize()
     g = torch.Generator().manual_seed(13)
     rows = sorted(set([0, T - 1, N // 2, N - 1] + torch.randint(0, N, (8,), generator=g).tolist()))
-    for h in (0, 2, 3, 6):
+    for h in (0, 3, 4, 6):
         o_ref, lse_ref = oracle.fwd_rows(q[0, h], k[0, h], v[0, h], T, sc, rows)
         check_o(o[0, h, rows], o_ref, f"head {h}")
         check_lse(lse[0, h, rows], lse_ref, f"head {h}")
