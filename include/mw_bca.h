@@ -321,6 +321,9 @@ mw_status mw_device_status(void* stream, int clear);
  *   "fwd_group_waves"  forward CTAs per head group, in multiples of the SM
  *                      count (default 2; 0 restores it): the query blocks of
  *                      a group's heads run together and share their K/V in L2
+ *   "bwd_group_heads"  heads per group of the backward's CTA order, 0 =
+ *                      automatic (groups sized by their work, Q/dO/dQ
+ *                      bytes within 48 MB); 1 = one head after another
  *   "pdl"              0 launches the forward, the split combine and the
  *                      commit without programmatic dependent launch
  *                      (default 1)

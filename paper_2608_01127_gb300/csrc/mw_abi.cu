@@ -33,6 +33,7 @@ long long g_opt_cache_splits = 0;
 long long g_opt_budget_ms = 2000;
 long long g_opt_skip_q = 0;
 long long g_opt_group_waves = 2;
+long long g_opt_bwd_group_heads = 0;
 
 mw_status fail(mw_status s, const char* fmt, ...) {
   char buf[512];
@@ -220,6 +221,33 @@ int plan_splits(int BH, int rows_q, int cache_len) {
     }
   }
   return best;
+}
+
+// Head groups of the backward's CTA order.  A key tile's CTA runs one step
+// per visible query tile, plus a fixed cost of about three; the longest CTA
+// (the first key tile) must start at least twice its length before the end,
+// so the last group holds at least twice its work on every SM.  A group's
+// Q, dO and fp32 dQ accumulator (what its CTAs share through L2) stay
+// within 48 MB.  Groups of nearly equal size; one group per head when the
+// heads alone are that large.
+int bwd_head_groups(int BH, int N_pad, int T, int qrows, int d_io, int D) {
+  if (g_opt_bwd_group_heads > 0) return ceil_div(BH, std::min<long long>(BH, g_opt_bwd_group_heads));
+  constexpr long long kFixed = 3;
+  constexpr long long kGroupBytes = 48LL << 20;
+  const int n_kt = N_pad / mw::kTileRows;
+  const int n_qt = N_pad / qrows;
+  long long per_head = 0, longest = 0;
+  for (int kt = 0; kt < n_kt; ++kt) {
+    const long long first_q = static_cast<long long>(kt) * mw::kTileRows / T * T;
+    const long long w = n_qt - first_q / qrows + kFixed;
+    per_head += w;
+    longest = std::max(longest, w);
+  }
+  const long long head_bytes = static_cast<long long>(N_pad) * (4LL * d_io + 4LL * D + 32);
+  const long long per_group = std::max(1LL, std::min<long long>(
+      std::min<long long>(BH, kGroupBytes / head_bytes),
+      (2 * longest * sm_count() + per_head - 1) / per_head));
+  return ceil_div(BH, per_group);
 }
 
 size_t cache_ws_bytes(int splits, int BH, int rows_q, int d) {
@@ -423,6 +451,8 @@ mw_status mw_set_option(const char* name, long long value) {
     g_opt_skip_q = value;
   } else if (std::strcmp(name, "fwd_group_waves") == 0) {
     g_opt_group_waves = value > 0 ? value : 2;
+  } else if (std::strcmp(name, "bwd_group_heads") == 0) {
+    g_opt_bwd_group_heads = value;
   } else if (std::strcmp(name, "pdl") == 0) {
     mw::g_pdl_enabled = value != 0;
   } else {
@@ -523,6 +553,7 @@ mw_status mw_bca_bwd_stage(int stage, const void* q, const void* k, const void* 
     if (bias != nullptr) MW_TRY(encode_bias_map(&tbias, bias, N_pad, BH, qrows));
     mw::BwdParams p{};
     p.BH = BH;
+    p.head_groups = bwd_head_groups(BH, N_pad, T_chunk, qrows, d, D);
     p.N = static_cast<int>(N);
     p.N_pad = N_pad;
     p.d_io = d;

@@ -154,11 +154,32 @@ __global__ void __launch_bounds__(BwdLayout<D, DM>::THREADS, 1)
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
 
-  // ---- work item: head-major (the CTAs running together share one head's
-  // Q, dO and dQ accumulator in L2), key tiles near the start (most work) first
+  // ---- work item: p.head_groups groups of heads one after another (sizes
+  // differ by at most one, the larger first), so that the CTAs running
+  // together share a few heads' Q, dO and dQ accumulator in L2; inside a
+  // group the key tiles near the start (the most work) come first, those of
+  // all the group's heads side by side, so that the longest CTAs of the last
+  // group do not start near the end of the launch
   const int n_kt = p.N_pad / kTileRows;
-  const int bh = blockIdx.x / n_kt;
-  const int kt = blockIdx.x % n_kt;
+  int bh, kt;
+  {
+    const int x = blockIdx.x;
+    const int g_base = p.BH / p.head_groups, g_rem = p.BH % p.head_groups;
+    const int big = (g_base + 1) * n_kt;  // CTAs of one larger group
+    int gsize, h0, in_grp;
+    if (x < g_rem * big) {
+      gsize = g_base + 1;
+      h0 = (x / big) * gsize;
+      in_grp = x % big;
+    } else {
+      const int y = x - g_rem * big;
+      gsize = g_base;
+      h0 = g_rem * (g_base + 1) + (y / (g_base * n_kt)) * g_base;
+      in_grp = y % (g_base * n_kt);
+    }
+    bh = h0 + in_grp % gsize;
+    kt = in_grp / gsize;
+  }
   const int k0 = kt * kTileRows;
   const int first_q = (k0 / p.T) * p.T;  // first query that sees key k0
   const int m_begin = first_q / QN;

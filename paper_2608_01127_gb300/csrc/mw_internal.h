@@ -62,6 +62,7 @@ struct FwdParams {
 
 struct BwdParams {
   int BH;
+  int head_groups;  // CTA order: groups of heads one after another
   int N;            // tokens per (b,h)
   int N_pad;        // N rounded up to kTileRows
   int d_io;         // head dim of the caller's tensors (<= the kernel's D)

@@ -185,6 +185,35 @@ def test_head_groups_of_unequal_size(mw):
     assert mw.mw_device_status() == 0
 
 
+def test_backward_head_groups_of_unequal_size(mw):
+    """Seven heads of 32K tokens: the backward schedules its key tiles in
+    head groups sized by their work and L2 footprint (here 2 + 2 + 2 + 1
+    heads), the key tiles of a group's heads side by side, the first
+    (longest) ones first.  Sampled dQ rows and dK, dV key rows of a head
+    from each group against the oracle's row-by-row forms, and
+    sum_j dV_j = sum_i dO_i on every head."""
+    B, H, N, T, d = 1, 7, 32768, 2048, 64
+    q, k, v, do = _inputs(B, H, N // T, T, d, seed=67)
+    sc = 1.0 / math.sqrt(d)
+    qc, kc, vc, doc = (t.cuda() for t in (q, k, v, do))
+    o, lse = mw.mw_bca_fwd(qc, kc, vc, T, sc)
+    dq, dk, dv = mw.mw_bca_bwd(qc, kc, vc, o, lse, doc, T, sc)
+    torch.cuda.synchronize()
+    g = torch.Generator().manual_seed(17)
+    rows = sorted(set([0, N // 2, N - 1] + torch.randint(0, N, (5,), generator=g).tolist()))
+    krows = sorted(set([0, 127, 128, N - T, N - 1] + torch.randint(0, N, (3,), generator=g).tolist()))
+    for h in (0, 2, 4, 6):
+        q1, k1, v1, do1 = (t[0, h] for t in (q, k, v, do))
+        check_grad(dq[0, h, rows], oracle.dq_rows(q1, k1, v1, do1, T, sc, rows), f"head {h} dQ")
+        dk_ref, dv_ref = oracle.dkv_rows(q1, k1, v1, do1, T, sc, krows)
+        check_grad(dk[0, h, krows], dk_ref, f"head {h} dK")
+        check_grad(dv[0, h, krows], dv_ref, f"head {h} dV")
+    sum_do = do[0].double().sum(1)
+    err = (dv[0].double().cpu().sum(1) - sum_do).norm(dim=-1) / sum_do.norm(dim=-1)
+    assert float(err.max()) < 2e-2, err
+    assert mw.mw_device_status() == 0
+
+
 def test_forward_is_deterministic_and_stays_in_bounds(mw):
     B, H, n, T, d = 1, 2, 3, 100, 64
     q, k, v, _ = _inputs(B, H, n, T, d, seed=7)
