@@ -316,8 +316,9 @@ mw_status mw_device_status(void* stream, int clear);
  *                      (the workspace size follows this setting)
  *   "wait_budget_ms"   time limit of every bounded wait inside the kernels
  *                      (default 2000)
- *   "debug_skip_q_load" non-zero: forward kernels never load Q, so their
- *                      first wait expires; for testing the timeout path only
+ *   "debug_skip_q_load" non-zero: the forward and backward kernels never
+ *                      load Q, so their first wait expires; for testing the
+ *                      timeout path only
  *   "fwd_group_waves"  forward CTAs per head group, in multiples of the SM
  *                      count (default 2; 0 restores it): the query blocks of
  *                      a group's heads run together and share their K/V in L2

@@ -567,6 +567,7 @@ mw_status mw_bca_bwd_stage(int stage, const void* q, const void* k, const void* 
     p.dv = static_cast<__nv_bfloat16*>(dv);
     p.status = status;
     p.budget_ns = budget_ns();
+    p.debug_skip_q = static_cast<int>(g_opt_skip_q);
     MW_TRY(launch_status(mw::launch_bwd_main(D, mma_d(d), tq, tk, tv, tdo, tdq, tbias, p, s),
                          "backward kernel launch"));
   }

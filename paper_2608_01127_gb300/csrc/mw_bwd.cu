@@ -127,33 +127,6 @@ __global__ void __launch_bounds__(BwdLayout<D, DM>::THREADS, 1)
   constexpr int QN = L::QN;
   constexpr int CW = L::CW;
   extern __shared__ __align__(1024) uint8_t smem[];
-  if ((smem_u32(smem) & 1023u) != 0u) {
-    if (threadIdx.x == 0) atomicOr(p.status, kDevMisaligned);
-    return;  // uniform across the CTA, before any barrier or TMEM use
-  }
-  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + L::OFF_BAR);
-  uint64_t* kv_full = bars;
-  uint64_t* q_full = bars + 1;
-  uint64_t* q_empty = q_full + NS;
-  uint64_t* do_full = q_empty + NS;
-  uint64_t* do_empty = do_full + NS;
-  uint64_t* s_full = do_empty + NS;
-  uint64_t* s_free = s_full + 1;
-  uint64_t* dp_full = s_free + 1;
-  uint64_t* dp_free = dp_full + 1;
-  uint64_t* pt_ready = dp_free + 1;
-  uint64_t* pt_free = pt_ready + 1;
-  uint64_t* p_ready = pt_free + 1;
-  uint64_t* dq_full = p_ready + 1;
-  uint64_t* dq_free = dq_full + 1;
-  uint64_t* ds_free = dq_free + 1;
-  uint64_t* dkv_full = ds_free + L::DS_BUFS;
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + L::OFF_MISC);
-  volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + L::OFF_MISC + 4);
-
-  const int warp = threadIdx.x >> 5;
-  const int lane = threadIdx.x & 31;
-
   // ---- work item: p.head_groups groups of heads one after another (sizes
   // differ by at most one, the larger first), so that the CTAs running
   // together share a few heads' Q, dO and dQ accumulator in L2; inside a
@@ -180,6 +153,43 @@ __global__ void __launch_bounds__(BwdLayout<D, DM>::THREADS, 1)
     bh = h0 + in_grp % gsize;
     kt = in_grp / gsize;
   }
+  if ((smem_u32(smem) & 1023u) != 0u) {
+    // nothing runs without aligned shared memory: report it, and give this
+    // key tile's dK and dV rows a defined value (zero) instead of leaving
+    // stale ones behind
+    if (threadIdx.x == 0) atomicOr(p.status, kDevMisaligned);
+    const int krow = kt * kTileRows + static_cast<int>(threadIdx.x & 127);
+    if (threadIdx.x < 256 && krow < p.N) {
+      const int d_io = (D == 64) ? D : p.d_io;
+      __nv_bfloat16* out = threadIdx.x < 128 ? p.dk : p.dv;
+      uint4* dst = reinterpret_cast<uint4*>(out + (static_cast<size_t>(bh) * p.N + krow) * d_io);
+      for (int c = 0; c < d_io / 8; ++c) dst[c] = make_uint4(0u, 0u, 0u, 0u);
+    }
+    return;  // uniform across the CTA, before any barrier or TMEM use
+  }
+  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + L::OFF_BAR);
+  uint64_t* kv_full = bars;
+  uint64_t* q_full = bars + 1;
+  uint64_t* q_empty = q_full + NS;
+  uint64_t* do_full = q_empty + NS;
+  uint64_t* do_empty = do_full + NS;
+  uint64_t* s_full = do_empty + NS;
+  uint64_t* s_free = s_full + 1;
+  uint64_t* dp_full = s_free + 1;
+  uint64_t* dp_free = dp_full + 1;
+  uint64_t* pt_ready = dp_free + 1;
+  uint64_t* pt_free = pt_ready + 1;
+  uint64_t* p_ready = pt_free + 1;
+  uint64_t* dq_full = p_ready + 1;
+  uint64_t* dq_free = dq_full + 1;
+  uint64_t* ds_free = dq_free + 1;
+  uint64_t* dkv_full = ds_free + L::DS_BUFS;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + L::OFF_MISC);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + L::OFF_MISC + 4);
+
+  const int warp = threadIdx.x >> 5;
+  const int lane = threadIdx.x & 31;
+
   const int k0 = kt * kTileRows;
   const int first_q = (k0 / p.T) * p.T;  // first query that sees key k0
   const int m_begin = first_q / QN;
@@ -260,14 +270,16 @@ __global__ void __launch_bounds__(BwdLayout<D, DM>::THREADS, 1)
         const int q0 = (m_begin + (j + q_rot) % n_q) * QN;
         const size_t voff = static_cast<size_t>(bh) * p.N_pad + q0;
         if (!mbar_wait(&q_empty[st], ph ^ 1, ctl)) break;
-        mbar_arrive_expect_tx(&q_full[st], L::QTILE + L::BIAS_BYTES + L::VEC_BYTES);
-        for (int r = 0; r < L::REG; ++r)
-          tma_load_3d(sQ + st * L::QSTRIDE + r * L::QREGION, &tm_q, &q_full[st], 64 * r, q0, bh);
-        if constexpr (L::FOLD)
-          tma_load_3d(sQ + st * L::QSTRIDE + L::QTILE, &tm_bias, &q_full[st], 0, q0, bh);
-        else
-          bulk_load(sLSE + st * QN, p.lse2 + voff, L::VEC_BYTES, &q_full[st]);
-        ++issued_q;
+        if (!p.debug_skip_q) {
+          mbar_arrive_expect_tx(&q_full[st], L::QTILE + L::BIAS_BYTES + L::VEC_BYTES);
+          for (int r = 0; r < L::REG; ++r)
+            tma_load_3d(sQ + st * L::QSTRIDE + r * L::QREGION, &tm_q, &q_full[st], 64 * r, q0, bh);
+          if constexpr (L::FOLD)
+            tma_load_3d(sQ + st * L::QSTRIDE + L::QTILE, &tm_bias, &q_full[st], 0, q0, bh);
+          else
+            bulk_load(sLSE + st * QN, p.lse2 + voff, L::VEC_BYTES, &q_full[st]);
+          ++issued_q;
+        }
         if (!mbar_wait(&do_empty[st], ph ^ 1, ctl)) break;
         mbar_arrive_expect_tx(&do_full[st], L::QTILE + L::VEC_BYTES);
         for (int r = 0; r < L::REG; ++r)
@@ -607,11 +619,12 @@ __global__ void __launch_bounds__(BwdLayout<D, DM>::THREADS, 1)
       }
     }
     // ---- epilogue: warpgroup 0 writes dK (x scale), warpgroup 1 writes dV
+    // (zeros if a wait gave up: the rows get a defined value either way)
     const bool have = ok && warp_wait(dkv_full, 0, ctl);
     tc_fence_after();
-    if (have) {
+    {
       const uint32_t col0 = wg == 0 ? L::DK_COL : L::DV_COL;
-      const float mul = wg == 0 ? p.scale : 1.f;
+      const float mul = have ? (wg == 0 ? p.scale : 1.f) : 0.f;
       __nv_bfloat16* out = wg == 0 ? p.dk : p.dv;
       // the caller's rows hold d_io <= D columns (multiples of 8); only the
       // 128-wide kernel serves padded head dims
@@ -620,8 +633,13 @@ __global__ void __launch_bounds__(BwdLayout<D, DM>::THREADS, 1)
 #pragma unroll
       for (int c = 0; c < (DM + 31) / 32; ++c) {  // the chunks holding the DM columns
         uint32_t r[32];
-        tmem_ld32(lane_base + col0 + 32 * c, r);
-        tmem_wait_ld();
+        if (have) {
+          tmem_ld32(lane_base + col0 + 32 * c, r);
+          tmem_wait_ld();
+        } else {
+#pragma unroll
+          for (int k = 0; k < 32; ++k) r[k] = 0u;
+        }
         if (k_valid && 32 * c < d_io) {
           const int n16 = min(4, (d_io - 32 * c) / 8);
           uint4* dst = reinterpret_cast<uint4*>(out + row_off + 32 * c);

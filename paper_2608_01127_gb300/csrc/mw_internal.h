@@ -76,6 +76,7 @@ struct BwdParams {
   __nv_bfloat16* dv;
   unsigned* status;
   unsigned long long budget_ns;
+  int debug_skip_q;  // test hook: never load Q, so the first S^T wait expires
 };
 
 // A ring commit (Sec. 3.5): rows [0, rows) of each head of k_src / v_src
