@@ -16,6 +16,8 @@
 //                    warpgroup 2 for the register re-split)
 // TMEM (512 columns): S_t at column 128 t (P_t, bf16, overwrites its first 64
 // columns), O_t at 256 + D t.
+#include <type_traits>
+
 #include "mw_internal.h"
 #include "mw_ptx.cuh"
 
@@ -687,30 +689,40 @@ __global__ void __launch_bounds__(256) combine_kernel(const float* __restrict__ 
   const int row = blockIdx.x * 8 + (threadIdx.x >> 5);
   const int lane = threadIdx.x & 31;
   if (row >= n_rows) return;
-  float m = -INFINITY;
-  for (int s = 0; s < splits; ++s) m = fmaxf(m, lse_part[static_cast<size_t>(s) * n_rows + row]);
   constexpr int PER = D / 32;
   float acc[PER];
 #pragma unroll
   for (int k = 0; k < PER; ++k) acc[k] = 0.f;
-  float wsum = 0.f;
-  for (int s = 0; s < splits; ++s) {
-    const float ls = lse_part[static_cast<size_t>(s) * n_rows + row];
-    if (ls == -INFINITY) continue;
-    const float w = __expf(ls - m);
+  float wsum = 0.f, m = -INFINITY;
+  using Vec = typename std::conditional<PER == 4, float4, float2>::type;  // a lane's columns
+  // a split whose LSE is -inf saw no key of the row: its O part is skipped
+  // (never multiplied: it may hold anything)
+  auto add = [&](float ls, const Vec& x) {
+    const float w = ls == -INFINITY ? 0.f : __expf(ls - m);
     wsum += w;
-    const float* src = o_part + (static_cast<size_t>(s) * n_rows + row) * D + lane * PER;
-    if constexpr (PER == 4) {  // one 16-byte load per lane
-      const float4 x = *reinterpret_cast<const float4*>(src);
+    if (w > 0.f) {
       acc[0] += w * x.x;
       acc[1] += w * x.y;
-      acc[2] += w * x.z;
-      acc[3] += w * x.w;
-    } else {  // PER == 2: one 8-byte load per lane
-      const float2 x = *reinterpret_cast<const float2*>(src);
-      acc[0] += w * x.x;
-      acc[1] += w * x.y;
+      if constexpr (PER == 4) {
+        acc[2] += w * x.z;
+        acc[3] += w * x.w;
+      }
     }
+  };
+  const Vec* src0 = reinterpret_cast<const Vec*>(o_part + static_cast<size_t>(row) * D) + lane;
+  const size_t split_stride = static_cast<size_t>(n_rows) * D / PER;  // in Vec
+  if (splits == 2) {
+    // the usual case: both LSEs and both O parts requested at once (one
+    // memory round trip instead of four)
+    const float l0 = lse_part[row], l1 = lse_part[static_cast<size_t>(n_rows) + row];
+    const Vec x0 = src0[0], x1 = src0[split_stride];
+    m = fmaxf(l0, l1);
+    add(l0, x0);
+    add(l1, x1);
+  } else {
+    for (int s = 0; s < splits; ++s) m = fmaxf(m, lse_part[static_cast<size_t>(s) * n_rows + row]);
+    for (int s = 0; s < splits; ++s)
+      add(lse_part[static_cast<size_t>(s) * n_rows + row], src0[s * split_stride]);
   }
   const float inv = wsum > 0.f ? 1.f / wsum : 0.f;
   __nv_bfloat16* dst = o + static_cast<size_t>(row) * d_io + lane * PER;
