@@ -320,7 +320,7 @@ mw_status mw_device_status(void* stream, int clear);
  *                      load Q, so their first wait expires; for testing the
  *                      timeout path only
  *   "fwd_group_waves"  forward CTAs per head group, in multiples of the SM
- *                      count (default 2; 0 restores it): the query blocks of
+ *                      count (default 3; 0 restores it): the query blocks of
  *                      a group's heads run together and share their K/V in L2
  *   "bwd_group_heads"  heads per group of the backward's CTA order, 0 =
  *                      automatic (groups sized by their work, Q/dO/dQ

@@ -32,7 +32,7 @@ std::mutex g_mutex;
 long long g_opt_cache_splits = 0;
 long long g_opt_budget_ms = 2000;
 long long g_opt_skip_q = 0;
-long long g_opt_group_waves = 2;
+long long g_opt_group_waves = 3;
 long long g_opt_bwd_group_heads = 0;
 
 mw_status fail(mw_status s, const char* fmt, ...) {
@@ -377,11 +377,13 @@ mw_status fwd_common(const void* q, const void* k, const void* v, const void* kr
   p.d_io = d;
   p.T = T;
   p.n_qblocks = ceil_div(rows_q, mw::kFwdBlockRows);
-  // head groups of about two waves of CTAs each: a group's K/V stay in L2
+  // head groups of about three waves of CTAs each: a group's K/V stay in L2
   // while its query blocks run, and the longest blocks of each group start
   // first; groups of (nearly) equal size keep the last one from ending late
   // (at d = 128, groups of four waves hold 8 heads' K/V, 76 MB, and miss L2
-  // often enough to read 1.44x the algorithmic bytes; two waves, 0.95x)
+  // often enough to read 1.44x the algorithmic bytes, three waves 1.04x;
+  // two waves, 0.95x, leave more group boundaries, which cost the cache
+  // forward with a sink anchor 4%)
   {
     const int per_group = std::max(1, std::min(BH, ceil_div(g_opt_group_waves * sm_count(),
                                                             static_cast<long long>(p.n_qblocks) * splits)));
@@ -450,7 +452,7 @@ mw_status mw_set_option(const char* name, long long value) {
   } else if (std::strcmp(name, "debug_skip_q_load") == 0) {
     g_opt_skip_q = value;
   } else if (std::strcmp(name, "fwd_group_waves") == 0) {
-    g_opt_group_waves = value > 0 ? value : 2;
+    g_opt_group_waves = value > 0 ? value : 3;
   } else if (std::strcmp(name, "bwd_group_heads") == 0) {
     g_opt_bwd_group_heads = value;
   } else if (std::strcmp(name, "pdl") == 0) {

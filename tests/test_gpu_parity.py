@@ -168,9 +168,9 @@ def test_long_sequence_sampled_rows_and_invariants(mw, d, N, T):
 
 def test_head_groups_of_unequal_size(mw):
     """Seven heads of 64K tokens: the forward schedules its query blocks in
-    head groups of about two waves of CTAs (here 2 + 2 + 2 + 1 heads), the
-    larger groups first; every head's rows come out as the oracle's (sampled
-    rows of a head from each group)."""
+    head groups of about three waves of CTAs (here 2 + 2 + 2 + 1 heads),
+    the larger groups first; every head's rows come out as the oracle's
+    (sampled rows of a head from each group)."""
     B, H, N, T, d = 1, 7, 65536, 4096, 64
     q, k, v, _ = _inputs(B, H, N // T, T, d, seed=61)
     sc = 1.0 / math.sqrt(d)
