@@ -324,7 +324,9 @@ mw_status mw_device_status(void* stream, int clear);
  *                      a group's heads run together and share their K/V in L2
  *   "bwd_group_heads"  heads per group of the backward's CTA order, 0 =
  *                      automatic (groups sized by their work, Q/dO/dQ
- *                      bytes within 48 MB); 1 = one head after another
+ *                      bytes within 48 MB, taken where list scheduling
+ *                      predicts a 1% shorter launch); 1 = one head after
+ *                      another; head dims over 80 always run head by head
  *   "pdl"              0 launches the forward, the split combine and the
  *                      commit without programmatic dependent launch
  *                      (default 1)

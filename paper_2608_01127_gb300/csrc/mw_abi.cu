@@ -10,8 +10,13 @@
 #include <cstdio>
 #include <cmath>
 #include <cstring>
+#include <functional>
+#include <map>
 #include <mutex>
+#include <queue>
 #include <string>
+#include <tuple>
+#include <vector>
 
 #include "mw_bca.h"
 #include "mw_internal.h"
@@ -223,31 +228,86 @@ int plan_splits(int BH, int rows_q, int cache_len) {
   return best;
 }
 
+// Finish time of the last SM when CTAs of the given lengths start in the given
+// order, each on the SM that frees first (the hardware's dispatch, modelled
+// as list scheduling).
+long long list_makespan(const std::vector<int>& order_work, int sms) {
+  std::priority_queue<long long, std::vector<long long>, std::greater<long long>> free_at;
+  for (int i = 0; i < sms; ++i) free_at.push(0);
+  long long end = 0;
+  for (int w : order_work) {
+    const long long t = free_at.top() + w;
+    free_at.pop();
+    free_at.push(t);
+    end = std::max(end, t);
+  }
+  return end;
+}
+
+// CTA lengths of the backward in its launch order for `groups` head groups
+// (the kernel's decode: groups of nearly equal size, the larger first; in a
+// group, key tile after key tile, each over the group's heads)
+std::vector<int> bwd_order_work(const std::vector<int>& kt_work, int BH, int groups) {
+  const int n_kt = static_cast<int>(kt_work.size());
+  const int g_base = BH / groups, g_rem = BH % groups;
+  std::vector<int> out;
+  out.reserve(static_cast<size_t>(BH) * n_kt);
+  for (int g = 0; g < groups; ++g) {
+    const int gsize = g_base + (g < g_rem ? 1 : 0);
+    for (int kt = 0; kt < n_kt; ++kt)
+      for (int h = 0; h < gsize; ++h) out.push_back(kt_work[kt]);
+  }
+  return out;
+}
+
 // Head groups of the backward's CTA order.  A key tile's CTA runs one step
-// per visible query tile, plus a fixed cost of about three; the longest CTA
-// (the first key tile) must start at least twice its length before the end,
-// so the last group holds at least twice its work on every SM.  A group's
-// Q, dO and fp32 dQ accumulator (what its CTAs share through L2) stay
-// within 48 MB.  Groups of nearly equal size; one group per head when the
-// heads alone are that large.
+// per visible query tile, plus a fixed cost of about three.  Head by head
+// (groups of one head), the last head's longest key tiles start near the end
+// of the launch; grouping heads lets them start earlier.  The candidate:
+// the last group holds at least twice the longest CTA's steps on every SM,
+// and a group's Q, dO and fp32 dQ accumulator stay within 48 MB.  It is
+// taken when list scheduling puts its end at least 1% before that of head
+// by head (the grouped decode and its wider L2 footprint cost about that
+// much where the tail is small).  Decisions are cached per shape.  The
+// kernel variant with 128-wide MMAs always runs head by head.
 int bwd_head_groups(int BH, int N_pad, int T, int qrows, int d_io, int D) {
+  if (D == 128 && mma_d(d_io) == 128) return BH;  // that kernel variant runs head by head
   if (g_opt_bwd_group_heads > 0) return ceil_div(BH, std::min<long long>(BH, g_opt_bwd_group_heads));
-  constexpr long long kFixed = 3;
+  const int sms = sm_count();
+  static std::mutex mu;
+  static std::map<std::tuple<int, int, int, int, int, int, int>, int> cache;
+  const auto key = std::make_tuple(BH, N_pad, T, qrows, d_io, D, sms);
+  {
+    std::lock_guard<std::mutex> lock(mu);
+    const auto it = cache.find(key);
+    if (it != cache.end()) return it->second;
+  }
+  constexpr int kFixed = 3;
   constexpr long long kGroupBytes = 48LL << 20;
   const int n_kt = N_pad / mw::kTileRows;
   const int n_qt = N_pad / qrows;
+  std::vector<int> kt_work(n_kt);
   long long per_head = 0, longest = 0;
   for (int kt = 0; kt < n_kt; ++kt) {
     const long long first_q = static_cast<long long>(kt) * mw::kTileRows / T * T;
-    const long long w = n_qt - first_q / qrows + kFixed;
-    per_head += w;
-    longest = std::max(longest, w);
+    kt_work[kt] = static_cast<int>(n_qt - first_q / qrows + kFixed);
+    per_head += kt_work[kt];
+    longest = std::max<long long>(longest, kt_work[kt]);
   }
   const long long head_bytes = static_cast<long long>(N_pad) * (4LL * d_io + 4LL * D + 32);
   const long long per_group = std::max(1LL, std::min<long long>(
       std::min<long long>(BH, kGroupBytes / head_bytes),
-      (2 * longest * sm_count() + per_head - 1) / per_head));
-  return ceil_div(BH, per_group);
+      (2 * longest * sms + per_head - 1) / per_head));
+  int groups = BH;  // head by head
+  const int candidate = ceil_div(BH, per_group);
+  if (candidate < BH) {
+    const long long t_heads = list_makespan(bwd_order_work(kt_work, BH, BH), sms);
+    const long long t_groups = list_makespan(bwd_order_work(kt_work, BH, candidate), sms);
+    if (100 * t_groups <= 99 * t_heads) groups = candidate;
+  }
+  std::lock_guard<std::mutex> lock(mu);
+  cache.emplace(key, groups);
+  return groups;
 }
 
 size_t cache_ws_bytes(int splits, int BH, int rows_q, int d) {

@@ -97,6 +97,11 @@ struct BwdLayout {
   static constexpr uint32_t PDS_COL = SHARED_X ? S_COL : 384u;
   static constexpr uint32_t DQ_COL = SHARED_X ? 384u : 448u;
   static constexpr int THREADS = 512;
+  // CTA order in head groups (BwdParams::head_groups).  The 128-wide MMA
+  // variant runs head by head with the key tile taken straight from the CTA
+  // index: with the group decode it measured 2-3% slower even in head-by-
+  // head order, and its training shapes have no tail for groups to win back.
+  static constexpr bool GROUPED = !(D == 128 && DM == 128);
   // registers per thread after the re-split: the P/dS warpgroups get more,
   // the drain warpgroup and the control warpgroup (TMA, MMA) less; the three
   // shares add up to exactly the launch's 512 threads x 128 registers (at
@@ -134,8 +139,11 @@ __global__ void __launch_bounds__(BwdLayout<D, DM>::THREADS, 1)
   // all the group's heads side by side, so that the longest CTAs of the last
   // group do not start near the end of the launch
   const int n_kt = p.N_pad / kTileRows;
-  int bh, kt;
-  {
+  int bh_decoded, kt;
+  if constexpr (!L::GROUPED) {
+    bh_decoded = blockIdx.x / n_kt;
+    kt = blockIdx.x % n_kt;
+  } else {
     const int x = blockIdx.x;
     const int g_base = p.BH / p.head_groups, g_rem = p.BH % p.head_groups;
     const int big = (g_base + 1) * n_kt;  // CTAs of one larger group
@@ -150,7 +158,7 @@ __global__ void __launch_bounds__(BwdLayout<D, DM>::THREADS, 1)
       h0 = g_rem * (g_base + 1) + (y / (g_base * n_kt)) * g_base;
       in_grp = y % (g_base * n_kt);
     }
-    bh = h0 + in_grp % gsize;
+    bh_decoded = h0 + in_grp % gsize;
     kt = in_grp / gsize;
   }
   if ((smem_u32(smem) & 1023u) != 0u) {
@@ -162,7 +170,7 @@ __global__ void __launch_bounds__(BwdLayout<D, DM>::THREADS, 1)
     if (threadIdx.x < 256 && krow < p.N) {
       const int d_io = (D == 64) ? D : p.d_io;
       __nv_bfloat16* out = threadIdx.x < 128 ? p.dk : p.dv;
-      uint4* dst = reinterpret_cast<uint4*>(out + (static_cast<size_t>(bh) * p.N + krow) * d_io);
+      uint4* dst = reinterpret_cast<uint4*>(out + (static_cast<size_t>(bh_decoded) * p.N + krow) * d_io);
       for (int c = 0; c < d_io / 8; ++c) dst[c] = make_uint4(0u, 0u, 0u, 0u);
     }
     return;  // uniform across the CTA, before any barrier or TMEM use
@@ -186,18 +194,35 @@ __global__ void __launch_bounds__(BwdLayout<D, DM>::THREADS, 1)
   uint64_t* dkv_full = ds_free + L::DS_BUFS;
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + L::OFF_MISC);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + L::OFF_MISC + 4);
+  // In grouped order the head and key tile are read back from shared memory
+  // by each role, so that nothing derived from the decode above is held in a
+  // register from the kernel's start (the decode is too long for the
+  // compiler to redo, and the P/dS warps of the 80-wide variant spilled for
+  // it); head by head they come straight from the CTA index.
+  volatile int* head_slot = reinterpret_cast<volatile int*>(smem + L::OFF_MISC + 8);
+  volatile int* tile_slot = reinterpret_cast<volatile int*>(smem + L::OFF_MISC + 12);
+  auto head = [&]() -> int { return L::GROUPED ? *head_slot : static_cast<int>(blockIdx.x) / n_kt; };
+  struct Sweep {
+    int k0;       // first key row of the tile
+    int m_begin;  // first query tile that sees it
+    int n_q;      // query tiles visited
+    int q_rot;    // where the sweep starts: each key tile at its own offset,
+                  // so that the key tiles of one head running side by side
+                  // reduce into different dQ tiles instead of contending for
+                  // the same L2 lines
+  };
+  auto sweep = [&]() {
+    const int t = L::GROUPED ? *tile_slot : static_cast<int>(blockIdx.x) % n_kt;
+    Sweep w;
+    w.k0 = t * kTileRows;
+    w.m_begin = (w.k0 / p.T) * p.T / QN;  // the first query that sees key k0, in tiles
+    w.n_q = p.N_pad / QN - w.m_begin;
+    w.q_rot = t % w.n_q;
+    return w;
+  };
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
-
-  const int k0 = kt * kTileRows;
-  const int first_q = (k0 / p.T) * p.T;  // first query that sees key k0
-  const int m_begin = first_q / QN;
-  const int n_q = p.N_pad / QN - m_begin;
-  // each key tile starts its sweep over the query tiles at its own offset, so
-  // that the key tiles of one head running side by side reduce into different
-  // dQ tiles instead of contending for the same L2 lines
-  const int q_rot = kt % n_q;
 
   if constexpr (L::FOLD) {
     // A rows of the bias MMAs: [1 1 0 0 | 1 1 0 0] picks the LSE pair of a
@@ -211,6 +236,8 @@ __global__ void __launch_bounds__(BwdLayout<D, DM>::THREADS, 1)
     }
   }
   if (threadIdx.x == 0) {
+    *head_slot = bh_decoded;
+    *tile_slot = kt;
     mbar_init(kv_full, 1);
     for (int s = 0; s < NS; ++s) {
       mbar_init(&q_full[s], 1);
@@ -256,6 +283,8 @@ __global__ void __launch_bounds__(BwdLayout<D, DM>::THREADS, 1)
   if (warp == 12) {
     // ------------------------------------------------------------ TMA producer
     if (lane == 0) {
+      const int bh = head();
+      const auto [k0, m_begin, n_q, q_rot] = sweep();
       prefetch_tmap(&tm_q);
       prefetch_tmap(&tm_do);
       mbar_arrive_expect_tx(kv_full, 2 * L::KTILE);
@@ -297,6 +326,7 @@ __global__ void __launch_bounds__(BwdLayout<D, DM>::THREADS, 1)
     }
   } else if (warp == 13 || (L::TWO_ISSUERS && warp == 14)) {
     // ------------------------------------------------------------ MMA issuers (whole warps)
+    const int n_q = sweep().n_q;
     // d = 64: warp 13 issues S^T, dV and dP^T, warp 14 dK and dQ, so that one
     // warp's waits never leave the tensor core's short queue empty.  They
     // share no TMEM columns; the P/dS barriers order their operands.
@@ -469,6 +499,7 @@ __global__ void __launch_bounds__(BwdLayout<D, DM>::THREADS, 1)
   } else if (warp < 8) {
     regs_inc<L::REGS_PDS>();
     // ------------------------------------------------------------ P / dS (thread = key row)
+    const auto [k0, m_begin, n_q, q_rot] = sweep();
     const int wg = warp >> 2;            // query columns [CW wg, CW wg + CW)
     const int wq = warp & 3;             // TMEM lane quadrant
     const int j_local = wq * 32 + lane;
@@ -629,7 +660,7 @@ __global__ void __launch_bounds__(BwdLayout<D, DM>::THREADS, 1)
       // the caller's rows hold d_io <= D columns (multiples of 8); only the
       // 128-wide kernel serves padded head dims
       const int d_io = (D == 64) ? D : p.d_io;
-      const size_t row_off = (static_cast<size_t>(bh) * p.N + krow) * d_io;
+      const size_t row_off = (static_cast<size_t>(head()) * p.N + krow) * d_io;
 #pragma unroll
       for (int c = 0; c < (DM + 31) / 32; ++c) {  // the chunks holding the DM columns
         uint32_t r[32];
@@ -656,6 +687,8 @@ __global__ void __launch_bounds__(BwdLayout<D, DM>::THREADS, 1)
     regs_dec<L::REGS_DRAIN>();
     // ------------------------------------------------------------ dQ drain
     const int wq = warp & 3;
+    const int bh = head();
+    const auto [k0, m_begin, n_q, q_rot] = sweep();
     const uint32_t lane_base = tmem + (static_cast<uint32_t>(wq * 32) << 16);
     for (int j = 0; j < n_q; ++j) {
       const int q0 = (m_begin + (j + q_rot) % n_q) * QN;

@@ -186,13 +186,13 @@ def test_head_groups_of_unequal_size(mw):
 
 
 def test_backward_head_groups_of_unequal_size(mw):
-    """Seven heads of 32K tokens: the backward schedules its key tiles in
-    head groups sized by their work and L2 footprint (here 2 + 2 + 2 + 1
-    heads), the key tiles of a group's heads side by side, the first
-    (longest) ones first.  Sampled dQ rows and dK, dV key rows of a head
-    from each group against the oracle's row-by-row forms, and
-    sum_j dV_j = sum_i dO_i on every head."""
-    B, H, N, T, d = 1, 7, 32768, 2048, 64
+    """Eleven heads of 16K tokens: head by head, the last head's longest key
+    tiles would start near the end of the backward launch, so the key tiles
+    run in head groups (here 4 + 4 + 3 heads), those of a group's heads side
+    by side, the first (longest) ones first.  Sampled dQ rows and dK, dV key
+    rows of a head from each group against the oracle's row-by-row forms,
+    and sum_j dV_j = sum_i dO_i on every head."""
+    B, H, N, T, d = 1, 11, 16384, 2048, 64
     q, k, v, do = _inputs(B, H, N // T, T, d, seed=67)
     sc = 1.0 / math.sqrt(d)
     qc, kc, vc, doc = (t.cuda() for t in (q, k, v, do))
@@ -202,7 +202,7 @@ def test_backward_head_groups_of_unequal_size(mw):
     g = torch.Generator().manual_seed(17)
     rows = sorted(set([0, N // 2, N - 1] + torch.randint(0, N, (5,), generator=g).tolist()))
     krows = sorted(set([0, 127, 128, N - T, N - 1] + torch.randint(0, N, (3,), generator=g).tolist()))
-    for h in (0, 2, 4, 6):
+    for h in (0, 5, 10):
         q1, k1, v1, do1 = (t[0, h] for t in (q, k, v, do))
         check_grad(dq[0, h, rows], oracle.dq_rows(q1, k1, v1, do1, T, sc, rows), f"head {h} dQ")
         dk_ref, dv_ref = oracle.dkv_rows(q1, k1, v1, do1, T, sc, krows)
