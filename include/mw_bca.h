@@ -76,6 +76,20 @@ mw_status mw_bca_fwd(const void* q, const void* k, const void* v, void* o, float
 size_t mw_bca_bwd_workspace_size(int B, int H, int n_chunks, int T_chunk, int d);
 
 /*
+ * The CTA order the backward key-tile kernel takes for these sizes: the
+ * number of head groups its key tiles run in, one after another (B*H = one
+ * head after another).  Host-side planning only, no device work: with
+ * sm_count > 0 it plans for that many SMs, else for the current device.
+ * The heads form groups of nearly equal size, and in a group the key tiles
+ * of all its heads run side by side, the first (longest) ones first.  The
+ * groups are taken where a list-scheduling model of the launch ends at least
+ * 1% before head by head; head dims over 80 always run head by head; the
+ * option "bwd_group_heads" overrides the choice.  Returns -1 on invalid
+ * sizes (mw_last_error says why).
+ */
+int mw_bca_bwd_head_groups(int B, int H, int n_chunks, int T_chunk, int d, int sm_count);
+
+/*
  * Backward of mw_bca_fwd: the analytic gradient of sum(O * dO) with respect
  * to q, k, v (training in bf16 mixed precision, Sec. 4.1), P recomputed from
  * the saved LSE.

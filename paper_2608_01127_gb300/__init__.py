@@ -29,7 +29,8 @@ import torch
 __all__ = [
     "MWError", "library", "lib_path", "mw_bca_fwd", "mw_bca_bwd", "mw_bca_cache_fwd",
     "mw_bca_cache_fwd_sink", "mw_bca_cache_fwd_rope", "mw_bca_cache_step",
-    "mw_bca_cache_commit", "mw_bca_bwd_workspace_size", "mw_bca_cache_workspace_size",
+    "mw_bca_cache_commit", "mw_bca_bwd_workspace_size", "mw_bca_bwd_head_groups",
+    "mw_bca_cache_workspace_size",
     "mw_device_status", "mw_set_option", "mw_qkv_rope_split", "BlockCausalAttention",
     "EXPORTED_SYMBOLS",
     "RingState",
@@ -43,7 +44,7 @@ EXPORTED_SYMBOLS = (
     "mw_bca_cache_workspace_size",
     "mw_bca_cache_fwd", "mw_bca_cache_commit", "mw_status_string", "mw_last_error",
     "mw_device_status", "mw_set_option", "mw_bca_cache_fwd_noalloc", "mw_bca_cache_fwd_sink",
-    "mw_bca_cache_fwd_rope", "mw_qkv_rope_split", "mw_bca_cache_step",
+    "mw_bca_cache_fwd_rope", "mw_qkv_rope_split", "mw_bca_cache_step", "mw_bca_bwd_head_groups",
 )
 
 STATUS = {0: "MW_OK", 1: "MW_ERR_INVALID_ARG", 2: "MW_ERR_UNSUPPORTED", 3: "MW_ERR_CUDA",
@@ -79,6 +80,7 @@ def library() -> ctypes.CDLL:
     sig = {
         "mw_bca_fwd": (_I, [_P, _P, _P, _P, _P, _I, _I, _I, _I, _I, _F, _P]),
         "mw_bca_bwd_workspace_size": (_Z, [_I, _I, _I, _I, _I]),
+        "mw_bca_bwd_head_groups": (_I, [_I, _I, _I, _I, _I, _I]),
         "mw_bca_bwd": (_I, [_P, _P, _P, _P, _P, _P, _P, _P, _P, _P, _Z,
                             _I, _I, _I, _I, _I, _F, _P]),
         "mw_bca_bwd_stage": (_I, [_I, _P, _P, _P, _P, _P, _P, _P, _P, _P, _P, _Z,
@@ -232,6 +234,16 @@ def mw_bca_fwd(q: torch.Tensor, k: torch.Tensor, v: torch.Tensor, T_chunk: int,
 
 def mw_bca_bwd_workspace_size(B: int, H: int, n_chunks: int, T_chunk: int, d: int) -> int:
     return int(library().mw_bca_bwd_workspace_size(B, H, n_chunks, T_chunk, d))
+
+
+def mw_bca_bwd_head_groups(B: int, H: int, n_chunks: int, T_chunk: int, d: int,
+                           sm_count: int = 0) -> int:
+    """Head groups of the backward's CTA order for these sizes (B*H = head by
+    head); host-side planning only."""
+    g = int(library().mw_bca_bwd_head_groups(B, H, n_chunks, T_chunk, d, sm_count))
+    if g < 0:
+        raise MWError(1, library().mw_last_error().decode(errors="replace"))
+    return g
 
 
 def mw_bca_bwd(q, k, v, o, lse, dout, T_chunk: int, scale: Optional[float] = None,

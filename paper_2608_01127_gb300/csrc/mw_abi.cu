@@ -270,10 +270,9 @@ std::vector<int> bwd_order_work(const std::vector<int>& kt_work, int BH, int gro
 // by head (the grouped decode and its wider L2 footprint cost about that
 // much where the tail is small).  Decisions are cached per shape.  The
 // kernel variant with 128-wide MMAs always runs head by head.
-int bwd_head_groups(int BH, int N_pad, int T, int qrows, int d_io, int D) {
+int bwd_head_groups(int BH, int N_pad, int T, int qrows, int d_io, int D, int sms) {
   if (D == 128 && mma_d(d_io) == 128) return BH;  // that kernel variant runs head by head
   if (g_opt_bwd_group_heads > 0) return ceil_div(BH, std::min<long long>(BH, g_opt_bwd_group_heads));
-  const int sms = sm_count();
   static std::mutex mu;
   static std::map<std::tuple<int, int, int, int, int, int, int>, int> cache;
   const auto key = std::make_tuple(BH, N_pad, T, qrows, d_io, D, sms);
@@ -543,6 +542,20 @@ mw_status mw_bca_fwd(const void* q, const void* k, const void* v, void* o, float
                     static_cast<cudaStream_t>(stream));
 }
 
+int mw_bca_bwd_head_groups(int B, int H, int n_chunks, int T_chunk, int d, int sm_count_arg) {
+  if (check_dims(B, H, d) != MW_OK) return -1;
+  if (n_chunks < 1 || T_chunk < 1) {
+    fail(MW_ERR_INVALID_ARG, "n_chunks=%d and T_chunk=%d must be >= 1", n_chunks, T_chunk);
+    return -1;
+  }
+  const long long N = static_cast<long long>(n_chunks) * T_chunk;
+  if (check_rows(N, "n_chunks*T_chunk") != MW_OK) return -1;
+  const int N_pad = ceil_div(N, mw::kTileRows) * mw::kTileRows;
+  const int D = kernel_d(d);
+  return bwd_head_groups(B * H, N_pad, T_chunk, mw::bwd_q_rows(D), d, D,
+                         sm_count_arg > 0 ? sm_count_arg : sm_count());
+}
+
 size_t mw_bca_bwd_workspace_size(int B, int H, int n_chunks, int T_chunk, int d) {
   if (B < 1 || H < 1 || n_chunks < 1 || T_chunk < 1 || !d_supported(d)) return 0;
   const long long N = static_cast<long long>(n_chunks) * T_chunk;
@@ -615,7 +628,7 @@ mw_status mw_bca_bwd_stage(int stage, const void* q, const void* k, const void* 
     if (bias != nullptr) MW_TRY(encode_bias_map(&tbias, bias, N_pad, BH, qrows));
     mw::BwdParams p{};
     p.BH = BH;
-    p.head_groups = bwd_head_groups(BH, N_pad, T_chunk, qrows, d, D);
+    p.head_groups = bwd_head_groups(BH, N_pad, T_chunk, qrows, d, D, sm_count());
     p.N = static_cast<int>(N);
     p.N_pad = N_pad;
     p.d_io = d;

@@ -225,6 +225,73 @@ def test_workspace_follows_split_override(mw):
         lib.mw_set_option(b"cache_splits", 0)
 
 
+def _makespan(lengths, sms):
+    """List scheduling: each CTA, in order, starts on the SM that frees first."""
+    import heapq
+    free = [0] * sms
+    end = 0
+    for w in lengths:
+        t = heapq.heappop(free) + w
+        heapq.heappush(free, t)
+        end = max(end, t)
+    return end
+
+
+def _backward_plan(B, H, n, T, d, sms):
+    """The backward's CTA-order rule, restated: a key tile's length is the
+    query tiles that see it (+3); head groups hold at least twice the longest
+    tile's steps on every SM and at most 48 MB of Q, dO and fp32 dQ; they win
+    over head by head when the modelled launch ends >= 1% earlier."""
+    BH, N = B * H, n * T
+    N_pad = -(-N // 128) * 128
+    if d > 80 and d != 64:
+        return BH
+    D = 64 if d == 64 else 128
+    kt_len = [N_pad // 128 - (kt * 128 // T * T) // 128 + 3 for kt in range(N_pad // 128)]
+    cap = (48 << 20) // (N_pad * (4 * d + 4 * D + 32))
+    per_group = max(1, min(BH, cap, -(-2 * max(kt_len) * sms // sum(kt_len))))
+    cand = -(-BH // per_group)
+
+    def order(groups):
+        base, rem = divmod(BH, groups)
+        return [w for g in range(groups) for w in kt_len for _ in range(base + (g < rem))]
+
+    if cand < BH and 100 * _makespan(order(cand), sms) <= 99 * _makespan(order(BH), sms):
+        return cand
+    return BH
+
+
+@pytest.mark.parametrize("B,H,n,T,d,expect", [
+    (2, 12, 16, 880, 64, 4),     # the d=64 training workload: 4 groups of 6 heads
+    (1, 16, 16, 880, 72, 4),     # 80-wide MMAs, 16 heads: 4 groups of 4
+    (1, 11, 8, 2048, 64, 3),     # 4 + 4 + 3 heads
+    (1, 16, 21, 880, 128, 16),   # head dims over 80: head by head
+    (1, 12, 32, 600, 96, 12),
+    (1, 1, 4, 64, 64, 1),
+    (8, 16, 2, 256, 64, None),   # short sequences, many heads: whatever the model says
+])
+def test_backward_head_groups_follow_the_list_scheduling_rule(mw, B, H, n, T, d, expect):
+    got = mw.mw_bca_bwd_head_groups(B, H, n, T, d, sm_count=152)
+    assert got == _backward_plan(B, H, n, T, d, 152)
+    if expect is not None:
+        assert got == expect
+    # the modelled grouped launch never ends later than head by head
+    assert 1 <= got <= B * H
+
+
+def test_backward_head_groups_override_and_errors(mw):
+    lib = mw.library()
+    try:
+        assert lib.mw_set_option(b"bwd_group_heads", 5) == OK
+        assert mw.mw_bca_bwd_head_groups(2, 12, 16, 880, 64, sm_count=152) == 5   # ceil(24 / 5)
+        assert mw.mw_bca_bwd_head_groups(1, 16, 21, 880, 128, sm_count=152) == 16  # d > 80: head by head
+    finally:
+        lib.mw_set_option(b"bwd_group_heads", 0)
+    assert lib.mw_bca_bwd_head_groups(0, 1, 1, 1, 64, 152) == -1
+    assert lib.mw_bca_bwd_head_groups(1, 1, 0, 1, 64, 152) == -1
+    assert lib.mw_bca_bwd_head_groups(1, 1, 1, 1, 65, 152) == -1
+
+
 def test_python_binding_has_no_cpu_path(mw):
     q = torch.zeros(1, 1, 64, 64, dtype=torch.bfloat16)
     with pytest.raises(ValueError):
