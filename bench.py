@@ -748,7 +748,11 @@ def bench_rolling(mw, dev, peaks):
                    "the 64 steps replayed as one CUDA graph; separate_calls: forward and "
                    "commit as two API calls. The ring (57.7 MB) stays L2-resident across "
                    "steps, as in streaming"}
+    # the roofline fields at the top level are from the graph time; the same
+    # fields from the eager median sit under "eager"
     res.update(_cache_roofline(cfg, g_us, peaks))
+    res["roofline_time"] = "us_per_step_graph"
+    res["eager"] = {"us_per_step": round(med, 2), **_cache_roofline(cfg, med, peaks)}
     # the same stream through the RoPE re-shift entry point (32 rotated
     # channels; keys stored as rotated at their stream frames, two 440-token
     # frames per chunk, so each step's eviction moves the window by two
