@@ -3,35 +3,43 @@
 // (training is bf16 mixed precision, Sec. 4.1).
 //
 //   pre : D_i = <dO_i, O_i>, LSE2_i = LSE_i * log2(e) (+inf on padding rows),
-//         dQacc = 0
+//         dQacc = 0; at d = 64 also the bias rows (-LSE/scale and -D as tf32
+//         high and low parts) that the main kernel's MMAs add
 //   main: one CTA per 128-row key tile of one (b,h); it owns dK, dV in TMEM
 //         and visits only the query rows whose chunks can see it
 //         (queries i >= chunk(k0) * T), QN query rows per step j:
-//           S^T  = K Q^T                        (tcgen05 -> TMEM)
-//           dP^T = V dO^T                       (tcgen05 -> TMEM)
-//           P^T  = exp2(S^T scale log2e - LSE2) (registers)
-//           dS^T = P^T (dP^T - D)               (registers)
-//           P^T, dS^T (bf16) -> TMEM over the dP^T columns; dS^T -> smem
-//           dV += P^T dO ;  dK += dS^T Q        (tcgen05, A from TMEM)
+//           S^T  = K Q^T            (tcgen05 -> TMEM; d = 64: + the -LSE bias)
+//           dP^T = V dO^T           (tcgen05 -> TMEM; d = 64: + the -D bias)
+//           P^T  = exp2(scale log2e S^T - LSE2)     (registers)
+//           dS^T = P^T (dP^T - D)                   (registers)
+//           P^T (bf16) -> TMEM; dS^T (bf16) -> shared memory (d = 128: to
+//                 TMEM as well, beside P^T)
+//           dV += P^T dO            (tcgen05, A = P^T from TMEM)
+//           dK += dS^T Q            (d = 64: A from shared memory; d = 128:
+//                                    from TMEM)
 //           d = 64 : dQ_j = dS K    (query rows in TMEM lanes)
 //           d = 128: dQ_j^T = K^T dS^T (head-dim columns in TMEM lanes)
-//           dQacc += dQ_j  (fp32 reductions, each warp instruction covering
-//                           contiguous memory)
+//           dQacc += dQ_j  (fp32: TMA reduce-add of swizzled shared-memory
+//                           boxes at d = 64, red.global at d = 128)
 //   post: dQ = scale * dQacc -> bf16
 //
 // Software pipeline: the P/dS warps copy S^T and dP^T into registers and
 // release their TMEM columns at once, so S^T and dP^T of step j+1 are
 // computed while they work on step j; P^T is handed over before dS is
 // computed, so dV_j overlaps that math; dK, dQ of step j run while the P/dS
-// warps start step j+1.
+// warps start step j+1.  At d = 128 TMEM holds one block X for S^T, then
+// dP^T, then P^T / dS^T in turn, so those steps follow one another.
 //
 // Roles (512 threads): warps 0-7 P/dS (two warpgroups, one half of the query
 // columns each, one key row per thread), warps 8-11 dQ drain, warp 12 TMA
-// producer, warp 13 MMA issuer.
-// TMEM: dV [0,D), dK [D,2D), S^T [2D,2D+QN), dP^T [2D+QN,2D+2QN), dQ from
-// column 384 (D columns, or QN when transposed), P^T and dS^T (bf16 pairs) at PDS: d = 128 uses
-// [448,512); d = 64 uses [384,512), its P^T half shared with dQ (dQ_j is
-// written after dV_j has read P^T_j, and the next P^T waits for the drain).
+// producer, warp 13 MMA issuer (d = 64: warp 13 issues S^T, dV, dP^T and
+// warp 14 dK, dQ).
+// TMEM (512 columns): d = 64: dV [0,64), dK [64,128), S^T [128,256),
+// dP^T [256,384), P^T [384,448), dQ [448,512); d = 128: dV [0,128),
+// dK [128,256), X [256,384), dQ^T [384,512).
+// CTA order: head by head, or (where the host's model of the launch says it
+// ends sooner) in head groups whose key tiles run side by side, the first
+// (longest) ones first.
 #include "mw_internal.h"
 #include "mw_ptx.cuh"
 

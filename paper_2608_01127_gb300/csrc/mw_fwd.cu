@@ -12,10 +12,15 @@
 //   warp 8           TMA producer (Q once, then K/V tiles through a ring of stages)
 //   warp 9           tcgen05 issuer (S = Q K^T into TMEM, O += P V with P in TMEM)
 //   warps 10-11      RoPE re-shift of the sink anchor's key tiles in shared
-//                    memory when it is enabled (otherwise idle; they complete
-//                    warpgroup 2 for the register re-split)
+//                    memory when it is enabled; with 80-wide MMAs on the
+//                    128-wide tiles (and no re-shift) the ones columns of V;
+//                    otherwise idle (they complete warpgroup 2 for the
+//                    register re-split)
 // TMEM (512 columns): S_t at column 128 t (P_t, bf16, overwrites its first 64
-// columns), O_t at 256 + D t.
+// columns), O_t at 256 + OW t (OW = the MMA width, plus 16 columns where the
+// PV MMA also sums P through ones in V).
+// CTA order: groups of heads of about three waves of CTAs, one group after
+// another; in a group the longest query blocks first.
 #include <type_traits>
 
 #include "mw_internal.h"
