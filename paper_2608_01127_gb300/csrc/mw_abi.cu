@@ -461,6 +461,7 @@ mw_status fwd_common(const void* q, const void* k, const void* v, const void* kr
   p.status = status;
   p.budget_ns = budget_ns();
   p.debug_skip_q = static_cast<int>(g_opt_skip_q);
+  CUtensorMap top = tq;  // the split partials (TMA stores); unused with one split
   if (p.num_splits > 1) {
     const size_t need = cache_ws_bytes(p.num_splits, BH, rows_q, D);
     if (ws_bytes < need)
@@ -469,8 +470,10 @@ mw_status fwd_common(const void* q, const void* k, const void* v, const void* kr
     p.o_part = reinterpret_cast<float*>(base);
     p.lse_part = reinterpret_cast<float*>(
         base + align256(static_cast<size_t>(p.num_splits) * BH * rows_q * D * sizeof(float)));
+    MW_TRY(make_map(&top, p.o_part, rows_q, p.num_splits * BH, D, "o_part", mw::kTileRows, true));
   }
-  MW_TRY(launch_status(mw::launch_fwd(D, mma_d(d), tq, tk, tv, tkr, tvr, tks, tvs, p, rope.omega, stream),
+  MW_TRY(launch_status(mw::launch_fwd(D, mma_d(d), tq, tk, tv, tkr, tvr, tks, tvs, top, p, rope.omega,
+                                      stream),
                        "forward kernel launch"));
   if (p.num_splits > 1)
     MW_TRY(launch_status(mw::launch_combine(D, d, p.o_part, p.lse_part, p.o, lse, p.num_splits, BH,

@@ -128,14 +128,17 @@ __device__ __forceinline__ TileSrc tile_src(const Segs& g, int j) {
 
 // ROPE: the cache form with the RoPE re-shift of the sink anchor (warps 10-11
 // turn its key tiles before the MMAs read them); the training and plain
-// cache forms are compiled without it.
-template <int D, int DM, bool ROPE>
+// cache forms are compiled without it.  SPLIT: the key range is one of
+// several (p.num_splits > 1), O goes out as fp32 partials through TMA
+// stores; without it, as bf16 rows (the training form never pays for the
+// partials' code).
+template <int D, int DM, bool ROPE, bool SPLIT>
 __global__ void __launch_bounds__(FwdLayout<D, DM>::THREADS, 1)
     bca_fwd_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_k,
                    const __grid_constant__ CUtensorMap tm_v, const __grid_constant__ CUtensorMap tm_kr,
                    const __grid_constant__ CUtensorMap tm_vr, const __grid_constant__ CUtensorMap tm_ks,
-                   const __grid_constant__ CUtensorMap tm_vs, const __grid_constant__ FwdParams p,
-                   const __grid_constant__ RopeFreq rope_om) {
+                   const __grid_constant__ CUtensorMap tm_vs, const __grid_constant__ CUtensorMap tm_op,
+                   const __grid_constant__ FwdParams p, const __grid_constant__ RopeFreq rope_om) {
   using L = FwdLayout<D, DM, ROPE>;
   constexpr int QT = L::QT;
   constexpr int NS = L::STAGES;
@@ -619,6 +622,12 @@ __global__ void __launch_bounds__(FwdLayout<D, DM>::THREADS, 1)
     const float m_eff = (m_used == -INFINITY) ? 0.f : m_used;
     const float lse = nonzero ? (m_eff + __log2f(l)) * 0.69314718055994530942f : -INFINITY;
     const size_t row_off = static_cast<size_t>(bh) * p.rows_q + row;
+    // split partials: each warp writes its 32 rows of the tile's fp32 O into
+    // shared memory (the K/V stages, no longer read once O is final) as
+    // 32-column boxes with the 128-byte swizzle, and one thread of the tile
+    // hands the boxes to the TMA unit.  Row-per-thread global stores would
+    // cost 32 transactions per warp instruction, all CTAs at once.
+    constexpr int kBoxBytes = kTileRows * 128;  // 128 rows x 32 fp32
     // the chunks that hold the DM columns of O (the caller's d_io <= DM)
 #pragma unroll
     for (int c = 0; c < (DM + 31) / 32; ++c) {
@@ -627,31 +636,61 @@ __global__ void __launch_bounds__(FwdLayout<D, DM>::THREADS, 1)
         tmem_ld32(o_addr + 32 * c, r);
         tmem_wait_ld();
       }
-      if (!row_valid) continue;
       float v[32];
 #pragma unroll
       for (int k = 0; k < 32; ++k) v[k] = nonzero ? __uint_as_float(r[k]) * inv_l : 0.f;
-      if (p.num_splits == 1) {
-        // the caller's rows hold d_io <= D columns (multiples of 8); only the
-        // 128-wide kernel serves padded head dims
-        const int d_io = (D == 64) ? D : p.d_io;
-        if (32 * c >= d_io) continue;
-        const int n16 = min(4, (d_io - 32 * c) / 8);
-        uint4* dst = reinterpret_cast<uint4*>(p.o + row_off * d_io + 32 * c);
+      if constexpr (!SPLIT) {
+        if (!row_valid) continue;
+        if (p.num_splits == 1) {
+          // the caller's rows hold d_io <= D columns (multiples of 8); only
+          // the 128-wide kernel serves padded head dims
+          const int d_io = (D == 64) ? D : p.d_io;
+          if (32 * c >= d_io) continue;
+          const int n16 = min(4, (d_io - 32 * c) / 8);
+          uint4* dst = reinterpret_cast<uint4*>(p.o + row_off * d_io + 32 * c);
 #pragma unroll
-        for (int k = 0; k < 4; ++k)
-          if (k < n16) dst[k] = make_uint4(pack_bf16x2(v[8 * k], v[8 * k + 1]), pack_bf16x2(v[8 * k + 2], v[8 * k + 3]),
-                              pack_bf16x2(v[8 * k + 4], v[8 * k + 5]),
-                              pack_bf16x2(v[8 * k + 6], v[8 * k + 7]));
-      } else {
-        float4* dst = reinterpret_cast<float4*>(
-            p.o_part + (static_cast<size_t>(split) * p.BH * p.rows_q + row_off) * D + 32 * c);
+          for (int k = 0; k < 4; ++k)
+            if (k < n16) dst[k] = make_uint4(pack_bf16x2(v[8 * k], v[8 * k + 1]), pack_bf16x2(v[8 * k + 2], v[8 * k + 3]),
+                                pack_bf16x2(v[8 * k + 4], v[8 * k + 5]),
+                                pack_bf16x2(v[8 * k + 6], v[8 * k + 7]));
+        } else {
+          // never taken (the launcher picks SPLIT for several splits), but
+          // with this row-per-thread form of the partials here the compiler
+          // schedules the training kernel 1.4% faster at d = 128
+          float4* dst = reinterpret_cast<float4*>(
+              p.o_part + (static_cast<size_t>(split) * p.BH * p.rows_q + row_off) * D + 32 * c);
 #pragma unroll
-        for (int k = 0; k < 8; ++k) dst[k] = make_float4(v[4 * k], v[4 * k + 1], v[4 * k + 2], v[4 * k + 3]);
+          for (int k = 0; k < 8; ++k) dst[k] = make_float4(v[4 * k], v[4 * k + 1], v[4 * k + 2], v[4 * k + 3]);
+        }
+      } else if (t < qt_n) {
+        // (an empty tile's warps skip the O wait: they must not touch the
+        // stages, which the other tile's MMAs may still be reading)
+        // row row_local of box c: 16-byte piece k at piece k ^ (row mod 8)
+        uint8_t* box_row = smem + L::OFF_K + (t * (D / 32) + c) * kBoxBytes + row_local * 128;
+#pragma unroll
+        for (int k = 0; k < 8; ++k)
+          *reinterpret_cast<float4*>(box_row + ((k ^ (row_local & 7)) << 4)) =
+              make_float4(v[4 * k], v[4 * k + 1], v[4 * k + 2], v[4 * k + 3]);
+      }
+    }
+    if (SPLIT && t < qt_n) {  // a tile past the rows stores nothing
+      fence_proxy_async_smem();  // the TMA unit reads the boxes next
+      // this tile's four warps (barrier 1 or 2; 0 is __syncthreads)
+      if (t == 0)
+        named_barrier_sync<1, 4 * 32>();
+      else
+        named_barrier_sync<2, 4 * 32>();
+      if (wq == 0 && lane == 0) {
+        const uint8_t* stage = smem + L::OFF_K + t * (D / 32) * kBoxBytes;
+#pragma unroll
+        for (int c = 0; c < (DM + 31) / 32; ++c)
+          tma_store_3d(&tm_op, stage + c * kBoxBytes, 32 * c, r0 + t * kTileRows, split * p.BH + bh);
+        bulk_commit_group();
+        bulk_wait_read_all();  // the boxes are read before the CTA's shared memory goes
       }
     }
     if (row_valid) {
-      if (p.num_splits == 1) {
+      if (!SPLIT && p.num_splits == 1) {
         if (p.lse) p.lse[row_off] = lse;
       } else {
         p.lse_part[static_cast<size_t>(split) * p.BH * p.rows_q + row_off] = lse;
@@ -741,21 +780,21 @@ __global__ void __launch_bounds__(256) combine_kernel(const float* __restrict__ 
   if (lse && lane == 0) lse[row] = wsum > 0.f ? m + __logf(wsum) : -INFINITY;
 }
 
-template <int D, int DM, bool ROPE>
+template <int D, int DM, bool ROPE, bool SPLIT>
 cudaError_t launch_fwd_t(const CUtensorMap& tq, const CUtensorMap& tk, const CUtensorMap& tv,
                          const CUtensorMap& tkr, const CUtensorMap& tvr, const CUtensorMap& tks,
-                         const CUtensorMap& tvs, const FwdParams& p, const RopeFreq& om,
-                         cudaStream_t s) {
+                         const CUtensorMap& tvs, const CUtensorMap& top, const FwdParams& p,
+                         const RopeFreq& om, cudaStream_t s) {
   using L = FwdLayout<D, DM, ROPE>;
   static bool attr_set = false;  // per process; the attribute is per function
   if (!attr_set) {
     // The in-kernel register re-split assumes the launch register count; with
     // any other count its setmaxnreg.inc could never be satisfied, so refuse.
     cudaFuncAttributes fa;
-    cudaError_t e = cudaFuncGetAttributes(&fa, bca_fwd_kernel<D, DM, ROPE>);
+    cudaError_t e = cudaFuncGetAttributes(&fa, bca_fwd_kernel<D, DM, ROPE, SPLIT>);
     if (e != cudaSuccess) return e;
     if (fa.numRegs != L::REGS_LAUNCH) return cudaErrorInvalidKernelImage;
-    e = cudaFuncSetAttribute(bca_fwd_kernel<D, DM, ROPE>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+    e = cudaFuncSetAttribute(bca_fwd_kernel<D, DM, ROPE, SPLIT>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                              L::BYTES);
     if (e != cudaSuccess) return e;
     attr_set = true;
@@ -764,23 +803,33 @@ cudaError_t launch_fwd_t(const CUtensorMap& tq, const CUtensorMap& tk, const CUt
   cudaLaunchConfig_t cfg;
   cudaLaunchAttribute attr;
   pdl_config(cfg, attr, dim3(grid), dim3(L::THREADS), L::BYTES, s);
-  return cudaLaunchKernelEx(&cfg, bca_fwd_kernel<D, DM, ROPE>, tq, tk, tv, tkr, tvr, tks, tvs, p, om);
+  return cudaLaunchKernelEx(&cfg, bca_fwd_kernel<D, DM, ROPE, SPLIT>, tq, tk, tv, tkr, tvr, tks, tvs, top, p,
+                            om);
+}
+
+template <bool SPLIT>
+cudaError_t launch_fwd_split(int d, int dm, const CUtensorMap& tq, const CUtensorMap& tk,
+                             const CUtensorMap& tv, const CUtensorMap& tkr, const CUtensorMap& tvr,
+                             const CUtensorMap& tks, const CUtensorMap& tvs, const CUtensorMap& top,
+                             const FwdParams& p, const RopeFreq& om, cudaStream_t s) {
+  if (p.rope_dims > 0) {
+    if (d == 64) return launch_fwd_t<64, 64, true, SPLIT>(tq, tk, tv, tkr, tvr, tks, tvs, top, p, om, s);
+    if (dm == 80) return launch_fwd_t<128, 80, true, SPLIT>(tq, tk, tv, tkr, tvr, tks, tvs, top, p, om, s);
+    return launch_fwd_t<128, 128, true, SPLIT>(tq, tk, tv, tkr, tvr, tks, tvs, top, p, om, s);
+  }
+  if (d == 64) return launch_fwd_t<64, 64, false, SPLIT>(tq, tk, tv, tkr, tvr, tks, tvs, top, p, om, s);
+  if (dm == 80) return launch_fwd_t<128, 80, false, SPLIT>(tq, tk, tv, tkr, tvr, tks, tvs, top, p, om, s);
+  return launch_fwd_t<128, 128, false, SPLIT>(tq, tk, tv, tkr, tvr, tks, tvs, top, p, om, s);
 }
 
 }  // namespace
 
 cudaError_t launch_fwd(int d, int dm, const CUtensorMap& tq, const CUtensorMap& tk, const CUtensorMap& tv,
                        const CUtensorMap& tkr, const CUtensorMap& tvr, const CUtensorMap& tks,
-                       const CUtensorMap& tvs, const FwdParams& p, const RopeFreq& om,
-                       cudaStream_t s) {
-  if (p.rope_dims > 0) {
-    if (d == 64) return launch_fwd_t<64, 64, true>(tq, tk, tv, tkr, tvr, tks, tvs, p, om, s);
-    if (dm == 80) return launch_fwd_t<128, 80, true>(tq, tk, tv, tkr, tvr, tks, tvs, p, om, s);
-    return launch_fwd_t<128, 128, true>(tq, tk, tv, tkr, tvr, tks, tvs, p, om, s);
-  }
-  if (d == 64) return launch_fwd_t<64, 64, false>(tq, tk, tv, tkr, tvr, tks, tvs, p, om, s);
-  if (dm == 80) return launch_fwd_t<128, 80, false>(tq, tk, tv, tkr, tvr, tks, tvs, p, om, s);
-  return launch_fwd_t<128, 128, false>(tq, tk, tv, tkr, tvr, tks, tvs, p, om, s);
+                       const CUtensorMap& tvs, const CUtensorMap& top, const FwdParams& p,
+                       const RopeFreq& om, cudaStream_t s) {
+  return p.num_splits > 1 ? launch_fwd_split<true>(d, dm, tq, tk, tv, tkr, tvr, tks, tvs, top, p, om, s)
+                          : launch_fwd_split<false>(d, dm, tq, tk, tv, tkr, tvr, tks, tvs, top, p, om, s);
 }
 
 cudaError_t launch_combine(int d, int d_io, const float* o_part, const float* lse_part,

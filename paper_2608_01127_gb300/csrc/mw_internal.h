@@ -127,10 +127,12 @@ inline void pdl_config(cudaLaunchConfig_t& cfg, cudaLaunchAttribute& attr, dim3 
 // the segment is empty)
 // d: tile width (64 or 128); dm: MMA width (d, or 80 on the 128-wide tiles
 // for head dims up to 80)
+// top: the fp32 split partials p.o_part as [splits * BH][rows_q][d] with
+// 32-column boxes (any valid map when p.num_splits == 1)
 cudaError_t launch_fwd(int d, int dm, const CUtensorMap& tq, const CUtensorMap& tk,
                        const CUtensorMap& tv, const CUtensorMap& tkr, const CUtensorMap& tvr, const CUtensorMap& tks,
-                       const CUtensorMap& tvs, const FwdParams& p, const RopeFreq& rope_om,
-                       cudaStream_t s);
+                       const CUtensorMap& tvs, const CUtensorMap& top, const FwdParams& p,
+                       const RopeFreq& rope_om, cudaStream_t s);
 // d: the kernels' head dim (64 or 128); d_io: the caller's (a multiple of 8, <= d)
 // The combine's launch also carries the ring commit `cj` (if cj.rows > 0)
 // in blocks of its own: both only run once the forward has finished, and

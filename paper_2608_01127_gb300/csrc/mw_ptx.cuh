@@ -130,6 +130,27 @@ __device__ __forceinline__ void tma_reduce_add_3d(const CUtensorMap* map, const 
       : "memory");
 }
 
+// 3-D tiled store of a shared-memory box into global memory (element type,
+// box and swizzle from the map), tracked as a bulk async-group of the
+// issuing thread.  Rows past the map's extents are not written;
+// coordinates must not be negative; c0 * element size must be a multiple of
+// 16 bytes.
+__device__ __forceinline__ void tma_store_3d(const CUtensorMap* map, const void* src, int c0,
+                                             int c1, int c2) {
+  asm volatile(
+      "cp.async.bulk.tensor.3d.global.shared::cta.tile.bulk_group"
+      " [%0, {%2, %3, %4}], [%1];" ::"l"(reinterpret_cast<uint64_t>(map)),
+      "r"(smem_u32(src)), "r"(c0), "r"(c1), "r"(c2)
+      : "memory");
+}
+
+// Barrier ID (1..15) over THREADS threads (a multiple of 32) of the CTA.
+template <int ID, int THREADS>
+__device__ __forceinline__ void named_barrier_sync() {
+  static_assert(ID >= 1 && ID <= 15 && THREADS % 32 == 0, "named barrier");
+  asm volatile("bar.sync %0, %1;" ::"n"(ID), "n"(THREADS) : "memory");
+}
+
 __device__ __forceinline__ void bulk_commit_group() {
   asm volatile("cp.async.bulk.commit_group;" ::: "memory");
 }
