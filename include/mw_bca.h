@@ -83,7 +83,8 @@ size_t mw_bca_bwd_workspace_size(int B, int H, int n_chunks, int T_chunk, int d)
  * The heads form groups of nearly equal size, and in a group the key tiles
  * of all its heads run side by side, the first (longest) ones first.  The
  * groups are taken where a list-scheduling model of the launch ends at least
- * 1% before head by head; head dims over 80 always run head by head; the
+ * 1% before head by head (launches of up to 2^18 CTAs; larger ones and head
+ * dims over 80 always run head by head); the
  * option "bwd_group_heads" overrides the choice.  Returns -1 on invalid
  * sizes (mw_last_error says why).
  */

@@ -299,12 +299,15 @@ int bwd_head_groups(int BH, int N_pad, int T, int qrows, int d_io, int D, int sm
       (2 * longest * sms + per_head - 1) / per_head));
   int groups = BH;  // head by head
   const int candidate = ceil_div(BH, per_group);
-  if (candidate < BH) {
+  // (past ~256K CTAs the model's host time passes a few ms, and with that
+  // many the tail of head-by-head order is a small share of the launch)
+  if (candidate < BH && static_cast<long long>(BH) * n_kt <= (1LL << 18)) {
     const long long t_heads = list_makespan(bwd_order_work(kt_work, BH, BH), sms);
     const long long t_groups = list_makespan(bwd_order_work(kt_work, BH, candidate), sms);
     if (100 * t_groups <= 99 * t_heads) groups = candidate;
   }
   std::lock_guard<std::mutex> lock(mu);
+  if (cache.size() >= 4096) cache.clear();  // bounded for callers that vary the sizes
   cache.emplace(key, groups);
   return groups;
 }

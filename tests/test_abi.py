@@ -256,7 +256,8 @@ def _backward_plan(B, H, n, T, d, sms):
         base, rem = divmod(BH, groups)
         return [w for g in range(groups) for w in kt_len for _ in range(base + (g < rem))]
 
-    if cand < BH and 100 * _makespan(order(cand), sms) <= 99 * _makespan(order(BH), sms):
+    if cand < BH and BH * len(kt_len) <= 1 << 18 and \
+            100 * _makespan(order(cand), sms) <= 99 * _makespan(order(BH), sms):
         return cand
     return BH
 
@@ -269,6 +270,7 @@ def _backward_plan(B, H, n, T, d, sms):
     (1, 12, 32, 600, 96, 12),
     (1, 1, 4, 64, 64, 1),
     (8, 16, 2, 256, 64, None),   # short sequences, many heads: whatever the model says
+    (64, 32, 16, 880, 64, 2048),  # 2^19 CTAs: past the model's limit, head by head
 ])
 def test_backward_head_groups_follow_the_list_scheduling_rule(mw, B, H, n, T, d, expect):
     got = mw.mw_bca_bwd_head_groups(B, H, n, T, d, sm_count=152)
