@@ -214,6 +214,35 @@ def test_backward_head_groups_of_unequal_size(mw):
     assert mw.mw_device_status() == 0
 
 
+@pytest.mark.parametrize("d", [64, 72])
+def test_backward_cta_order_does_not_change_the_gradients(mw, d):
+    """The backward's CTA order (head by head, or head groups of any size)
+    only changes when each key tile runs: dK and dV (each key tile's own)
+    come out bit for bit the same, and dQ (fp32 sums in another order)
+    within rounding."""
+    B, H, n, T = 1, 5, 6, 256
+    q, k, v, do = _inputs(B, H, n, T, d, seed=71)
+    sc = 1.0 / math.sqrt(d)
+    qc, kc, vc, doc = (t.cuda() for t in (q, k, v, do))
+    o, lse = mw.mw_bca_fwd(qc, kc, vc, T, sc)
+    results = []
+    try:
+        for g in (1, 2, 3, 5):
+            mw.mw_set_option("bwd_group_heads", g)
+            results.append(mw.mw_bca_bwd(qc, kc, vc, o, lse, doc, T, sc))
+    finally:
+        mw.mw_set_option("bwd_group_heads", 0)
+    dq0, dk0, dv0 = results[0]
+    for dq, dk, dv in results[1:]:
+        assert torch.equal(dk, dk0) and torch.equal(dv, dv0)
+        assert float((dq.float() - dq0.float()).norm() / dq0.float().norm()) < 1e-3
+    dq_r, dk_r, dv_r = oracle.bwd(q, k, v, do, T, sc)
+    check_grad(dk0, dk_r, "dK")
+    check_grad(dv0, dv_r, "dV")
+    check_grad(dq0, dq_r, "dQ")
+    assert mw.mw_device_status() == 0
+
+
 def test_forward_is_deterministic_and_stays_in_bounds(mw):
     B, H, n, T, d = 1, 2, 3, 100, 64
     q, k, v, _ = _inputs(B, H, n, T, d, seed=7)
